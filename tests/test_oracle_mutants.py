@@ -1,0 +1,63 @@
+"""Plant one plausible mistake at a time in a private copy of the oracle's C
+source (on the CPU) and check that at least one pin catches it.  This shows
+the pins constrain every index, sign and term of the oracle's arithmetic."""
+import os
+
+import pytest
+
+import oracle
+import pins
+
+SRC = open(oracle.SOURCE).read()
+
+MUTANTS = {
+    "ky_kx_swapped_in_position": (
+        "const int ix = ox * stride - pad + kx;", "const int ix = ox * stride - pad + ky;"),
+    "kernel_offset_order_transposed": (
+        "const int pk = ky * kw + kx;", "const int pk = kx * kh + ky;"),
+    "padding_sign_flipped": (
+        "const int ix = ox * stride - pad + kx;", "const int ix = ox * stride + pad + kx;"),
+    "stride_dropped": (
+        "const int ix = ox * stride - pad + kx;", "const int ix = ox - pad + kx;"),
+    "subspaces_interleaved": (
+        "acc += s[(i64)(m * Csp + j) * s_stride] * dk[j];",
+        "acc += s[(i64)(j * M + m) * s_stride] * dk[j];"),
+    "codebook_transposed": (
+        "acc += s[(i64)(m * Csp + j) * s_stride] * dk[j];",
+        "acc += s[(i64)(m * Csp + j) * s_stride] * D[((i64)m * Csp + j) * K + k];"),
+    "fc_codes_transposed": (
+        "t += lut[(i64)m * K + codes[(i64)m * Ct + ct]];",
+        "t += lut[(i64)m * K + codes[(i64)ct * M + m]];"),
+    "conv_codes_layout_wrong": (
+        "const int k = codes[((i64)ct * KK + pk) * M + m];",
+        "const int k = codes[((i64)ct * M + m) * KK + pk];"),
+    "codeword_order_reversed": (
+        "t += lut[((i64)m * P + ps) * K + k];", "t += lut[((i64)m * P + ps) * K + (K - 1 - k)];"),
+    "last_subspace_dropped": (
+        "for (int m = 0; m < M; ++m) {\n                                const int k",
+        "for (int m = 0; m < M - 1; ++m) {\n                                const int k"),
+    "fc_bias_dropped": (
+        "            if (bias) t += bias[ct];\n            if (relu",
+        "            if (relu"),
+    "conv_relu_before_bias": (
+        "                    if (bias) t += bias[ct];\n                    if (relu && t < 0.0) t = 0.0;",
+        "                    if (relu && t < 0.0) t = 0.0;\n                    if (bias) t += bias[ct];"),
+    "first_input_row_skipped": (
+        "if (iy < 0 || iy >= H) continue;", "if (iy <= 0 || iy >= H) continue;"),
+    "pool_window_short": (
+        "for (int dy = 0; dy < k; ++dy)", "for (int dy = 0; dy < k - 1; ++dy)"),
+    "lut_dot_product_drops_last_dim": (
+        "for (int j = 0; j < Csp; ++j)\n                acc +=",
+        "for (int j = 0; j < Csp - 1; ++j)\n                acc +="),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    assert SRC.count(old) == 1, f"mutation site for {name} not unique in the source"
+    src = tmp_path / "mutant.c"
+    src.write_text(SRC.replace(old, new))
+    so = oracle.compile_c(str(src), str(tmp_path / "libmutant.so"))
+    fails = pins.run_all(oracle.Oracle(so))
+    assert fails, f"no pin caught the planted mistake {name!r}"
