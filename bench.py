@@ -1,0 +1,421 @@
+#!/usr/bin/env python
+"""Throughput of the Q-CNN test-phase forward on GB300.
+
+Workload: AlexNet-shaped (ungrouped, CaffeNet-style) Q-CNN, batch 128 per GPU:
+conv1 11x11/4 (C's=3, K=128), conv2 5x5 p2, conv3-5 3x3 p1 (C's=4, K=128),
+3x3/2 max-pools, fc6-8 (C's=4, K=32); seeded synthetic images and
+random-initialised codebooks/codes/biases (synth.alexnet()).  A step is one
+forward of one batch through qcnn_net_forward (every layer, every stage).
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the float64 CPU
+oracle on the same workload instead (the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = ("Q-CNN layer/net images/sec and dense-equiv GFLOP/s at batch 1/128; "
+          "% of per-stage roofline")
+WORKLOAD = "alexnet_qcnn"
+BATCH = 128
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=30)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["qcnn", "reference"], default="qcnn")
+    p.add_argument("--batch", type=int, default=BATCH)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-sample", type=int, default=0,
+                   help="images in the CPU-baseline sample (default: one per worker)")
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------- oracle
+def _oracle_worker(args):
+    """Run the float64 oracle on image `i` of the workload (spawned process)."""
+    i, batch = args
+    sys.path.insert(0, ROOT)
+    import oracle as orc
+    w = synth.WORKLOADS[WORKLOAD]
+    params = w.params()
+    layers = [synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, params)]
+    x = w.input(batch)[i:i + 1]
+    t = time.perf_counter()
+    orc.net_forward(x, layers)
+    return time.perf_counter() - t
+
+
+def _cpu_info():
+    model = ""
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part", "hardware")):
+                model = line.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    return model
+
+
+def oracle_pool(cores):
+    import oracle as orc
+    orc.build()
+    ctx = mp.get_context("spawn")
+    pool = ctx.Pool(cores)
+    pool.map(_oracle_ping, range(cores))
+    return pool
+
+
+def _oracle_ping(_):
+    sys.path.insert(0, ROOT)
+    import oracle as orc  # noqa: F401
+    orc.default()
+    return 0
+
+
+def time_oracle(pool, cores, sample, batch):
+    """Wall time of `sample` images through the oracle on `cores` processes."""
+    t = time.perf_counter()
+    pool.map(_oracle_worker, [(i % batch, batch) for i in range(sample)])
+    return time.perf_counter() - t
+
+
+def reference_arm(a):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    cores = min(os.cpu_count() or 1, 16)
+    pool = oracle_pool(cores)
+    sample = cores
+    for _ in range(a.warmup):
+        time_oracle(pool, cores, sample, a.batch)
+    tot = 0.0
+    for _ in range(a.steps):
+        tot += time_oracle(pool, cores, sample, a.batch)
+    pool.close()
+    value = sample * a.steps / tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",
+        "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
+        "ms_per_step": 1e3 * tot / a.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "global_batch": a.batch, "images_per_step": sample},
+        "cpu_baseline": {"value": value, "unit": "images/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{sample} images of the batch-{a.batch} workload per step, "
+                                   f"one image per process, {cores} spawned processes, "
+                                   f"float64 C oracle, host {_cpu_info()}"},
+        "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.6)
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.perf_counter(), line.strip()))
+
+    def mark(self):
+        return time.perf_counter()
+
+    def stop(self, t0, t1):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for t, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) != 7:
+                continue
+            try:
+                rows.append((t, float(parts[0]), float(parts[1]), parts[3:]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 - 0.06 <= r[0] <= t1 + 0.06] or rows
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])),
+                "sm_max_mhz": max(r[2] for r in inside), "reasons": reasons,
+                "samples": len(inside)}
+
+
+# -------------------------------------------------------------- our arm
+def load_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        return {}
+
+
+def main():
+    a = parse()
+    if a.impl == "reference":
+        return reference_arm(a)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    # The CPU-baseline pool is spawned before the first GPU call.
+    pool = None
+    cores = min(os.cpu_count() or 1, 16)
+    if rank == 0 and world == 1 and not a.no_cpu_baseline:
+        pool = oracle_pool(cores)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_1512_06473_gb300 as q
+    from paper_1512_06473_gb300 import costmodel as cm
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = synth.WORKLOADS[WORKLOAD]
+    N = a.batch
+    params = w.params()
+    x_host = torch.from_numpy(w.input(N, rank)).pin_memory()
+    x = x_host.to(dev)
+
+    # model load: codes re-laid out once, outside the timed region
+    layers, shapes = [], w.shapes()
+    for L, P in zip(w.layers, params):
+        if isinstance(L, synth.Conv):
+            codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
+            layers.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
+                                      torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
+                                      L.stride, L.pad, L.relu, packed=True))
+        elif isinstance(L, synth.FC):
+            layers.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
+                                    torch.from_numpy(P["codes"]).to(dev),
+                                    torch.from_numpy(P["bias"]).to(dev), L.relu))
+        else:
+            layers.append(q.PoolLayer(L.k, L.s))
+    net = q.Net(layers, tuple(w.in_shape))
+    ws = net.alloc_workspace(N, dev)
+    out = net._out(N, dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        net.forward(x, out=out, workspace=ws)
+
+    for _ in range(max(a.warmup, 3)):
+        step()
+    torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    l0 = q.launch_count()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t0 = clocks.mark()
+    for i in range(a.steps):
+        flush.zero_()
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    t1 = clocks.mark()
+    if world > 1:
+        dist.barrier()
+    launches = q.launch_count() - l0
+    clk = clocks.stop(t0, t1)
+    ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / a.steps
+    value = N * world * a.steps / (ms / 1e3)
+
+    # ---- per-stage timing: the same layers launched one by one, events between
+    conv_costs, per_layer = [], []
+    hshape = tuple(w.in_shape)
+    bufs = []
+    h = x
+    for L, qL, (sin, sout) in zip(w.layers, layers, shapes):
+        o = torch.empty((N, *sout), dtype=torch.float32, device=dev)
+        bufs.append(o)
+    stage_ms = [0.0] * len(layers)
+    lws = torch.empty(ws.numel(), dtype=torch.uint8, device=dev)
+    for it in range(a.steps + 2):
+        flush.zero_()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(layers) + 1)]
+        ev[0].record(stream)
+        h = x
+        for j, (L, qL) in enumerate(zip(w.layers, layers)):
+            o = bufs[j]
+            if isinstance(qL, q.ConvLayer):
+                q.conv_forward(h, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias,
+                               qL.relu, packed=True, Ct=qL.Ct, out=o, workspace=lws)
+            elif isinstance(qL, q.FCLayer):
+                q.fc_forward(h.reshape(N, -1), qL.D, qL.codes, qL.bias, qL.relu, out=o.reshape(N, -1),
+                             workspace=lws)
+            else:
+                q.maxpool(h, qL.k, qL.s, out=o)
+            ev[j + 1].record(stream)
+            h = o
+        torch.cuda.synchronize(dev)
+        if it >= 2:
+            for j in range(len(layers)):
+                stage_ms[j] += ev[j].elapsed_time(ev[j + 1])
+    stage_ms = [s / a.steps for s in stage_ms]
+
+    peaks = load_peaks()
+    sm_max = float(peaks.get("sm_max_mhz") or 2070.0)
+    nsm = torch.cuda.get_device_properties(dev).multi_processor_count
+    smem_peak_gbs = nsm * 128 * sm_max * 1e6 / 1e9
+    stages = []
+    dense_macs = 0.0
+    for j, (L, (sin, sout)) in enumerate(zip(w.layers, shapes)):
+        if isinstance(L, synth.Conv):
+            c = cm.conv_cost(L.Cs, L.Ct, sin[1], sin[2], L.kh, L.kw, sout[1], sout[2], L.Csp, L.K)
+        elif isinstance(L, synth.FC):
+            c = cm.fc_cost(L.Cs, L.Ct, L.Csp, L.K)
+        else:
+            stages.append({"layer": j, "kind": "maxpool", "ms": round(stage_ms[j], 4)})
+            continue
+        dense_macs += c.dense_macs
+        alg_bytes = 4.0 * (c.lookups + c.lut_entries) * N
+        ach = alg_bytes / (stage_ms[j] / 1e3) / 1e9
+        stages.append({"layer": j, "kind": L.kind, "ms": round(stage_ms[j], 4),
+                       "lookups": c.lookups * N, "lut_entries": c.lut_entries * N,
+                       "smem_alg_GBs": round(ach, 1), "frac_smem": round(ach / smem_peak_gbs, 4)})
+    dom = max((s for s in stages if s["kind"] != "maxpool"), key=lambda s: s["ms"])
+    dom_alg = 4.0 * (dom["lookups"] + dom["lut_entries"])
+    roofline = {
+        "bound": "smem", "kernel": f"layer {dom['layer']} ({dom['kind']})",
+        "achieved": round(dom_alg / (dom["ms"] / 1e3) / 1e9, 1),
+        "peak": round(smem_peak_gbs, 1), "unit": "GB/s",
+        "frac": round(dom_alg / (dom["ms"] / 1e3) / 1e9 / smem_peak_gbs, 4),
+        "traffic": None,
+        "peak_basis": f"{nsm} SMs x 128 B/clk shared-memory loads x {sm_max:.0f} MHz max SM clock",
+        "alg_bytes_per_launch": dom_alg,
+    }
+
+    # ---- end to end through qcnn_net_forward_host (pinned host buffers)
+    ws_h = net.alloc_workspace(N, dev, host_io=True)
+    y_host = torch.empty(tuple(out.shape), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        net.forward_host(x_host, y_host, ws_h)
+    e2e_t = 0.0
+    for _ in range(a.steps):
+        flush.zero_()
+        torch.cuda.synchronize(dev)
+        t = time.perf_counter()
+        net.forward_host(x_host, y_host, ws_h)
+        e2e_t += time.perf_counter() - t
+    if world > 1:
+        t = torch.tensor([e2e_t], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_t = float(t.item())
+    e2e = {"value": N * world * a.steps / e2e_t, "unit": "images/s",
+           "h2d_bytes_per_step": x_host.numel() * 4, "d2h_bytes_per_step": y_host.numel() * 4}
+
+    # ---- batch 1 latency (plain launches)
+    x1 = x[:1].contiguous()
+    ws1 = net.alloc_workspace(1, dev)
+    o1 = net._out(1, dev)
+    for _ in range(5):
+        net.forward(x1, out=o1, workspace=ws1)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    lat = []
+    for _ in range(20):
+        flush.zero_()
+        e0.record(stream)
+        net.forward(x1, out=o1, workspace=ws1)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        lat.append(e0.elapsed_time(e1))
+    b1_ms = float(np.median(lat))
+
+    cpu = None
+    if pool is not None:
+        sample = a.cpu_sample or cores
+        dt = time_oracle(pool, cores, sample, N)
+        pool.close()
+        cpu = {"value": sample / dt, "unit": "images/s", "cores": cores, "kind": "oracle",
+               "sample": f"{sample} images of the batch-{N} workload, one per spawned process, "
+                         f"float64 C oracle, host {_cpu_info()}, {dt:.1f} s wall"}
+
+    if world > 1:
+        dist.destroy_process_group()
+    if rank != 0:
+        return 0
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "images/s", "n_gpus": world,
+        "steps": a.steps, "warmup": a.warmup, "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded images, random-init codebooks/codes/biases)",
+        "config": {"workload": WORKLOAD, "global_batch": N * world, "per_gpu_batch": N,
+                   "image": "3x227x227", "parallelism": f"replicas x{world}",
+                   "l2": "flushed (256 MB write) before every timed step",
+                   "codes": "packed once at model load (outside the timed region)"},
+        "dense_equiv_gflops": round(2 * dense_macs * value / 1e9, 1),
+        "batch1": {"latency_ms": round(b1_ms, 4), "images_per_s": round(1e3 / b1_ms, 1)},
+        "roofline": roofline, "stages": stages,
+        "cpu_baseline": cpu, "e2e": {k: (round(v, 1) if isinstance(v, float) else v)
+                                     for k, v in e2e.items()},
+        "gpu_launches": int(launches), "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,208 @@
+/*
+ * qcnn.h -- C ABI of libqcnn, the GB300 (sm_103a) implementation of the
+ * test-phase response of product-quantized (PQ) layers from
+ *   J. Wu, C. Leng, Y. Wang, Q. Hu, J. Cheng, "Quantized Convolutional Neural
+ *   Networks for Mobile Devices", arXiv 1512.06473 (Q-CNN).
+ *
+ * The method (Sec. 3.1-3.2): split the C_s input channels into M contiguous
+ * sub-spaces of C'_s channels (Csp); for every input vector S^(m) and every
+ * sub-codeword D^(m)_k compute the table entry <S^(m), D^(m)_k>; then every
+ * output is a sum of table entries selected by stored uint8 indices
+ * k_m(c_t) (FC, Eq. 5) or k_m(c_t, p_k) (conv, Eq. 7), plus a bias.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Tensors are caller-owned DEVICE pointers (cudaMalloc / torch memory),
+ *    fp32 unless stated, dense and row-major in the order written in each
+ *    comment ("[N][C][H][W]" = NCHW).  The only host pointers are the layer
+ *    array of qcnn_net_* and the x/y buffers of qcnn_net_forward_host.
+ *  - Sub-codebooks: D[m][k][j], m < M = Cs / Csp, k < K, j < Csp
+ *    (the k-th column of D^(m) in the paper is row k here).
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
+ *    call only enqueues work on it and returns; results are ready when the
+ *    stream reaches that point.  Exception: qcnn_net_forward_host, which
+ *    synchronizes the stream before returning.
+ *  - Scratch memory comes from a caller-provided device workspace whose size
+ *    is given by the matching *_workspace_size query.  No call allocates or
+ *    frees device memory.  The workspace may be reused by the next call on
+ *    the same stream; calls that run concurrently need separate workspaces.
+ *  - Limits: 1 <= Csp <= 8, 1 <= K <= 256, Cs % Csp == 0, every size > 0 and
+ *    every element count below 2^31.  Outside them: QCNN_ERR_INVALID_ARG,
+ *    returned before any work is enqueued.
+ *  - Codes >= K are a caller error.  Kernels clamp every index into [0, K),
+ *    so such codes never cause an out-of-bounds access, but the outputs are
+ *    then unspecified.
+ *  - A failed launch returns QCNN_ERR_CUDA; the CUDA error is in
+ *    qcnn_last_cuda_error().  The library is stateless apart from that
+ *    value and a launch counter, and is safe to call from several threads.
+ */
+#ifndef QCNN_H
+#define QCNN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    QCNN_OK = 0,
+    QCNN_ERR_INVALID_ARG = 1, /* bad size, null pointer, limit exceeded     */
+    QCNN_ERR_UNSUPPORTED = 2, /* valid request this build cannot serve      */
+    QCNN_ERR_WORKSPACE = 3,   /* workspace smaller than the query asked for */
+    QCNN_ERR_CUDA = 4         /* a CUDA call or kernel launch failed        */
+} qcnn_status;
+
+typedef enum {
+    QCNN_ALGO_AUTO = 0,    /* library picks (fused whenever it applies)       */
+    QCNN_ALGO_FUSED = 1,   /* table tile built in shared memory, stride 1 only */
+    QCNN_ALGO_UNFUSED = 2  /* tables materialised in the workspace first      */
+} qcnn_algo;
+
+typedef enum {
+    QCNN_CODES_CANONICAL = 0, /* conv codes [Ct][kh*kw][M]                   */
+    QCNN_CODES_PACKED = 1     /* output of qcnn_conv_pack_codes              */
+} qcnn_codes_layout;
+
+/* Human-readable name of a status value (static string, never NULL). */
+const char *qcnn_status_string(qcnn_status s);
+
+/* The last CUDA error code seen by a failing call in this process (0 if none). */
+int qcnn_last_cuda_error(void);
+
+/* Number of kernels this library has launched in this process so far. */
+uint64_t qcnn_launch_count(void);
+
+/*
+ * qcnn_lut_build -- the look-up tables alone (Sec. 3.1, the paragraph after
+ * Eq. 5; Sec. 3.2, the paragraph after Eq. 7):
+ *     lut[n][m][p][k] = sum_{j < Csp} x[n][m*Csp + j][p] * D[m][k][j]
+ * for every input position p = y*W + x (H = W = 1 for an FC input).
+ *   x    [N][Cs][H][W]   fp32, device
+ *   D    [M][K][Csp]     fp32, device
+ *   lut  [N][M][H*W][K]  fp32, device, written
+ */
+qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W,
+                           const float *D, int Csp, int K, float *lut,
+                           void *stream);
+
+/*
+ * qcnn_fc_forward -- PQ fully-connected layer, Eq. 5:
+ *     y[n][ct] = bias[ct] + sum_{m < M} lut_n[m][codes[m][ct]]    (then ReLU if relu)
+ * with lut_n the tables of x[n].  Tables are built tile by tile in shared
+ * memory and never written to device memory.
+ *   x      [N][Cs]   fp32       D [M][K][Csp] fp32
+ *   codes  [M][Ct]   uint8      bias [Ct] fp32, or NULL for none
+ *   y      [N][Ct]   fp32, written
+ *   workspace: at least qcnn_fc_workspace_size(...) bytes, 256-byte aligned
+ *   (may be NULL when that size is 0).
+ */
+qcnn_status qcnn_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K,
+                                   size_t *bytes);
+qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
+                            const float *D, int Csp, int K,
+                            const uint8_t *codes, const float *bias, float *y,
+                            int relu, void *workspace, size_t workspace_bytes,
+                            void *stream);
+
+/*
+ * qcnn_conv_pack_codes -- re-layout conv codes once, at model-load time,
+ * for the fused kernels: packed[m][pk][ct] (ct padded with code 0 to a
+ * multiple of 256), every code clamped into [0, K).
+ *   codes  [Ct][kh*kw][M] uint8, device;  packed: qcnn_conv_packed_codes_bytes
+ */
+size_t qcnn_conv_packed_codes_bytes(int Ct, int kh, int kw, int M);
+qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw,
+                                 int M, int K, uint8_t *packed, void *stream);
+
+/*
+ * qcnn_conv_forward -- PQ convolutional layer, Eq. 7:
+ *     y[n][ct][oy][ox] = bias[ct] + sum_{ky<kh, kx<kw} sum_{m<M}
+ *                        lut_n[m][iy*W + ix][codes[ct][ky*kw + kx][m]]
+ * with iy = oy*stride - pad + ky, ix = ox*stride - pad + kx; a position
+ * outside the map contributes 0 (zero padding); then ReLU if relu.
+ * Output size Ho = (H + 2 pad - kh) / stride + 1 (floor), same for Wo.
+ *   x      [N][Cs][H][W]   fp32         D [M][K][Csp] fp32
+ *   codes  [Ct][kh*kw][M]  uint8 (codes_layout CANONICAL) or the output of
+ *          qcnn_conv_pack_codes (PACKED)
+ *   bias   [Ct] or NULL;   y [N][Ct][Ho][Wo] fp32, written
+ *   algo:  QCNN_ALGO_FUSED needs stride 1, else QCNN_ERR_UNSUPPORTED.
+ *   workspace: at least qcnn_conv_workspace_size(...) bytes, 256-byte aligned.
+ */
+qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct,
+                                     int kh, int kw, int stride, int pad,
+                                     int Csp, int K, int codes_layout,
+                                     int algo, size_t *bytes);
+qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W,
+                              int Ct, int kh, int kw, int stride, int pad,
+                              const float *D, int Csp, int K,
+                              const uint8_t *codes, int codes_layout,
+                              const float *bias, float *y, int relu, int algo,
+                              void *workspace, size_t workspace_bytes,
+                              void *stream);
+
+/*
+ * qcnn_maxpool -- k x k max-pool, stride s, no padding, floor output size
+ * (the pooling between the layers of the whole-network experiments,
+ * Sec. 4.2.3).  x [N][C][H][W] -> y [N][C][Ho][Wo], Ho = (H - k) / s + 1.
+ */
+qcnn_status qcnn_maxpool(const float *x, int N, int C, int H, int W, int k,
+                         int s, float *y, void *stream);
+
+/*
+ * Whole network: a stack of PQ conv / PQ FC / max-pool layers (Sec. 4.2.3,
+ * Table 8).  An FC layer that follows a conv or pool layer reads its input
+ * flattened in C*H*W order.  The input channel count of each layer is the
+ * output channel count of the layer before it.
+ */
+typedef enum { QCNN_LAYER_CONV = 0, QCNN_LAYER_FC = 1, QCNN_LAYER_MAXPOOL = 2 } qcnn_layer_kind;
+
+typedef struct {
+    int kind;           /* qcnn_layer_kind                                   */
+    int Ct;             /* CONV / FC: output channels                        */
+    int kh, kw;         /* CONV: kernel size; MAXPOOL: window (kh == kw)     */
+    int stride, pad;    /* CONV: stride, zero padding; MAXPOOL: stride       */
+    int Csp, K;         /* CONV / FC: sub-space dimension, sub-codewords     */
+    int relu;           /* CONV / FC: 1 = ReLU after the bias                */
+    int algo;           /* CONV: qcnn_algo                                   */
+    int codes_layout;   /* CONV: qcnn_codes_layout of `codes`                */
+    const float *D;     /* CONV / FC: [M][K][Csp], device                    */
+    const uint8_t *codes; /* CONV: see qcnn_conv_forward; FC: [M][Ct]; device */
+    const float *bias;  /* [Ct] or NULL, device                              */
+} qcnn_layer;
+
+/* Output shape of the stack for one image (C, H, W; H = W = 1 after an FC). */
+qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers,
+                                  int C, int H, int W, int *out_C, int *out_H,
+                                  int *out_W);
+
+/*
+ * qcnn_net_workspace_size: bytes of workspace for qcnn_net_forward
+ * (host_io = 0) or qcnn_net_forward_host (host_io = 1, which also stages
+ * the input and output in the workspace).
+ */
+qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers,
+                                    int N, int C, int H, int W, int host_io,
+                                    size_t *bytes);
+
+/* x [N][C][H][W] device -> y [N][out_C][out_H][out_W] device. */
+qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers,
+                             const float *x, int N, int C, int H, int W,
+                             float *y, void *workspace, size_t workspace_bytes,
+                             void *stream);
+
+/*
+ * qcnn_net_forward_host -- the same, with x and y in HOST memory (pinned
+ * memory gives the fastest copies).  Copies x to the device, runs the
+ * stack, copies y back, and synchronizes `stream` before returning.
+ */
+qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers,
+                                  const float *x_host, int N, int C, int H,
+                                  int W, float *y_host, void *workspace,
+                                  size_t workspace_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QCNN_H */

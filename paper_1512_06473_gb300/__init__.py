@@ -1,0 +1,274 @@
+"""GB300 (sm_103a) implementation of the test-phase response of
+product-quantized conv and FC layers (Q-CNN, Wu et al., arXiv 1512.06473).
+
+This module only marshals arguments: every step of the path runs in the CUDA
+kernels of libqcnn.so behind the C ABI of include/qcnn.h.  PyTorch provides
+device memory and the current stream.  There is no CPU fallback: if the
+library cannot be built or loaded, every call raises.
+
+Layouts (fp32 unless stated, all CUDA tensors, contiguous):
+  FC   : x [N, Cs], D [M, K, Csp], codes [M, Ct] uint8, bias [Ct]  -> [N, Ct]
+  conv : x [N, Cs, H, W], D [M, K, Csp], codes [Ct, kh*kw, M] uint8 -> [N, Ct, Ho, Wo]
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+import torch
+
+from . import _lib
+from ._lib import QcnnError, load  # noqa: F401
+
+__all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
+           "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _need(t: torch.Tensor, name: str, dtype, ndim: int):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if t.dim() != ndim or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous {ndim}-d tensor, got shape {tuple(t.shape)}")
+
+
+def _workspace(nbytes: int, device, workspace: Optional[torch.Tensor]):
+    if nbytes == 0:
+        return None, 0
+    if workspace is not None:
+        return workspace, workspace.numel() * workspace.element_size()
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + nbytes], nbytes
+
+
+def launch_count() -> int:
+    """Kernels launched by libqcnn in this process so far."""
+    return int(load().qcnn_launch_count())
+
+
+def lut_build(x: torch.Tensor, D: torch.Tensor, out: Optional[torch.Tensor] = None, stream=None):
+    """Tables lut[n, m, p, k] = <x[n, m*Csp:(m+1)*Csp, p], D[m, k]> (Sec. 3.1 / 3.2).
+    x is [N, Cs] (FC input) or [N, Cs, H, W]; returns [N, M, H*W, K]."""
+    if x.dim() == 2:
+        N, Cs = x.shape
+        H = W = 1
+    else:
+        _need(x, "x", torch.float32, 4)
+        N, Cs, H, W = x.shape
+    _need(x, "x", torch.float32, x.dim())
+    _need(D, "D", torch.float32, 3)
+    M, K, Csp = D.shape
+    if out is None:
+        out = torch.empty((N, M, H * W, K), dtype=torch.float32, device=x.device)
+    _need(out, "out", torch.float32, 4)
+    _lib.check(load().qcnn_lut_build(_ptr(x), N, Cs, H, W, _ptr(D), Csp, K, _ptr(out),
+                                     _stream(stream)), "qcnn_lut_build")
+    return out
+
+
+def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, stream=None):
+    """Eq. 5: y[n, ct] = bias[ct] + sum_m LUT_n[m, codes[m, ct]] (then ReLU)."""
+    _need(x, "x", torch.float32, 2)
+    _need(D, "D", torch.float32, 3)
+    _need(codes, "codes", torch.uint8, 2)
+    N, Cs = x.shape
+    M, K, Csp = D.shape
+    Ct = codes.shape[1]
+    if bias is not None:
+        _need(bias, "bias", torch.float32, 1)
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)),
+               "qcnn_fc_workspace_size")
+    ws, wsb = _workspace(nb.value, x.device, workspace)
+    if out is None:
+        out = torch.empty((N, Ct), dtype=torch.float32, device=x.device)
+    _lib.check(lib.qcnn_fc_forward(_ptr(x), N, Cs, Ct, _ptr(D), Csp, K, _ptr(codes),
+                                   _ptr(bias), _ptr(out), int(bool(relu)), _ptr(ws), wsb,
+                                   _stream(stream)), "qcnn_fc_forward")
+    return out
+
+
+def conv_pack_codes(codes: torch.Tensor, K: int, kh: int, kw: int, stream=None) -> torch.Tensor:
+    """Model-load-time re-layout of conv codes [Ct, kh*kw, M] for the fused kernels."""
+    _need(codes, "codes", torch.uint8, 3)
+    Ct, kk, M = codes.shape
+    if kk != kh * kw:
+        raise ValueError("codes.shape[1] must be kh*kw")
+    lib = load()
+    nbytes = lib.qcnn_conv_packed_codes_bytes(Ct, kh, kw, M)
+    packed = torch.empty(nbytes + 256, dtype=torch.uint8, device=codes.device)
+    off = (-packed.data_ptr()) % 256
+    packed = packed[off:off + nbytes]
+    _lib.check(lib.qcnn_conv_pack_codes(_ptr(codes), Ct, kh, kw, M, K, _ptr(packed),
+                                        _stream(stream)), "qcnn_conv_pack_codes")
+    return packed
+
+
+def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, algo="auto",
+                 packed=False, Ct=None, out=None, workspace=None, stream=None):
+    """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,
+    then ``Ct`` is required) the output of conv_pack_codes."""
+    _need(x, "x", torch.float32, 4)
+    _need(D, "D", torch.float32, 3)
+    N, Cs, H, W = x.shape
+    M, K, Csp = D.shape
+    if packed:
+        if Ct is None:
+            raise ValueError("Ct is required with packed codes")
+        _need(codes, "codes", torch.uint8, 1)
+    else:
+        _need(codes, "codes", torch.uint8, 3)
+        Ct = codes.shape[0]
+    if bias is not None:
+        _need(bias, "bias", torch.float32, 1)
+    layout = _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL
+    a = _lib.ALGO[algo]
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, layout,
+                                            a, ctypes.byref(nb)), "qcnn_conv_workspace_size")
+    ws, wsb = _workspace(nb.value, x.device, workspace)
+    Ho = (H + 2 * pad - kh) // stride + 1
+    Wo = (W + 2 * pad - kw) // stride + 1
+    if out is None:
+        out = torch.empty((N, Ct, Ho, Wo), dtype=torch.float32, device=x.device)
+    _lib.check(lib.qcnn_conv_forward(_ptr(x), N, Cs, H, W, Ct, kh, kw, stride, pad, _ptr(D), Csp,
+                                     K, _ptr(codes), layout, _ptr(bias), _ptr(out),
+                                     int(bool(relu)), a, _ptr(ws), wsb, _stream(stream)),
+               "qcnn_conv_forward")
+    return out
+
+
+def maxpool(x, k, s, out=None, stream=None):
+    _need(x, "x", torch.float32, 4)
+    N, C, H, W = x.shape
+    if out is None:
+        out = torch.empty((N, C, (H - k) // s + 1, (W - k) // s + 1), dtype=torch.float32,
+                          device=x.device)
+    _lib.check(load().qcnn_maxpool(_ptr(x), N, C, H, W, k, s, _ptr(out), _stream(stream)),
+               "qcnn_maxpool")
+    return out
+
+
+# ------------------------------------------------------------------ network
+@dataclass
+class ConvLayer:
+    D: torch.Tensor
+    codes: torch.Tensor         # [Ct, kh*kw, M] (canonical) or packed bytes
+    bias: Optional[torch.Tensor]
+    Ct: int
+    kh: int
+    kw: int
+    stride: int = 1
+    pad: int = 0
+    relu: bool = True
+    algo: str = "auto"
+    packed: bool = False
+
+
+@dataclass
+class FCLayer:
+    D: torch.Tensor
+    codes: torch.Tensor         # [M, Ct]
+    bias: Optional[torch.Tensor]
+    relu: bool = True
+
+
+@dataclass
+class PoolLayer:
+    k: int
+    s: int
+
+
+class Net:
+    """A stack of PQ conv / PQ FC / max-pool layers run by qcnn_net_forward."""
+
+    def __init__(self, layers: Sequence, in_shape: Sequence[int]):
+        self.layers = list(layers)
+        self.in_shape = tuple(in_shape)
+        arr = (_lib.Layer * len(self.layers))()
+        for i, L in enumerate(self.layers):
+            d = arr[i]
+            if isinstance(L, ConvLayer):
+                M, K, Csp = L.D.shape
+                d.kind, d.Ct, d.kh, d.kw, d.stride, d.pad = _lib.LAYER_CONV, L.Ct, L.kh, L.kw, L.stride, L.pad
+                d.Csp, d.K, d.relu, d.algo = Csp, K, int(L.relu), _lib.ALGO[L.algo]
+                d.codes_layout = _lib.CODES_PACKED if L.packed else _lib.CODES_CANONICAL
+                d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
+            elif isinstance(L, FCLayer):
+                M, K, Csp = L.D.shape
+                d.kind, d.Ct, d.Csp, d.K, d.relu = _lib.LAYER_FC, L.codes.shape[1], Csp, K, int(L.relu)
+                d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
+            elif isinstance(L, PoolLayer):
+                d.kind, d.kh, d.kw, d.stride = _lib.LAYER_MAXPOOL, L.k, L.k, L.s
+            else:
+                raise TypeError(f"unknown layer {L!r}")
+        self._arr = arr
+        C, H, W = self.in_shape
+        oc, oh, ow = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+        _lib.check(load().qcnn_net_output_shape(arr, len(arr), C, H, W, ctypes.byref(oc),
+                                                ctypes.byref(oh), ctypes.byref(ow)),
+                   "qcnn_net_output_shape")
+        self.out_shape = (oc.value, oh.value, ow.value)
+
+    def _out(self, N, device):
+        C, H, W = self.out_shape
+        shape = (N, C) if (H, W) == (1, 1) else (N, C, H, W)
+        return torch.empty(shape, dtype=torch.float32, device=device)
+
+    def workspace_bytes(self, N: int, host_io: bool = False) -> int:
+        nb = ctypes.c_size_t()
+        C, H, W = self.in_shape
+        _lib.check(load().qcnn_net_workspace_size(self._arr, len(self._arr), N, C, H, W,
+                                                  int(host_io), ctypes.byref(nb)),
+                   "qcnn_net_workspace_size")
+        return nb.value
+
+    def alloc_workspace(self, N: int, device="cuda", host_io: bool = False):
+        nb = self.workspace_bytes(N, host_io)
+        ws, _ = _workspace(max(nb, 1), torch.device(device), None)
+        return ws
+
+    def forward(self, x: torch.Tensor, out=None, workspace=None, stream=None):
+        _need(x, "x", torch.float32, 4)
+        N, C, H, W = x.shape
+        if (C, H, W) != self.in_shape:
+            raise ValueError(f"input shape {(C, H, W)} != {self.in_shape}")
+        if workspace is None:
+            workspace = self.alloc_workspace(N, x.device)
+        if out is None:
+            out = self._out(N, x.device)
+        wsb = workspace.numel()
+        _lib.check(load().qcnn_net_forward(self._arr, len(self._arr), _ptr(x), N, C, H, W,
+                                           _ptr(out), _ptr(workspace), wsb, _stream(stream)),
+                   "qcnn_net_forward")
+        return out
+
+    def forward_host(self, x_host: torch.Tensor, out_host: torch.Tensor, workspace: torch.Tensor,
+                     stream=None):
+        """x_host / out_host are CPU tensors (pinned for speed); workspace must be
+        alloc_workspace(N, host_io=True).  Synchronizes the stream."""
+        if x_host.is_cuda or out_host.is_cuda:
+            raise TypeError("forward_host takes CPU tensors")
+        if not (x_host.is_contiguous() and out_host.is_contiguous()):
+            raise ValueError("host tensors must be contiguous")
+        N, C, H, W = x_host.shape
+        _lib.check(load().qcnn_net_forward_host(self._arr, len(self._arr), _ptr(x_host), N, C, H,
+                                                W, _ptr(out_host), _ptr(workspace),
+                                                workspace.numel(), _stream(stream)),
+                   "qcnn_net_forward_host")
+        return out_host

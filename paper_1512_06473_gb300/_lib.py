@@ -1,0 +1,99 @@
+"""ctypes view of libqcnn.so (include/qcnn.h).  Loading fails loudly: there is
+no CPU fallback and no other backend."""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+
+from . import build as _build
+
+c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_uint64
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+ALGO = {"auto": 0, "fused": 1, "unfused": 2}
+CODES_CANONICAL, CODES_PACKED = 0, 1
+LAYER_CONV, LAYER_FC, LAYER_MAXPOOL = 0, 1, 2
+
+
+class QcnnError(RuntimeError):
+    def __init__(self, status: int, what: str, msg: str):
+        super().__init__(f"{what}: {msg} (status {status})")
+        self.status = status
+
+
+class Layer(ctypes.Structure):
+    """Mirror of qcnn_layer."""
+    _fields_ = [("kind", c_int), ("Ct", c_int), ("kh", c_int), ("kw", c_int),
+                ("stride", c_int), ("pad", c_int), ("Csp", c_int), ("K", c_int),
+                ("relu", c_int), ("algo", c_int), ("codes_layout", c_int),
+                ("D", c_void_p), ("codes", c_void_p), ("bias", c_void_p)]
+
+
+_SIGS = {
+    "qcnn_status_string": (ctypes.c_char_p, [c_int]),
+    "qcnn_last_cuda_error": (c_int, []),
+    "qcnn_launch_count": (c_uint64, []),
+    "qcnn_lut_build": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
+                               c_void_p, c_void_p]),
+    "qcnn_fc_workspace_size": (c_int, [c_int, c_int, c_int, c_int, c_int, ctypes.POINTER(c_size_t)]),
+    "qcnn_fc_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
+                                c_void_p, c_void_p, c_int, c_void_p, c_size_t, c_void_p]),
+    "qcnn_conv_packed_codes_bytes": (c_size_t, [c_int, c_int, c_int, c_int]),
+    "qcnn_conv_pack_codes": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_void_p,
+                                     c_void_p]),
+    "qcnn_conv_workspace_size": (c_int, [c_int] * 13 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_conv_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_int,
+                                  c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int,
+                                  c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t,
+                                  c_void_p]),
+    "qcnn_maxpool": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_void_p,
+                             c_void_p]),
+    "qcnn_net_output_shape": (c_int, [ctypes.POINTER(Layer), c_int, c_int, c_int, c_int,
+                                      ctypes.POINTER(c_int), ctypes.POINTER(c_int),
+                                      ctypes.POINTER(c_int)]),
+    "qcnn_net_workspace_size": (c_int, [ctypes.POINTER(Layer), c_int, c_int, c_int, c_int, c_int,
+                                        c_int, ctypes.POINTER(c_size_t)]),
+    "qcnn_net_forward": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int, c_int,
+                                 c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "qcnn_net_forward_host": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int,
+                                      c_int, c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
+}
+
+_lock = threading.Lock()
+_lib = None
+
+
+def header_functions(path: str | None = None):
+    """Names of the functions include/qcnn.h declares."""
+    path = path or os.path.join(_build.INCLUDE, "qcnn.h")
+    text = open(path).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(qcnn_[a-z0-9_]+)\s*\(", text)))
+
+
+def load(path: str | None = None):
+    """Load (building first when the sources are newer) and bind libqcnn.so."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        so = path or _build.build()
+        lib = ctypes.CDLL(so)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(lib, name)
+            f.restype = res
+            f.argtypes = args
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def check(status: int, what: str):
+    if status != OK:
+        lib = load()
+        msg = lib.qcnn_status_string(status).decode()
+        if status == ERR_CUDA:
+            msg += f" (cudaError {lib.qcnn_last_cuda_error()})"
+        raise QcnnError(status, what, msg)

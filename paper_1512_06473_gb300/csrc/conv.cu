@@ -1,0 +1,557 @@
+// conv.cu -- PQ convolutional layer response (Sec. 3.2, Eq. 7):
+//   y[n][ct][oy][ox] = bias[ct] + sum_{ky,kx} sum_m LUT_n[m][p_s][k_m(ct, p_k)]
+//   LUT_n[m][p_s][k] = <x_n^(m)(p_s), D^(m)_k>,  p_s = (oy*s - pad + ky, ox*s - pad + kx)
+//
+// Two kernels compute it:
+//  * conv_fused (stride 1): one CTA owns an image, a band of TH output rows
+//    (all columns) and CT_CTA output channels.  For each sub-space m it
+//    builds the table of every halo position of the band in shared memory
+//    -- layout lut[k][h], h = linear index in the zero-padded halo grid of
+//    row pitch W + 2 pad -- and then gathers from it.  Lanes of a warp take
+//    consecutive positions of that padded grid, so for one (c_t, p_k) the
+//    whole warp shares one code k and reads 32 consecutive words of row k:
+//    bank-conflict free, and the kernel offset (ky, kx) is a plain shift
+//    ky*pitch + kx of the read address.  Lanes that fall on the padding
+//    columns compute values that are discarded.
+//  * conv_unfused (any stride): tables are first written to the workspace
+//    in a stride-phase-split layout lut[nb][m][k][ay][ax][py][px] with
+//    (iy, ix) = (py*s + ay, px*s + ax), so that consecutive output columns
+//    read consecutive words for every kernel offset; a gather kernel then
+//    reads them through L1/L2.  Images are processed in chunks sized to
+//    stay L2 resident.
+#include "qcnn_internal.cuh"
+
+#include <algorithm>
+#include <cmath>
+
+namespace qcnn {
+
+// ===================================================================== pack
+int packed_ct(int Ct) { return cdiv(Ct, 256) * 256; }
+size_t packed_codes_bytes(int Ct, int kk, int M) {
+    return (size_t)M * kk * (size_t)packed_ct(Ct);
+}
+
+// packed[m][pk][ct] = min(codes[ct][pk][m], K - 1); zero for ct >= Ct.
+__global__ void pack_codes_kernel(const uint8_t *__restrict__ codes, int Ct, int kk,
+                                  int M, int K, int CtP, uint8_t *__restrict__ packed) {
+    const size_t total = (size_t)M * kk * CtP;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int ct = (int)(i % CtP);
+        const size_t r = i / CtP;
+        const int pk = (int)(r % kk);
+        const int m = (int)(r / kk);
+        unsigned v = 0;
+        if (ct < Ct) {
+            v = codes[((size_t)ct * kk + pk) * M + m];
+            v = v < (unsigned)K ? v : (unsigned)(K - 1);
+        }
+        packed[i] = (uint8_t)v;
+    }
+}
+
+qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K,
+                              uint8_t *packed, cudaStream_t st) {
+    const size_t total = packed_codes_bytes(Ct, kk, M);
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
+    pack_codes_kernel<<<blocks, 256, 0, st>>>(codes, Ct, kk, M, K, packed_ct(Ct), packed);
+    return after_launch();
+}
+
+// ==================================================================== fused
+struct ConvFusedArgs {
+    const float *__restrict__ x;
+    const float *__restrict__ D;
+    const uint8_t *__restrict__ codes;  // packed [M][kk][CtP]
+    const float *__restrict__ bias;
+    float *__restrict__ y;
+    int N, Cs, H, W, Ct, kh, kw, pad, Csp, K, M, Ho, Wo;
+    int pitch, TH, KS, HP, ct_cta, CtP, relu;
+    int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
+};
+
+constexpr int kFusedThreads = 256;
+
+// Shared memory carve-up of the fused kernel (byte offsets, 16-aligned).
+struct FusedSmem {
+    size_t lut, xs, ds, cs, total;
+};
+__host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats,
+                                                       int csp4, int kk, int ct_cta) {
+    FusedSmem s;
+    s.lut = 0;
+    s.xs = ((size_t)K * KS * 4 + 15) / 16 * 16;
+    s.ds = s.xs + (size_t)2 * xs_floats * 4;
+    s.cs = s.ds + (size_t)2 * K * csp4 * 4;
+    s.total = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
+    return s;
+}
+
+// Load CTW consecutive code bytes (16-byte aligned in shared memory).
+template <int CTW>
+__device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[CTW / 4]) {
+    if constexpr (CTW % 16 == 0) {
+#pragma unroll
+        for (int i = 0; i < CTW / 16; ++i) {
+            const uint4 v = reinterpret_cast<const uint4 *>(p)[i];
+            w[4 * i + 0] = v.x;
+            w[4 * i + 1] = v.y;
+            w[4 * i + 2] = v.z;
+            w[4 * i + 3] = v.w;
+        }
+    } else if constexpr (CTW == 8) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(p);
+        w[0] = v.x;
+        w[1] = v.y;
+    } else {
+        static_assert(CTW == 4, "CTW must be 4, 8 or a multiple of 16");
+        w[0] = *reinterpret_cast<const unsigned *>(p);
+    }
+}
+
+// P     : 32-position slots per warp
+// CTW   : output channels per warp
+// WP    : warps along positions (8 / WP warps along channels)
+// CSP4  : C'_s rounded up to 4 or 8 (register width of one sub-vector)
+template <int P, int CTW, int WP, int CSP4>
+__global__ void __launch_bounds__(kFusedThreads, 2) conv_fused_kernel(const ConvFusedArgs a) {
+    constexpr int QB = 16 / CSP4;  // sub-codewords per lane per build pass
+    extern __shared__ __align__(16) unsigned char smem[];
+    const FusedSmem L = fused_smem_layout(a.K, a.KS, a.xs_floats, CSP4, a.kh * a.kw, a.ct_cta);
+    float *lut = reinterpret_cast<float *>(smem + L.lut);
+    float *xs = reinterpret_cast<float *>(smem + L.xs);
+    float *ds = reinterpret_cast<float *>(smem + L.ds);
+    uint8_t *cs = smem + L.cs;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int wp = warp % WP, wc = warp / WP;
+    const int oy0 = blockIdx.x * a.TH;
+    const int ct0 = blockIdx.y * a.ct_cta;
+    const int n = blockIdx.z;
+    const int kk = a.kh * a.kw;
+    const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
+
+    // ---- asynchronous staging of sub-space m into buffer b ---------------
+    auto stage = [&](int m, int b) {
+        float *xb = xs + b * a.xs_floats;
+        const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * a.H * a.W;
+        for (int e = tid; e < HP * CSP4; e += kFusedThreads) {
+            const int h = e % HP, j = e / HP;
+            const int r = h / pitch, c = h - r * pitch;
+            const int iy = oy0 - a.pad + r, ix = c - a.pad;
+            const bool ok = j < a.Csp && iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+            const float *src = ok ? xn + ((size_t)j * a.H + iy) * a.W + ix : a.x;
+            cp_async4(xb + h * CSP4 + j, src, ok);
+        }
+        float *db = ds + b * K * CSP4;
+        const float *dm = a.D + (size_t)m * K * a.Csp;
+        for (int e = tid; e < K * CSP4; e += kFusedThreads) {
+            const int k = e / CSP4, j = e - k * CSP4;
+            const bool ok = j < a.Csp;
+            cp_async4(db + e, ok ? dm + k * a.Csp + j : a.D, ok);
+        }
+        uint8_t *cb = cs + (size_t)b * kk * a.ct_cta;
+        const int q16 = a.ct_cta / 16;
+        const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
+        for (int e = tid; e < kk * q16; e += kFusedThreads) {
+            const int pk = e / q16, q = e - pk * q16;
+            cp_async16(cb + pk * a.ct_cta + q * 16, cm + (size_t)pk * a.CtP + q * 16);
+        }
+        cp_async_commit();
+    };
+
+    float acc[CTW][P];
+#pragma unroll
+    for (int c = 0; c < CTW; ++c)
+#pragma unroll
+        for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
+
+    // Byte offset of this lane's first position inside a table row.
+    const int lane_off4 = (wp * P * 32 + lane) * 4;
+    const int KS4 = KS * 4;
+    const unsigned char *lutb = reinterpret_cast<const unsigned char *>(lut);
+    const unsigned kmax4 = (unsigned)(K - 1) * 0x01010101u;  // clamp codes into [0, K)
+
+    stage(0, 0);
+    for (int m = 0; m < a.M; ++m) {
+        const int b = m & 1;
+        cp_async_wait<0>();
+        __syncthreads();  // stage m visible; gather of m-1 finished everywhere
+        if (m + 1 < a.M) stage(m + 1, b ^ 1);
+
+        // ---- build: lut[k][h] = <x(h), D[m][k]> ----------------------------
+        {
+            const float *xb = xs + b * a.xs_floats;
+            const float *db = ds + b * K * CSP4;
+            const int hpw = cdiv(HP, 8);
+            const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
+            for (int q0 = 0; q0 < K; q0 += 32 * QB) {
+                float dk[QB][CSP4];
+#pragma unroll
+                for (int i = 0; i < QB; ++i) {
+                    const int k = q0 + 32 * i + lane;
+#pragma unroll
+                    for (int j = 0; j < CSP4; j += 4) {
+                        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (k < K) v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
+                        dk[i][j] = v.x;
+                        dk[i][j + 1] = v.y;
+                        dk[i][j + 2] = v.z;
+                        dk[i][j + 3] = v.w;
+                    }
+                }
+                for (int h = h0; h < h1; ++h) {
+                    float xv[CSP4];
+#pragma unroll
+                    for (int j = 0; j < CSP4; j += 4) {
+                        const float4 v = *reinterpret_cast<const float4 *>(xb + h * CSP4 + j);
+                        xv[j] = v.x;
+                        xv[j + 1] = v.y;
+                        xv[j + 2] = v.z;
+                        xv[j + 3] = v.w;
+                    }
+#pragma unroll
+                    for (int i = 0; i < QB; ++i) {
+                        const int k = q0 + 32 * i + lane;
+                        float v = 0.f;
+#pragma unroll
+                        for (int j = 0; j < CSP4; ++j) v = fmaf(xv[j], dk[i][j], v);
+                        if (k < K) lut[k * KS + h] = v;
+                    }
+                }
+            }
+        }
+        __syncthreads();
+
+        // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
+        {
+            const uint8_t *cb = cs + (size_t)b * kk * a.ct_cta + wc * CTW;
+            for (int ky = 0; ky < a.kh; ++ky) {
+                for (int kx = 0; kx < a.kw; ++kx) {
+                    const int pk = ky * a.kw + kx;
+                    unsigned w[CTW / 4];
+                    load_code_words<CTW>(cb + pk * a.ct_cta, w);
+#pragma unroll
+                    for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
+                    const int base4 = lane_off4 + (ky * pitch + kx) * 4;
+#pragma unroll
+                    for (int c = 0; c < CTW; ++c) {
+                        const unsigned code = byte_of(w[c >> 2], c & 3);
+                        const unsigned char *row = lutb + (int)code * KS4 + base4;
+#pragma unroll
+                        for (int p = 0; p < P; ++p)
+                            acc[c][p] += *reinterpret_cast<const float *>(row + p * 128);
+                    }
+                }
+            }
+        }
+    }
+
+    // ---- epilogue: bias, ReLU, store --------------------------------------
+#pragma unroll
+    for (int c = 0; c < CTW; ++c) {
+        const int ct = ct0 + wc * CTW + c;
+        if (ct >= a.Ct) continue;
+        const float bv = a.bias ? a.bias[ct] : 0.f;
+#pragma unroll
+        for (int p = 0; p < P; ++p) {
+            const int l = (wp * P + p) * 32 + lane;
+            const int r = l / pitch, col = l - r * pitch;
+            const int oy = oy0 + r;
+            if (r < a.TH && col < a.Wo && oy < a.Ho) {
+                float v = acc[c][p] + bv;
+                if (a.relu) v = fmaxf(v, 0.f);
+                a.y[(((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + col] = v;
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------- variant table --
+struct FusedVariant {
+    int P, CTW, WP, CSP4;
+    void (*fn)(ConvFusedArgs);
+};
+
+#define QCNN_FUSED(P, CTW, WP, C4) {P, CTW, WP, C4, conv_fused_kernel<P, CTW, WP, C4>}
+static const FusedVariant kFused[] = {
+    QCNN_FUSED(2, 32, 1, 4), QCNN_FUSED(4, 16, 1, 4), QCNN_FUSED(4, 8, 2, 4),
+    QCNN_FUSED(2, 32, 1, 8), QCNN_FUSED(4, 16, 1, 8), QCNN_FUSED(4, 8, 2, 8),
+};
+#undef QCNN_FUSED
+constexpr int kNumFused = sizeof(kFused) / sizeof(kFused[0]);
+
+static int ks_for(int need) {  // smallest KS >= need with KS % 32 == 1
+    int ks = need;
+    while (ks % 32 != 1) ++ks;
+    return ks;
+}
+
+ConvFusedPlan plan_conv_fused(const ConvShape &s) {
+    ConvFusedPlan best;
+    if (s.stride != 1 || s.Csp > kMaxCsp) return best;
+    const int csp4 = s.Csp <= 4 ? 4 : 8;
+    const int pitch = s.W + 2 * s.pad;
+    const int kk = s.kh * s.kw;
+    const int sms = num_sms();
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int smem_optin = 0;
+    if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess ||
+        smem_optin <= 0)
+        smem_optin = 227 * 1024;
+    int smem_sm = 0;
+    if (cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
+            cudaSuccess ||
+        smem_sm <= 0)
+        smem_sm = 228 * 1024;
+    for (int v = 0; v < kNumFused; ++v) {
+        const FusedVariant &fv = kFused[v];
+        if (fv.CSP4 != csp4) continue;
+        const int slots = fv.WP * fv.P;
+        int TH = std::min(slots * 32 / pitch, s.Ho);
+        if (TH < 1) continue;
+        const int row_tiles = cdiv(s.Ho, TH);
+        TH = cdiv(s.Ho, row_tiles);  // balance the bands
+        const int HP = (TH + s.kh - 1) * pitch;
+        const int KS = ks_for(slots * 32 + (s.kh - 1) * pitch + (s.kw - 1));
+        const int ct_cta = (8 / fv.WP) * fv.CTW;
+        const int xs_floats = cdiv(HP, 4) * 4 * csp4;
+        const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta).total;
+        if (smem > (size_t)smem_optin) continue;
+        const int cps = std::max(1, std::min(2, (int)(smem_sm / (smem + 1024))));
+        const int ct_tiles = cdiv(s.Ct, ct_cta);
+        const double ctas = (double)s.N * row_tiles * ct_tiles;
+        const double waves = std::ceil(ctas / (sms * cps));
+        // work per CTA in shared-memory wavefronts: gather + table build
+        const double gather = (double)slots * ct_cta * kk * s.M;
+        const double build = (double)HP * s.K * s.M * 1.5 / 32.0;
+        const double per_cta = gather + build;
+        const double score = waves * per_cta / cps * (cps == 1 ? 1.15 : 1.0);
+        if (!best.ok || score < best.score) {
+            best.ok = true;
+            best.variant = v;
+            best.P = fv.P;
+            best.CTW = fv.CTW;
+            best.WP = fv.WP;
+            best.TH = TH;
+            best.pitch = pitch;
+            best.KS = KS;
+            best.HP = HP;
+            best.ct_cta = ct_cta;
+            best.row_tiles = row_tiles;
+            best.ct_tiles = ct_tiles;
+            best.smem = smem;
+            best.score = score;
+        }
+    }
+    return best;
+}
+
+qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const float *x,
+                              const float *D, const uint8_t *packed, const float *bias,
+                              float *y, int relu, cudaStream_t st) {
+    const FusedVariant &fv = kFused[p.variant];
+    ConvFusedArgs a;
+    a.x = x;
+    a.D = D;
+    a.codes = packed;
+    a.bias = bias;
+    a.y = y;
+    a.N = s.N;
+    a.Cs = s.Cs;
+    a.H = s.H;
+    a.W = s.W;
+    a.Ct = s.Ct;
+    a.kh = s.kh;
+    a.kw = s.kw;
+    a.pad = s.pad;
+    a.Csp = s.Csp;
+    a.K = s.K;
+    a.M = s.M;
+    a.Ho = s.Ho;
+    a.Wo = s.Wo;
+    a.pitch = p.pitch;
+    a.TH = p.TH;
+    a.KS = p.KS;
+    a.HP = p.HP;
+    a.ct_cta = p.ct_cta;
+    a.CtP = packed_ct(s.Ct);
+    a.relu = relu;
+    a.xs_floats = cdiv(p.HP, 4) * 4 * fv.CSP4;
+    cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)p.smem);
+    if (e != cudaSuccess) return cuda_status(e);
+    dim3 grid(p.row_tiles, p.ct_tiles, s.N);
+    fv.fn<<<grid, kFusedThreads, p.smem, st>>>(a);
+    return after_launch();
+}
+
+// ================================================================== unfused
+// Tables of a chunk of NB images in the stride-phase-split layout
+//   lut[nb][m][k][ay][ax][py][px],  iy = py*s + ay,  ix = px*s + ax.
+struct UnfusedLutArgs {
+    const float *__restrict__ x;
+    const float *__restrict__ D;
+    float *__restrict__ lut;
+    int n0, NB, Cs, H, W, s, Csp, K, M, HQ, WQ;
+};
+
+__global__ void __launch_bounds__(256) conv_unfused_lut_kernel(const UnfusedLutArgs a) {
+    extern __shared__ __align__(16) float dsm[];  // D[m] : [K][Csp]
+    const int m = blockIdx.y, nb = blockIdx.z;
+    const int n = a.n0 + nb;
+    for (int e = threadIdx.x; e < a.K * a.Csp + kMaxCsp; e += blockDim.x)
+        dsm[e] = e < a.K * a.Csp ? a.D[(size_t)m * a.K * a.Csp + e] : 0.f;
+    __syncthreads();
+    const int PQ = a.s * a.s * a.HQ * a.WQ;
+    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    if (q >= PQ) return;
+    const int px = q % a.WQ;
+    int r = q / a.WQ;
+    const int py = r % a.HQ;
+    r /= a.HQ;
+    const int ax = r % a.s, ay = r / a.s;
+    const int iy = py * a.s + ay, ix = px * a.s + ax;
+    float xv[kMaxCsp];
+    const bool in = iy < a.H && ix < a.W;
+    const float *xp = a.x + (((size_t)n * a.Cs + (size_t)m * a.Csp) * a.H + (in ? iy : 0)) * a.W +
+                      (in ? ix : 0);
+#pragma unroll
+    for (int j = 0; j < kMaxCsp; ++j) {
+        // the address stays inside x even for the lanes j >= Csp that are discarded
+        const float v = __ldg(xp + (size_t)min(j, a.Csp - 1) * a.H * a.W);
+        xv[j] = (in && j < a.Csp) ? v : 0.f;
+    }
+    float *out = a.lut + ((size_t)nb * a.M + m) * a.K * (size_t)PQ + q;
+    for (int k = 0; k < a.K; ++k) {
+        const float *dk = dsm + k * a.Csp;  // dsm is padded by kMaxCsp floats
+        float v = 0.f;
+#pragma unroll
+        for (int j = 0; j < kMaxCsp; ++j)
+            if (j < a.Csp) v = fmaf(xv[j], dk[j], v);
+        out[(size_t)k * PQ] = v;
+    }
+}
+
+struct UnfusedGatherArgs {
+    const float *__restrict__ lut;
+    const uint8_t *__restrict__ codes;  // packed [M][kk][CtP]
+    const float *__restrict__ bias;
+    float *__restrict__ y;
+    int n0, Ct, CtP, H, W, kh, kw, s, pad, K, M, Ho, Wo, HQ, WQ, relu;
+    int col_tiles;
+};
+
+constexpr int kUnfCTW = 16;  // channels per warp
+constexpr int kUnfSL = 2;    // 32-column slots per warp
+
+// grid: x = row tile (8 rows, one per warp) * col tile, y = channel tile, z = image in chunk
+__global__ void __launch_bounds__(256) conv_unfused_gather_kernel(const UnfusedGatherArgs a) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rt = blockIdx.x / a.col_tiles, ctile = blockIdx.x % a.col_tiles;
+    const int oy = rt * 8 + warp;
+    const int ct0 = blockIdx.y * kUnfCTW;
+    const int nb = blockIdx.z;
+    if (oy >= a.Ho) return;
+    const int PQ = a.s * a.s * a.HQ * a.WQ;
+    float acc[kUnfCTW][kUnfSL];
+#pragma unroll
+    for (int c = 0; c < kUnfCTW; ++c)
+#pragma unroll
+        for (int sl = 0; sl < kUnfSL; ++sl) acc[c][sl] = 0.f;
+    int ox[kUnfSL];
+#pragma unroll
+    for (int sl = 0; sl < kUnfSL; ++sl) ox[sl] = (ctile * kUnfSL + sl) * 32 + lane;
+    const int kk = a.kh * a.kw;
+    for (int m = 0; m < a.M; ++m) {
+        const float *lm = a.lut + ((size_t)nb * a.M + m) * a.K * (size_t)PQ;
+        for (int ky = 0; ky < a.kh; ++ky) {
+            const int iy = oy * a.s - a.pad + ky;
+            if (iy < 0 || iy >= a.H) continue;
+            const int ay = iy % a.s, py = iy / a.s;
+            for (int kx = 0; kx < a.kw; ++kx) {
+                const int t = kx - a.pad;
+                const int ax = ((t % a.s) + a.s) % a.s;
+                const int dx = (t - ax) / a.s;  // exact
+                bool ok[kUnfSL];
+                int off[kUnfSL];
+#pragma unroll
+                for (int sl = 0; sl < kUnfSL; ++sl) {
+                    const int ix = ox[sl] * a.s + t;
+                    ok[sl] = ox[sl] < a.Wo && ix >= 0 && ix < a.W;
+                    off[sl] = ((ay * a.s + ax) * a.HQ + py) * a.WQ + ox[sl] + dx;
+                }
+                const uint8_t *cp = a.codes + ((size_t)m * kk + ky * a.kw + kx) * a.CtP + ct0;
+                const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(cp));
+                const unsigned kmax4 = (unsigned)(a.K - 1) * 0x01010101u;
+                const unsigned w[4] = {__vminu4(cw.x, kmax4), __vminu4(cw.y, kmax4),
+                                       __vminu4(cw.z, kmax4), __vminu4(cw.w, kmax4)};
+#pragma unroll
+                for (int c = 0; c < kUnfCTW; ++c) {
+                    const unsigned code = byte_of(w[c >> 2], c & 3);
+                    const float *row = lm + (size_t)code * PQ;
+#pragma unroll
+                    for (int sl = 0; sl < kUnfSL; ++sl)
+                        if (ok[sl]) acc[c][sl] += __ldg(row + off[sl]);
+                }
+            }
+        }
+    }
+    const int n = a.n0 + nb;
+#pragma unroll
+    for (int c = 0; c < kUnfCTW; ++c) {
+        const int ct = ct0 + c;
+        if (ct >= a.Ct) continue;
+        const float bv = a.bias ? a.bias[ct] : 0.f;
+#pragma unroll
+        for (int sl = 0; sl < kUnfSL; ++sl) {
+            if (ox[sl] >= a.Wo) continue;
+            float v = acc[c][sl] + bv;
+            if (a.relu) v = fmaxf(v, 0.f);
+            a.y[(((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + ox[sl]] = v;
+        }
+    }
+}
+
+constexpr size_t kUnfusedLutBudget = (size_t)64 << 20;  // keep a chunk L2 resident
+
+ConvUnfusedPlan plan_conv_unfused(const ConvShape &s) {
+    ConvUnfusedPlan p;
+    p.HQ = cdiv(s.H, s.stride);
+    p.WQ = cdiv(s.W, s.stride);
+    const size_t per_image =
+        (size_t)s.M * s.K * s.stride * s.stride * p.HQ * p.WQ * sizeof(float);
+    p.NB = (int)std::max<size_t>(1, std::min<size_t>(s.N, kUnfusedLutBudget / per_image));
+    p.lut_bytes = per_image * p.NB;
+    return p;
+}
+
+qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p, const float *x,
+                                const float *D, const uint8_t *packed, const float *bias,
+                                float *y, int relu, float *lut_ws, cudaStream_t st) {
+    const int PQ = s.stride * s.stride * p.HQ * p.WQ;
+    const int col_tiles = cdiv(s.Wo, 32 * kUnfSL);
+    for (int n0 = 0; n0 < s.N; n0 += p.NB) {
+        const int nb = std::min(p.NB, s.N - n0);
+        UnfusedLutArgs la{x, D, lut_ws, n0, nb, s.Cs, s.H, s.W, s.stride, s.Csp, s.K, s.M,
+                          p.HQ, p.WQ};
+        dim3 g1(cdiv(PQ, 256), s.M, nb);
+        conv_unfused_lut_kernel<<<g1, 256, ((size_t)s.K * s.Csp + kMaxCsp) * sizeof(float),
+                                  st>>>(la);
+        qcnn_status rc = after_launch();
+        if (rc != QCNN_OK) return rc;
+        UnfusedGatherArgs ga{lut_ws, packed, bias, y, n0, s.Ct, packed_ct(s.Ct), s.H, s.W,
+                             s.kh, s.kw, s.stride, s.pad, s.K, s.M, s.Ho, s.Wo, p.HQ, p.WQ,
+                             relu, col_tiles};
+        dim3 g2(cdiv(s.Ho, 8) * col_tiles, cdiv(s.Ct, kUnfCTW), nb);
+        conv_unfused_gather_kernel<<<g2, 256, 0, st>>>(ga);
+        rc = after_launch();
+        if (rc != QCNN_OK) return rc;
+    }
+    return QCNN_OK;
+}
+
+}  // namespace qcnn

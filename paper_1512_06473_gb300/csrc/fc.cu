@@ -1,0 +1,291 @@
+// fc.cu -- PQ fully-connected layer response (Sec. 3.1, Eq. 5):
+//   y[n][ct] = bias[ct] + sum_m LUT_n[m][k_m(ct)],  LUT_n[m][k] = <x_n^(m), D^(m)_k>
+//
+// One CTA owns NT images, CT_CTA outputs and a range of sub-spaces.  It walks
+// that range in chunks of MCH sub-spaces: the chunk's tables for its NT
+// images are built in shared memory, layout lut[mm][k][n] with an odd row
+// pitch NTP, then every lane -- which owns CPL = 4 consecutive outputs and
+// NW images -- adds lut[mm][code][n] for its codes.  Lanes of a warp hold
+// different codes for the same (mm, n): with the odd pitch, distinct codes
+// below 32 land in distinct banks and equal codes broadcast, so the gather is
+// conflict free for K <= 32.  Codes are read straight from device memory,
+// four per 32-bit load, coalesced along c_t; each code serves NW images.
+// When the sub-space range is split over several CTAs (to fill the GPU),
+// the partial sums go to the workspace and a second kernel adds them in a
+// fixed order (deterministic), then applies bias and ReLU.
+#include "qcnn_internal.cuh"
+
+#include <algorithm>
+#include <cmath>
+
+namespace qcnn {
+
+struct FcArgs {
+    const float *__restrict__ x;
+    const float *__restrict__ D;
+    const uint8_t *__restrict__ codes;  // [M][Ct]
+    const float *__restrict__ bias;
+    float *__restrict__ y;
+    float *__restrict__ partial;  // [splits][N][Ct] when splits > 1
+    int N, Cs, Ct, Csp, K, M;
+    int NT, CT_CTA, MCH, n_chunks, chunks_per_split, splits, relu;
+    int NTP;  // odd pitch of a table row (>= NT)
+    int NTX;  // odd pitch of a staged x row (>= NT)
+};
+
+constexpr int kFcThreads = 256;
+constexpr int kCPL = 4;  // outputs per lane
+
+struct FcSmem {
+    size_t lut, xs, ds, total;
+};
+__host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int NTP, int NTX, int Csp) {
+    FcSmem s;
+    s.lut = 0;
+    s.xs = ((size_t)MCH * K * NTP * 4 + 15) / 16 * 16;
+    s.ds = s.xs + ((size_t)2 * MCH * Csp * NTX * 4 + 15) / 16 * 16;
+    s.total = s.ds + (size_t)2 * MCH * K * Csp * 4;
+    return s;
+}
+
+// Four consecutive codes of row m starting at output ct (zero past Ct),
+// clamped into [0, K).
+__device__ __forceinline__ unsigned load_codes4(const uint8_t *__restrict__ codes, int Ct,
+                                                int m, int ct, bool vec, unsigned kmax4) {
+    unsigned w = 0;
+    const uint8_t *p = codes + (size_t)m * Ct + ct;
+    if (vec && ct + 3 < Ct) {
+        w = __ldg(reinterpret_cast<const unsigned *>(p));
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (ct + i < Ct) w |= (unsigned)__ldg(p + i) << (8 * i);
+    }
+    return __vminu4(w, kmax4);
+}
+
+// NW : images per lane;  WN : warps along images (8 / WN along outputs)
+template <int NW, int WN>
+__global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a) {
+    constexpr int MCH_MAX = 16;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const FcSmem L = fc_smem_layout(a.MCH, a.K, a.NTP, a.NTX, a.Csp);
+    float *lut = reinterpret_cast<float *>(smem + L.lut);
+    float *xs = reinterpret_cast<float *>(smem + L.xs);
+    float *ds = reinterpret_cast<float *>(smem + L.ds);
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int wn = warp % WN, wc = warp / WN;
+    const int ct0 = blockIdx.x * a.CT_CTA;
+    const int n0 = blockIdx.y * a.NT;
+    const int split = blockIdx.z;
+    const int c_begin = split * a.chunks_per_split;
+    const int c_end = min(a.n_chunks, c_begin + a.chunks_per_split);
+    const int ct_lane = ct0 + (wc * 32 + lane) * kCPL;
+    const int nbase = wn * NW;
+    const int CCH = a.MCH * a.Csp;  // staged x floats per image
+    const bool vec = (a.Ct & 3) == 0;
+    const unsigned kmax4 = (unsigned)(a.K - 1) * 0x01010101u;
+
+    auto stage = [&](int c, int b) {
+        const int m0 = c * a.MCH;
+        const int mch = min(a.MCH, a.M - m0);
+        float *xb = xs + (size_t)b * CCH * a.NTX;
+        for (int e = tid; e < CCH * a.NT; e += kFcThreads) {
+            const int cc = e % CCH, nn = e / CCH;
+            const bool ok = cc < mch * a.Csp && n0 + nn < a.N;
+            const float *src = ok ? a.x + (size_t)(n0 + nn) * a.Cs + (size_t)m0 * a.Csp + cc : a.x;
+            cp_async4(xb + cc * a.NTX + nn, src, ok);
+        }
+        float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
+        const int dn = a.MCH * a.K * a.Csp, dv = mch * a.K * a.Csp;
+        const float *dsrc = a.D + (size_t)m0 * a.K * a.Csp;
+        for (int e = tid; e < dn; e += kFcThreads) cp_async4(db + e, e < dv ? dsrc + e : a.D, e < dv);
+        cp_async_commit();
+    };
+
+    float acc[kCPL][NW];
+#pragma unroll
+    for (int c = 0; c < kCPL; ++c)
+#pragma unroll
+        for (int i = 0; i < NW; ++i) acc[c][i] = 0.f;
+
+    if (c_begin < c_end) stage(c_begin, 0);
+    for (int c = c_begin; c < c_end; ++c) {
+        const int b = (c - c_begin) & 1;
+        const int m0 = c * a.MCH;
+        const int mch = min(a.MCH, a.M - m0);
+        cp_async_wait<0>();
+        __syncthreads();  // chunk c staged; gather of c-1 finished
+        if (c + 1 < c_end) stage(c + 1, b ^ 1);
+
+        // codes of this chunk for this lane (latency hidden by the build)
+        unsigned cw[MCH_MAX];
+#pragma unroll
+        for (int mm = 0; mm < MCH_MAX; ++mm)
+            cw[mm] = (mm < mch && ct_lane < a.Ct) ? load_codes4(a.codes, a.Ct, m0 + mm, ct_lane, vec, kmax4)
+                                                  : 0u;
+
+        // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>
+        {
+            const float *xb = xs + (size_t)b * CCH * a.NTX;
+            const float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
+            const int tot = a.MCH * a.K * a.NT;
+            for (int e = tid; e < tot; e += kFcThreads) {
+                const int nn = e % a.NT;
+                const int r = e / a.NT;
+                const int k = r % a.K, mm = r / a.K;
+                const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                const float *dp = db + (mm * a.K + k) * a.Csp;
+                float v = 0.f;
+#pragma unroll
+                for (int j = 0; j < kMaxCsp; ++j)
+                    if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
+                lut[(mm * a.K + k) * a.NTP + nn] = v;
+            }
+        }
+        __syncthreads();
+
+        // gather
+#pragma unroll
+        for (int mm = 0; mm < MCH_MAX; ++mm) {
+            if (mm < mch) {
+#pragma unroll
+                for (int q = 0; q < kCPL; ++q) {
+                    const int code = (int)byte_of(cw[mm], q);
+                    const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
+#pragma unroll
+                    for (int i = 0; i < NW; ++i) acc[q][i] += row[i];
+                }
+            }
+        }
+    }
+
+    // epilogue
+#pragma unroll
+    for (int i = 0; i < NW; ++i) {
+        const int n = n0 + nbase + i;
+        if (n >= a.N) continue;
+#pragma unroll
+        for (int q = 0; q < kCPL; ++q) {
+            const int ct = ct_lane + q;
+            if (ct >= a.Ct) continue;
+            if (a.splits == 1) {
+                float v = acc[q][i] + (a.bias ? a.bias[ct] : 0.f);
+                if (a.relu) v = fmaxf(v, 0.f);
+                a.y[(size_t)n * a.Ct + ct] = v;
+            } else {
+                a.partial[((size_t)split * a.N + n) * a.Ct + ct] = acc[q][i];
+            }
+        }
+    }
+}
+
+__global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, int N, int Ct,
+                                 const float *__restrict__ bias, int relu, float *__restrict__ y) {
+    const size_t total = (size_t)N * Ct;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        float v = 0.f;
+        for (int s = 0; s < splits; ++s) v += partial[(size_t)s * total + i];
+        if (bias) v += bias[i % Ct];
+        if (relu) v = fmaxf(v, 0.f);
+        y[i] = v;
+    }
+}
+
+struct FcVariant {
+    int NW, WN;
+    void (*fn)(FcArgs);
+};
+#define QCNN_FC(NW, WN) {NW, WN, fc_fused_kernel<NW, WN>}
+static const FcVariant kFcVariants[] = {QCNN_FC(16, 2), QCNN_FC(8, 2), QCNN_FC(4, 1),
+                                        QCNN_FC(1, 1)};
+#undef QCNN_FC
+constexpr int kNumFc = sizeof(kFcVariants) / sizeof(kFcVariants[0]);
+
+FcPlan plan_fc(const FcShape &s) {
+    FcPlan best{};
+    double best_t = 1e300;
+    const int sms = num_sms();
+    const int MCH = s.K <= 32 ? 16 : std::max(1, 512 / s.K);
+    const int n_chunks = cdiv(s.M, MCH);
+    for (int v = 0; v < kNumFc; ++v) {
+        const FcVariant &fv = kFcVariants[v];
+        const int NT = fv.NW * fv.WN;
+        const int CT_CTA = (8 / fv.WN) * 32 * kCPL;
+        const int NTP = NT | 1, NTX = NT | 1;
+        const size_t smem = fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp).total;
+        if (smem > 110 * 1024) continue;
+        const int n_tiles = cdiv(s.N, NT), ct_tiles = cdiv(s.Ct, CT_CTA);
+        const int tiles = n_tiles * ct_tiles;
+        const int target = 2 * sms * 2;
+        int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
+        const int cps = cdiv(n_chunks, splits);
+        splits = cdiv(n_chunks, cps);
+        const double ctas = (double)tiles * splits;
+        const double waves = std::ceil(ctas / (2.0 * sms));
+        // one CTA: shared-memory wavefronts (gather + build) per chunk
+        const double per_chunk = (double)MCH * NT * CT_CTA / 32.0 + (double)MCH * s.K * NT / 32.0 * 2;
+        const double t_smem = waves * cps * per_chunk / 2.0 / 1.9e9;
+        const double bytes = (double)s.M * s.Ct * n_tiles + 4.0 * s.N * s.Cs * ct_tiles +
+                             (splits > 1 ? 8.0 * splits * s.N * s.Ct : 0.0);
+        const double t = std::max(t_smem, bytes / 6.0e12) + (splits > 1 ? 3e-6 : 0.0);
+        if (t < best_t) {
+            best_t = t;
+            best.variant = v;
+            best.NT = NT;
+            best.CT_CTA = CT_CTA;
+            best.MCH = MCH;
+            best.n_chunks = n_chunks;
+            best.splits = splits;
+            best.chunks_per_split = cps;
+            best.n_tiles = n_tiles;
+            best.ct_tiles = ct_tiles;
+            best.smem = smem;
+            best.partial_bytes = splits > 1 ? (size_t)splits * s.N * s.Ct * sizeof(float) : 0;
+        }
+    }
+    return best;
+}
+
+qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const float *D,
+                      const uint8_t *codes, const float *bias, float *y, int relu,
+                      float *partial_ws, cudaStream_t st) {
+    const FcVariant &fv = kFcVariants[p.variant];
+    FcArgs a;
+    a.x = x;
+    a.D = D;
+    a.codes = codes;
+    a.bias = bias;
+    a.y = y;
+    a.partial = partial_ws;
+    a.N = s.N;
+    a.Cs = s.Cs;
+    a.Ct = s.Ct;
+    a.Csp = s.Csp;
+    a.K = s.K;
+    a.M = s.M;
+    a.NT = p.NT;
+    a.CT_CTA = p.CT_CTA;
+    a.MCH = p.MCH;
+    a.n_chunks = p.n_chunks;
+    a.chunks_per_split = p.chunks_per_split;
+    a.splits = p.splits;
+    a.relu = relu;
+    a.NTP = p.NT | 1;
+    a.NTX = p.NT | 1;
+    cudaError_t e =
+        cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    if (e != cudaSuccess) return cuda_status(e);
+    dim3 grid(p.ct_tiles, p.n_tiles, p.splits);
+    fv.fn<<<grid, kFcThreads, p.smem, st>>>(a);
+    qcnn_status rc = after_launch();
+    if (rc != QCNN_OK || p.splits == 1) return rc;
+    const size_t total = (size_t)s.N * s.Ct;
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
+    fc_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu, y);
+    return after_launch();
+}
+
+}  // namespace qcnn

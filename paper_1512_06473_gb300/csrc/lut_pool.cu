@@ -1,0 +1,83 @@
+// lut_pool.cu -- the stand-alone look-up-table build (Sec. 3.1 / 3.2: the
+// tables of inner products pre-computed for every input vector) and the
+// max-pool used between the layers of the whole-network stack.
+#include "qcnn_internal.cuh"
+
+#include <algorithm>
+
+namespace qcnn {
+
+// lut[n][m][p][k] = sum_j x[n][m*Csp + j][p] * D[m][k][j].
+// A CTA owns 32 consecutive (m, p) units of one image; its 32*K outputs are
+// one contiguous, coalesced stretch of `lut`.  The kernel is bound by the
+// table writes (K/Csp floats written per float read).
+constexpr int kLutUnits = 32;
+
+__global__ void __launch_bounds__(256) lut_build_kernel(const float *__restrict__ x, int Cs,
+                                                        int P, const float *__restrict__ D,
+                                                        int Csp, int K, int M,
+                                                        float *__restrict__ lut) {
+    __shared__ float xs[kLutUnits][kMaxCsp];
+    const int n = blockIdx.y;
+    const long long units = (long long)M * P;
+    const long long u0 = (long long)blockIdx.x * kLutUnits;
+    for (int e = threadIdx.x; e < kLutUnits * kMaxCsp; e += blockDim.x) {
+        const int ul = e / kMaxCsp, j = e % kMaxCsp;
+        const long long u = u0 + ul;
+        float v = 0.f;
+        if (u < units && j < Csp) {
+            const int m = (int)(u / P), p = (int)(u % P);
+            v = x[((size_t)n * Cs + (size_t)m * Csp + j) * P + p];
+        }
+        xs[ul][j] = v;
+    }
+    __syncthreads();
+    const int nu = (int)std::min<long long>(kLutUnits, units - u0);
+    float *out = lut + ((size_t)n * units + u0) * K;
+    for (int e = threadIdx.x; e < nu * K; e += blockDim.x) {
+        const int ul = e / K, k = e % K;
+        const int m = (int)((u0 + ul) / P);
+        const float *dk = D + ((size_t)m * K + k) * Csp;
+        float v = 0.f;
+        for (int j = 0; j < Csp; ++j) v = fmaf(xs[ul][j], __ldg(dk + j), v);
+        out[e] = v;
+    }
+}
+
+qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *D, int Csp,
+                             int K, float *lut, cudaStream_t st) {
+    const int M = Cs / Csp;
+    const long long units = (long long)M * P;
+    dim3 grid((unsigned)((units + kLutUnits - 1) / kLutUnits), N);
+    lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M, lut);
+    return after_launch();
+}
+
+// k x k max-pool, stride s, no padding: one thread per output element.
+__global__ void maxpool_kernel(const float *__restrict__ x, int NC, int H, int W, int k, int s,
+                               int Ho, int Wo, float *__restrict__ y) {
+    const size_t total = (size_t)NC * Ho * Wo;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int ox = (int)(i % Wo);
+        const size_t r = i / Wo;
+        const int oy = (int)(r % Ho);
+        const size_t nc = r / Ho;
+        const float *p = x + (nc * H + (size_t)oy * s) * W + (size_t)ox * s;
+        float v = p[0];
+        for (int dy = 0; dy < k; ++dy)
+            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, __ldg(p + (size_t)dy * W + dx));
+        y[i] = v;
+    }
+}
+
+qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k, int s, float *y,
+                           cudaStream_t st) {
+    const int Ho = (H - k) / s + 1, Wo = (W - k) / s + 1;
+    const size_t total = (size_t)N * C * Ho * Wo;
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 16);
+    maxpool_kernel<<<blocks, 256, 0, st>>>(x, N * C, H, W, k, s, Ho, Wo, y);
+    return after_launch();
+}
+
+}  // namespace qcnn

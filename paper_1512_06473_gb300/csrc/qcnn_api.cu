@@ -1,0 +1,411 @@
+// qcnn_api.cu -- the extern "C" entry points of include/qcnn.h: argument
+// checks (all done on the host before anything is enqueued), workspace
+// carving, algorithm choice and the layer-stack driver.
+#include "qcnn_internal.cuh"
+
+#include <algorithm>
+#include <atomic>
+#include <climits>
+#include <vector>
+
+namespace qcnn {
+
+static std::atomic<uint64_t> g_launches{0};
+static std::atomic<int> g_last_cuda_error{0};
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+qcnn_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return QCNN_OK;
+    g_last_cuda_error.store((int)e);
+    return QCNN_ERR_CUDA;
+}
+
+qcnn_status after_launch() {
+    count_launch();
+    return cuda_status(cudaGetLastError());
+}
+
+int num_sms() {
+    static std::atomic<int> cached[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return 152;
+    }
+    int v = cached[dev].load();
+    if (v > 0) return v;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
+        cudaGetLastError();
+        v = 152;
+    }
+    cached[dev].store(v);
+    return v;
+}
+
+}  // namespace qcnn
+
+using namespace qcnn;
+
+namespace {
+
+inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+bool fits_int(long long v) { return v > 0 && v < (long long)INT_MAX; }
+
+bool pq_ok(int Cs, int Csp, int K) {
+    return Cs > 0 && Csp >= 1 && Csp <= kMaxCsp && K >= 1 && K <= kMaxK && Cs % Csp == 0;
+}
+
+bool conv_shape(int N, int Cs, int H, int W, int Ct, int kh, int kw, int stride, int pad,
+                int Csp, int K, ConvShape *s) {
+    if (N <= 0 || H <= 0 || W <= 0 || Ct <= 0 || kh <= 0 || kw <= 0 || stride <= 0 || pad < 0)
+        return false;
+    if (!pq_ok(Cs, Csp, K)) return false;
+    if (H + 2 * pad < kh || W + 2 * pad < kw) return false;
+    const int Ho = (H + 2 * pad - kh) / stride + 1, Wo = (W + 2 * pad - kw) / stride + 1;
+    if (Ho <= 0 || Wo <= 0) return false;
+    if (!fits_int((long long)N * Cs * H * W) || !fits_int((long long)N * Ct * Ho * Wo) ||
+        !fits_int((long long)Ct * kh * kw * (Cs / Csp)))
+        return false;
+    *s = ConvShape{N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, Cs / Csp, Ho, Wo};
+    return true;
+}
+
+bool fc_shape(int N, int Cs, int Ct, int Csp, int K, FcShape *s) {
+    if (N <= 0 || Ct <= 0 || !pq_ok(Cs, Csp, K)) return false;
+    if (!fits_int((long long)N * Cs) || !fits_int((long long)N * Ct) ||
+        !fits_int((long long)(Cs / Csp) * Ct))
+        return false;
+    *s = FcShape{N, Cs, Ct, Csp, K, Cs / Csp};
+    return true;
+}
+
+// ------------------------------------------------------------ conv plan ---
+struct ConvCall {
+    ConvShape s;
+    bool fused;
+    ConvFusedPlan fp;
+    ConvUnfusedPlan up;
+    size_t packed_off, lut_off, total;
+};
+
+qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvCall *c) {
+    if (codes_layout != QCNN_CODES_CANONICAL && codes_layout != QCNN_CODES_PACKED)
+        return QCNN_ERR_INVALID_ARG;
+    if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED)
+        return QCNN_ERR_INVALID_ARG;
+    c->s = s;
+    c->fused = false;
+    if (algo != QCNN_ALGO_UNFUSED) {
+        c->fp = plan_conv_fused(s);
+        c->fused = c->fp.ok;
+        if (algo == QCNN_ALGO_FUSED && !c->fused) return QCNN_ERR_UNSUPPORTED;
+    }
+    if (!c->fused) c->up = plan_conv_unfused(s);
+    size_t off = 0;
+    c->packed_off = off;
+    if (codes_layout == QCNN_CODES_CANONICAL)
+        off += align_up(packed_codes_bytes(s.Ct, s.kh * s.kw, s.M), kWsAlign);
+    c->lut_off = off;
+    if (!c->fused) off += align_up(c->up.lut_bytes, kWsAlign);
+    c->total = off;
+    return QCNN_OK;
+}
+
+qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const uint8_t *codes,
+                     int codes_layout, const float *bias, float *y, int relu, void *ws,
+                     cudaStream_t st) {
+    const uint8_t *packed = codes;
+    if (codes_layout == QCNN_CODES_CANONICAL) {
+        uint8_t *p = static_cast<uint8_t *>(ws) + c.packed_off;
+        qcnn_status rc =
+            launch_pack_codes(codes, c.s.Ct, c.s.kh * c.s.kw, c.s.M, c.s.K, p, st);
+        if (rc != QCNN_OK) return rc;
+        packed = p;
+    }
+    if (c.fused) return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, st);
+    float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
+    return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
+}
+
+bool ws_ok(const void *ws, size_t have, size_t need) {
+    if (need == 0) return true;
+    return ws != nullptr && have >= need && (reinterpret_cast<uintptr_t>(ws) % kWsAlign) == 0;
+}
+
+// -------------------------------------------------------------- net plan ---
+struct NetStep {
+    int kind;
+    ConvCall conv;
+    FcShape fc;
+    FcPlan fcp;
+    int C, H, W;        // input of this layer (per image)
+    int oC, oH, oW;     // output
+    size_t scratch;     // bytes of layer scratch
+};
+
+struct NetPlan {
+    int N;
+    std::vector<NetStep> steps;
+    size_t act_floats;  // floats of one ping-pong activation buffer
+    size_t scratch;     // max layer scratch
+    size_t act_off[2], scratch_off, xin_off, yout_off, total;
+};
+
+qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H, int W,
+                     int host_io, NetPlan *np) {
+    if (!layers || n_layers <= 0 || N <= 0 || C <= 0 || H <= 0 || W <= 0)
+        return QCNN_ERR_INVALID_ARG;
+    if (!fits_int((long long)N * C * H * W)) return QCNN_ERR_INVALID_ARG;
+    np->N = N;
+    np->steps.clear();
+    np->act_floats = 0;
+    np->scratch = 0;
+    int c = C, h = H, w = W;
+    for (int i = 0; i < n_layers; ++i) {
+        const qcnn_layer &L = layers[i];
+        NetStep st{};
+        st.kind = L.kind;
+        st.C = c;
+        st.H = h;
+        st.W = w;
+        if (L.kind == QCNN_LAYER_CONV) {
+            if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
+            ConvShape s;
+            if (!conv_shape(N, c, h, w, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K, &s))
+                return QCNN_ERR_INVALID_ARG;
+            qcnn_status rc = plan_conv_call(s, L.codes_layout, L.algo, &st.conv);
+            if (rc != QCNN_OK) return rc;
+            st.scratch = st.conv.total;
+            st.oC = L.Ct;
+            st.oH = s.Ho;
+            st.oW = s.Wo;
+        } else if (L.kind == QCNN_LAYER_FC) {
+            if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
+            const long long cs = (long long)c * h * w;
+            if (cs >= INT_MAX) return QCNN_ERR_INVALID_ARG;
+            if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, &st.fc)) return QCNN_ERR_INVALID_ARG;
+            st.fcp = plan_fc(st.fc);
+            st.scratch = align_up(st.fcp.partial_bytes, kWsAlign);
+            st.oC = L.Ct;
+            st.oH = 1;
+            st.oW = 1;
+        } else if (L.kind == QCNN_LAYER_MAXPOOL) {
+            if (L.kh <= 0 || L.stride <= 0 || L.kh > h || L.kh > w) return QCNN_ERR_INVALID_ARG;
+            st.oC = c;
+            st.oH = (h - L.kh) / L.stride + 1;
+            st.oW = (w - L.kh) / L.stride + 1;
+        } else {
+            return QCNN_ERR_INVALID_ARG;
+        }
+        const long long out = (long long)N * st.oC * st.oH * st.oW;
+        if (!fits_int(out)) return QCNN_ERR_INVALID_ARG;
+        if (i + 1 < n_layers) np->act_floats = std::max(np->act_floats, (size_t)out);
+        np->scratch = std::max(np->scratch, st.scratch);
+        c = st.oC;
+        h = st.oH;
+        w = st.oW;
+        np->steps.push_back(st);
+    }
+    size_t off = 0;
+    for (int b = 0; b < 2; ++b) {
+        np->act_off[b] = off;
+        off += align_up(np->act_floats * sizeof(float), kWsAlign);
+    }
+    np->scratch_off = off;
+    off += align_up(np->scratch, kWsAlign);
+    np->xin_off = np->yout_off = off;
+    if (host_io) {
+        np->xin_off = off;
+        off += align_up((size_t)N * C * H * W * sizeof(float), kWsAlign);
+        const NetStep &last = np->steps.back();
+        np->yout_off = off;
+        off += align_up((size_t)N * last.oC * last.oH * last.oW * sizeof(float), kWsAlign);
+    }
+    np->total = off;
+    return QCNN_OK;
+}
+
+qcnn_status run_net(const qcnn_layer *layers, const NetPlan &np, const float *x, float *y,
+                    void *ws, cudaStream_t st) {
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    const int n = (int)np.steps.size();
+    const float *in = x;
+    for (int i = 0; i < n; ++i) {
+        const NetStep &s = np.steps[i];
+        const qcnn_layer &L = layers[i];
+        float *out = (i + 1 == n) ? y : reinterpret_cast<float *>(base + np.act_off[i & 1]);
+        void *scratch = base + np.scratch_off;
+        qcnn_status rc = QCNN_OK;
+        if (s.kind == QCNN_LAYER_CONV) {
+            rc = run_conv(s.conv, in, L.D, L.codes, L.codes_layout, L.bias, out, L.relu,
+                          scratch, st);
+        } else if (s.kind == QCNN_LAYER_FC) {
+            rc = launch_fc(s.fc, s.fcp, in, L.D, L.codes, L.bias, out, L.relu,
+                           reinterpret_cast<float *>(scratch), st);
+        } else {
+            rc = launch_maxpool(in, np.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
+        }
+        if (rc != QCNN_OK) return rc;
+        in = out;
+    }
+    return QCNN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *qcnn_status_string(qcnn_status s) {
+    switch (s) {
+        case QCNN_OK: return "ok";
+        case QCNN_ERR_INVALID_ARG: return "invalid argument";
+        case QCNN_ERR_UNSUPPORTED: return "unsupported by this build";
+        case QCNN_ERR_WORKSPACE: return "workspace too small or misaligned";
+        case QCNN_ERR_CUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+int qcnn_last_cuda_error(void) { return g_last_cuda_error.load(); }
+
+uint64_t qcnn_launch_count(void) { return g_launches.load(); }
+
+qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W, const float *D, int Csp,
+                           int K, float *lut, void *stream) {
+    if (!x || !D || !lut || N <= 0 || H <= 0 || W <= 0 || !pq_ok(Cs, Csp, K))
+        return QCNN_ERR_INVALID_ARG;
+    const long long P = (long long)H * W;
+    if (!fits_int((long long)N * Cs * P) || !fits_int((long long)N * (Cs / Csp) * P * K))
+        return QCNN_ERR_INVALID_ARG;
+    return launch_lut_build(x, N, Cs, (int)P, D, Csp, K, lut, as_stream(stream));
+}
+
+qcnn_status qcnn_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K, size_t *bytes) {
+    FcShape s;
+    if (!bytes || !fc_shape(N, Cs, Ct, Csp, K, &s)) return QCNN_ERR_INVALID_ARG;
+    *bytes = align_up(plan_fc(s).partial_bytes, kWsAlign);
+    return QCNN_OK;
+}
+
+qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct, const float *D, int Csp,
+                            int K, const uint8_t *codes, const float *bias, float *y, int relu,
+                            void *workspace, size_t workspace_bytes, void *stream) {
+    FcShape s;
+    if (!x || !D || !codes || !y || !fc_shape(N, Cs, Ct, Csp, K, &s))
+        return QCNN_ERR_INVALID_ARG;
+    const FcPlan p = plan_fc(s);
+    if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
+    return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(workspace),
+                     as_stream(stream));
+}
+
+size_t qcnn_conv_packed_codes_bytes(int Ct, int kh, int kw, int M) {
+    if (Ct <= 0 || kh <= 0 || kw <= 0 || M <= 0) return 0;
+    return packed_codes_bytes(Ct, kh * kw, M);
+}
+
+qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw, int M, int K,
+                                 uint8_t *packed, void *stream) {
+    if (!codes || !packed || Ct <= 0 || kh <= 0 || kw <= 0 || M <= 0 || K < 1 || K > kMaxK)
+        return QCNN_ERR_INVALID_ARG;
+    if (!fits_int((long long)packed_ct(Ct) * kh * kw * M)) return QCNN_ERR_INVALID_ARG;
+    return launch_pack_codes(codes, Ct, kh * kw, M, K, packed, as_stream(stream));
+}
+
+qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh, int kw,
+                                     int stride, int pad, int Csp, int K, int codes_layout,
+                                     int algo, size_t *bytes) {
+    ConvShape s;
+    if (!bytes || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, &s))
+        return QCNN_ERR_INVALID_ARG;
+    ConvCall c;
+    qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    if (rc != QCNN_OK) return rc;
+    *bytes = c.total;
+    return QCNN_OK;
+}
+
+qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int Ct, int kh,
+                              int kw, int stride, int pad, const float *D, int Csp, int K,
+                              const uint8_t *codes, int codes_layout, const float *bias,
+                              float *y, int relu, int algo, void *workspace,
+                              size_t workspace_bytes, void *stream) {
+    ConvShape s;
+    if (!x || !D || !codes || !y ||
+        !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, &s))
+        return QCNN_ERR_INVALID_ARG;
+    ConvCall c;
+    qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    if (rc != QCNN_OK) return rc;
+    if (!ws_ok(workspace, workspace_bytes, c.total)) return QCNN_ERR_WORKSPACE;
+    return run_conv(c, x, D, codes, codes_layout, bias, y, relu, workspace, as_stream(stream));
+}
+
+qcnn_status qcnn_maxpool(const float *x, int N, int C, int H, int W, int k, int s, float *y,
+                         void *stream) {
+    if (!x || !y || N <= 0 || C <= 0 || H <= 0 || W <= 0 || k <= 0 || s <= 0 || k > H || k > W)
+        return QCNN_ERR_INVALID_ARG;
+    if (!fits_int((long long)N * C * H * W)) return QCNN_ERR_INVALID_ARG;
+    return launch_maxpool(x, N, C, H, W, k, s, y, as_stream(stream));
+}
+
+qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers, int C, int H, int W,
+                                  int *out_C, int *out_H, int *out_W) {
+    if (!out_C || !out_H || !out_W) return QCNN_ERR_INVALID_ARG;
+    NetPlan np;
+    qcnn_status rc = plan_net(layers, n_layers, 1, C, H, W, 0, &np);
+    if (rc != QCNN_OK) return rc;
+    *out_C = np.steps.back().oC;
+    *out_H = np.steps.back().oH;
+    *out_W = np.steps.back().oW;
+    return QCNN_OK;
+}
+
+qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers, int N, int C, int H,
+                                    int W, int host_io, size_t *bytes) {
+    if (!bytes) return QCNN_ERR_INVALID_ARG;
+    NetPlan np;
+    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, host_io, &np);
+    if (rc != QCNN_OK) return rc;
+    *bytes = np.total;
+    return QCNN_OK;
+}
+
+qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers, const float *x, int N,
+                             int C, int H, int W, float *y, void *workspace,
+                             size_t workspace_bytes, void *stream) {
+    if (!x || !y) return QCNN_ERR_INVALID_ARG;
+    NetPlan np;
+    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, 0, &np);
+    if (rc != QCNN_OK) return rc;
+    if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
+    return run_net(layers, np, x, y, workspace, as_stream(stream));
+}
+
+qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const float *x_host,
+                                  int N, int C, int H, int W, float *y_host, void *workspace,
+                                  size_t workspace_bytes, void *stream) {
+    if (!x_host || !y_host) return QCNN_ERR_INVALID_ARG;
+    NetPlan np;
+    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, 1, &np);
+    if (rc != QCNN_OK) return rc;
+    if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
+    cudaStream_t st = as_stream(stream);
+    uint8_t *base = static_cast<uint8_t *>(workspace);
+    float *xd = reinterpret_cast<float *>(base + np.xin_off);
+    float *yd = reinterpret_cast<float *>(base + np.yout_off);
+    const NetStep &last = np.steps.back();
+    const size_t xb = (size_t)N * C * H * W * sizeof(float);
+    const size_t yb = (size_t)N * last.oC * last.oH * last.oW * sizeof(float);
+    rc = cuda_status(cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st));
+    if (rc != QCNN_OK) return rc;
+    rc = run_net(layers, np, xd, yd, workspace, st);
+    if (rc != QCNN_OK) return rc;
+    rc = cuda_status(cudaMemcpyAsync(y_host, yd, yb, cudaMemcpyDeviceToHost, st));
+    if (rc != QCNN_OK) return rc;
+    return cuda_status(cudaStreamSynchronize(st));
+}
+
+}  // extern "C"

@@ -1,0 +1,138 @@
+// qcnn_internal.cuh -- declarations shared by the translation units of
+// libqcnn (never installed; the public interface is include/qcnn.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/qcnn.h"
+
+namespace qcnn {
+
+constexpr int kMaxCsp = 8;        // largest sub-space dimension C'_s served
+constexpr int kMaxK = 256;        // codes are uint8
+constexpr size_t kWsAlign = 256;  // alignment of every workspace carve-out
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+__host__ __device__ inline int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// Number of SMs of the current device (cached per device).
+int num_sms();
+
+// Book-keeping of launches and CUDA errors (qcnn_api.cu).
+void count_launch();
+qcnn_status cuda_status(cudaError_t e);
+// Check the launch that was just enqueued and count it.
+qcnn_status after_launch();
+
+// ---------------------------------------------------------------- conv ----
+struct ConvShape {
+    int N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, M, Ho, Wo;
+};
+
+// Fused plan: one CTA = (image, band of TH output rows, CT_CTA channels).
+struct ConvFusedPlan {
+    bool ok = false;
+    int variant = -1;   // index into the instantiated kernel table
+    int P, CTW, WP;     // slots per warp, channels per warp, warps on positions
+    int TH;             // output rows per CTA
+    int pitch;          // W + 2 pad
+    int KS;             // floats per table row (per sub-codeword)
+    int HP;             // halo positions with data: (TH + kh - 1) * pitch
+    int ct_cta;         // channels per CTA
+    int row_tiles, ct_tiles;
+    size_t smem;        // dynamic shared memory bytes
+    double score;       // estimated cost (lower is better)
+};
+
+ConvFusedPlan plan_conv_fused(const ConvShape &s);
+
+struct ConvUnfusedPlan {
+    int NB;             // images per table chunk
+    int HQ, WQ;         // positions per phase (ceil(H/s), ceil(W/s))
+    size_t lut_bytes;   // workspace bytes for one chunk of tables
+};
+ConvUnfusedPlan plan_conv_unfused(const ConvShape &s);
+
+size_t packed_codes_bytes(int Ct, int kk, int M);
+int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
+
+qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K,
+                              uint8_t *packed, cudaStream_t st);
+qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p,
+                              const float *x, const float *D,
+                              const uint8_t *packed, const float *bias, float *y,
+                              int relu, cudaStream_t st);
+qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
+                                const float *x, const float *D,
+                                const uint8_t *packed, const float *bias,
+                                float *y, int relu, float *lut_ws,
+                                cudaStream_t st);
+
+// ------------------------------------------------------------------ fc ----
+struct FcShape {
+    int N, Cs, Ct, Csp, K, M;
+};
+struct FcPlan {
+    int variant;        // kernel table index
+    int NT, CT_CTA;     // images and outputs per CTA
+    int MCH;            // sub-spaces per shared-memory chunk
+    int n_chunks;       // ceil(M / MCH)
+    int splits;         // CTAs along m (partial sums reduced afterwards)
+    int chunks_per_split;
+    int n_tiles, ct_tiles;
+    size_t smem;
+    size_t partial_bytes;  // workspace for split partial sums (0 if splits == 1)
+};
+FcPlan plan_fc(const FcShape &s);
+qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x,
+                      const float *D, const uint8_t *codes, const float *bias,
+                      float *y, int relu, float *partial_ws, cudaStream_t st);
+
+// ------------------------------------------------------------ lut, pool ----
+qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *D,
+                             int Csp, int K, float *lut, cudaStream_t st);
+qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k,
+                           int s, float *y, cudaStream_t st);
+
+}  // namespace qcnn
+
+// ----------------------------------------------------------- device side ----
+#ifdef __CUDACC__
+namespace qcnn {
+
+__device__ __forceinline__ unsigned smem_addr(const void *p) {
+    return static_cast<unsigned>(__cvta_generic_to_shared(p));
+}
+
+// 4-byte asynchronous global->shared copy; when `pred` is false nothing is
+// read and the destination is filled with zeros (src-size 0).
+__device__ __forceinline__ void cp_async4(void *dst, const void *src, bool pred) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(smem_addr(dst)),
+                 "l"(src), "r"(pred ? 4 : 0)
+                 : "memory");
+}
+
+// 16-byte asynchronous global->shared copy (both addresses 16-byte aligned).
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(smem_addr(dst)), "l"(src)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// Byte b (0..3) of w, zero-extended.
+__device__ __forceinline__ unsigned byte_of(unsigned w, int b) {
+    return __byte_perm(w, 0u, 0x4440u | (unsigned)b);
+}
+
+}  // namespace qcnn
+#endif

@@ -1,0 +1,153 @@
+"""The C ABI of include/qcnn.h: the library builds, loads and exports every
+declared function, and its host-side argument checks and workspace planning
+work without a GPU (no kernel is launched by these tests)."""
+import ctypes
+
+import pytest
+
+from paper_1512_06473_gb300 import _lib
+import synth
+
+lib = _lib.load()
+
+
+def test_every_declared_symbol_is_exported():
+    names = _lib.header_functions()
+    assert len(names) >= 15
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert missing == []
+    # and the binding knows the signature of each
+    assert sorted(_lib._SIGS) == names
+
+
+def test_status_strings():
+    for s in range(5):
+        assert lib.qcnn_status_string(s)
+    assert lib.qcnn_status_string(99) == b"unknown status"
+
+
+N0 = None  # null device pointer
+
+
+@pytest.mark.parametrize("args", [
+    (8, 10, 4, 3, 16),     # Cs not a multiple of Csp
+    (8, 12, 4, 3, 0),      # K = 0
+    (8, 12, 4, 3, 257),    # K > 256
+    (8, 18, 4, 9, 16),     # Csp > 8
+    (0, 12, 4, 3, 16),     # N = 0
+    (8, 12, 0, 3, 16),     # Ct = 0
+])
+def test_fc_rejects_bad_sizes(args):
+    N, Cs, Ct, Csp, K = args
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_forward(8, N, Cs, Ct, 8, Csp, K, 8, None, 8, 0, None, 0, None) \
+        == _lib.ERR_INVALID_ARG
+
+
+def test_fc_rejects_null_pointers():
+    assert lib.qcnn_fc_forward(None, 2, 8, 4, 8, 4, 16, 8, None, 8, 0, None, 0, None) \
+        == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, None, 4, 16, 8, None, 8, 0, None, 0, None) \
+        == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, None, None, 8, 0, None, 0, None) \
+        == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, 8, None, None, 0, None, 0, None) \
+        == _lib.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("args", [
+    (1, 8, 5, 5, 4, 7, 7, 1, 0, 4, 16),   # kernel larger than the padded map
+    (1, 8, 5, 5, 4, 3, 3, 0, 1, 4, 16),   # stride 0
+    (1, 8, 5, 5, 4, 3, 3, 1, -1, 4, 16),  # negative pad
+    (1, 9, 5, 5, 4, 3, 3, 1, 1, 4, 16),   # Cs % Csp
+    (1, 8, 5, 5, 4, 3, 3, 1, 1, 4, 300),  # K
+])
+def test_conv_rejects_bad_sizes(args):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = args
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, 0, 0,
+                                        ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_conv_forward(8, N, Cs, H, W, Ct, kh, kw, s, p, 8, Csp, K, 8, 0, None, 8, 0, 0,
+                                 None, 0, None) == _lib.ERR_INVALID_ARG
+
+
+def test_conv_bad_enums_and_fused_stride():
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 7, 0,
+                                        ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 9,
+                                        ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    # the fused kernel serves stride 1 only
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 1,
+                                        ctypes.byref(nb)) == _lib.ERR_UNSUPPORTED
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 0,
+                                        ctypes.byref(nb)) == _lib.OK
+
+
+def test_conv_workspace_too_small_is_reported_before_launch():
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 0,
+                                        ctypes.byref(nb)) == _lib.OK
+    assert nb.value > 0  # canonical codes are re-laid out in the workspace
+    assert lib.qcnn_conv_forward(8, 1, 8, 9, 9, 4, 3, 3, 1, 1, 8, 4, 16, 8, 0, None, 8, 0, 0,
+                                 None, 0, None) == _lib.ERR_WORKSPACE
+    # misaligned workspace
+    assert lib.qcnn_conv_forward(8, 1, 8, 9, 9, 4, 3, 3, 1, 1, 8, 4, 16, 8, 0, None, 8, 0, 0,
+                                 4096 + 8, nb.value, None) == _lib.ERR_WORKSPACE
+
+
+def _layers(workload, N=1):
+    arr = (_lib.Layer * len(workload.layers))()
+    for i, L in enumerate(workload.layers):
+        d = arr[i]
+        if isinstance(L, synth.Conv):
+            d.kind, d.Ct, d.kh, d.kw, d.stride, d.pad = 0, L.Ct, L.kh, L.kw, L.stride, L.pad
+            d.Csp, d.K, d.relu = L.Csp, L.K, int(L.relu)
+            d.D, d.codes = 8, 8
+        elif isinstance(L, synth.FC):
+            d.kind, d.Ct, d.Csp, d.K, d.relu = 1, L.Ct, L.Csp, L.K, int(L.relu)
+            d.D, d.codes = 8, 8
+        else:
+            d.kind, d.kh, d.kw, d.stride = 2, L.k, L.k, L.s
+    return arr
+
+
+@pytest.mark.parametrize("name", sorted(synth.WORKLOADS))
+def test_net_shapes_and_workspace(name):
+    w = synth.WORKLOADS[name]
+    if len(w.in_shape) == 1:
+        C, H, W = w.in_shape[0], 1, 1
+    else:
+        C, H, W = w.in_shape
+    arr = _layers(w)
+    oc, oh, ow = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    assert lib.qcnn_net_output_shape(arr, len(arr), C, H, W, ctypes.byref(oc), ctypes.byref(oh),
+                                     ctypes.byref(ow)) == _lib.OK
+    last = w.shapes()[-1][1]
+    assert (oc.value, oh.value, ow.value) == tuple(last) + (1,) * (3 - len(last))
+    for N in w.batches:
+        a, b = ctypes.c_size_t(), ctypes.c_size_t()
+        assert lib.qcnn_net_workspace_size(arr, len(arr), N, C, H, W, 0, ctypes.byref(a)) == 0
+        assert lib.qcnn_net_workspace_size(arr, len(arr), N, C, H, W, 1, ctypes.byref(b)) == 0
+        assert b.value >= a.value + N * C * H * W * 4
+
+
+def test_alexnet_output_is_1000_logits():
+    w = synth.alexnet()
+    arr = _layers(w)
+    oc, oh, ow = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    assert lib.qcnn_net_output_shape(arr, len(arr), 3, 227, 227, ctypes.byref(oc),
+                                     ctypes.byref(oh), ctypes.byref(ow)) == 0
+    assert (oc.value, oh.value, ow.value) == (1000, 1, 1)
+
+
+def test_net_rejects_mismatched_layer():
+    w = synth.alexnet()
+    arr = _layers(w)
+    arr[2].Csp = 5  # conv2 has 96 inputs: 96 % 5 != 0
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_net_workspace_size(arr, len(arr), 1, 3, 227, 227, 0, ctypes.byref(nb)) \
+        == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_net_workspace_size(None, 3, 1, 3, 227, 227, 0, ctypes.byref(nb)) \
+        == _lib.ERR_INVALID_ARG

@@ -1,0 +1,291 @@
+"""CUDA path (through the C ABI) against the float64 oracle, element by element.
+
+Tolerance: max|gpu - oracle| / max|oracle| <= 1e-5 for every fp32 result
+(the bar the method's fp32 path is held to); integer-valued inputs must give
+bit-identical results, since then every partial sum is exact in fp32."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_1512_06473_gb300 as q
+import synth
+
+pytestmark = pytest.mark.gpu
+TOL = 1e-5
+
+
+def rel(got, ref):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    return float(np.max(np.abs(got - ref)) / max(np.max(np.abs(ref)), 1e-30))
+
+
+def cuda(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def conv_case(seed, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=False):
+    M = Cs // Csp
+    if integer:
+        x = synth.small_integers((N, Cs, H, W), -8, 8, seed, 0)
+        D = synth.small_integers((M, K, Csp), -8, 8, seed, 1)
+        b = synth.small_integers((Ct,), -8, 8, seed, 3)
+    else:
+        x = synth.normal((N, Cs, H, W), 1.0, seed, 0)
+        D = synth.normal((M, K, Csp), 0.5, seed, 1)
+        b = synth.normal((Ct,), 0.1, seed, 3)
+    codes = synth.uniform_codes((Ct, kh * kw, M), K, seed, 2)
+    return x, D, codes, b
+
+
+# (N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K)
+CONV_SWEEP = [
+    (1, 4, 5, 5, 3, 3, 3, 1, 1, 4, 5),
+    (2, 8, 13, 13, 40, 3, 3, 1, 1, 4, 128),     # several bands, ragged channel tile
+    (1, 16, 27, 27, 70, 5, 5, 1, 2, 4, 128),    # AlexNet conv2-like, ragged Ct
+    (1, 12, 20, 33, 17, 3, 3, 1, 1, 3, 64),     # Csp = 3, wide map
+    (2, 16, 9, 11, 9, 3, 3, 1, 0, 8, 256),      # K = 256, no padding
+    (1, 8, 7, 7, 5, 1, 1, 1, 0, 2, 16),         # 1x1 kernel
+    (1, 8, 6, 9, 33, 3, 5, 1, 2, 1, 2),         # non-square kernel, Csp = 1
+    (1, 6, 15, 15, 20, 3, 3, 2, 1, 6, 32),      # stride 2
+    (1, 3, 39, 39, 24, 11, 11, 4, 0, 3, 128),   # conv1-like: stride 4, M = 1
+    (1, 8, 1, 1, 4, 1, 1, 1, 0, 4, 1),          # 1x1 map, K = 1
+    (3, 8, 4, 70, 65, 3, 3, 1, 1, 4, 32),       # map wider than one warp slot
+    (1, 8, 58, 3, 16, 3, 3, 1, 1, 8, 16),       # tall, narrow map
+]
+
+
+@pytest.mark.parametrize("case", CONV_SWEEP, ids=lambda c: "x".join(map(str, c)))
+@pytest.mark.parametrize("algo", ["auto", "unfused"])
+def test_conv_sweep(case, algo):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(hash(case) % 1000, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=False)
+    got = q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), algo=algo)
+    assert rel(host(got), ref) <= TOL
+    ref_r = np.maximum(ref, 0)
+    got_r = q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), relu=True, algo=algo)
+    assert rel(host(got_r), ref_r) <= TOL
+
+
+@pytest.mark.parametrize("case", [c for c in CONV_SWEEP if c[7] == 1], ids=lambda c: "x".join(map(str, c)))
+def test_conv_fused_forced(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(7, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b)
+    got = q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), algo="fused")
+    assert rel(host(got), ref) <= TOL
+
+
+@pytest.mark.parametrize("algo", ["fused", "unfused"])
+def test_conv_integer_bit_exact(algo):
+    case = (2, 16, 14, 13, 36, 3, 3, 1, 1, 4, 32)
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(3, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=True)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b)
+    got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), algo=algo))
+    assert np.array_equal(got.astype(np.float64), ref)
+
+
+def test_conv_codeword_renumbering_is_bit_identical():
+    N, Cs, H, W, Ct, kh, kw, Csp, K = 1, 16, 13, 13, 24, 3, 3, 4, 128
+    x, D, codes, b = conv_case(5, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    M = Cs // Csp
+    r = np.random.default_rng(1)
+    perm = np.stack([r.permutation(K) for _ in range(M)])
+    Dp = np.empty_like(D)
+    for m in range(M):
+        Dp[m, perm[m]] = D[m]
+    cp = perm[np.arange(M)[None, None, :], codes.astype(np.int64)].astype(np.uint8)
+    a = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, 1, 1, cuda(b)))
+    c = host(q.conv_forward(cuda(x), cuda(Dp), cuda(cp), kh, kw, 1, 1, cuda(b)))
+    assert np.array_equal(a, c)
+
+
+def test_conv_packed_codes_match_canonical():
+    N, Cs, H, W, Ct, kh, kw, Csp, K = 2, 24, 27, 27, 48, 5, 5, 4, 128
+    x, D, codes, b = conv_case(9, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    packed = q.conv_pack_codes(cuda(codes), K, kh, kw)
+    a = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, 1, 2, cuda(b)))
+    c = host(q.conv_forward(cuda(x), cuda(D), packed, kh, kw, 1, 2, cuda(b), packed=True, Ct=Ct))
+    assert np.array_equal(a, c)
+
+
+def test_conv_is_deterministic():
+    N, Cs, H, W, Ct, kh, kw, Csp, K = 2, 32, 27, 27, 64, 5, 5, 4, 128
+    x, D, codes, b = conv_case(11, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    a = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, 1, 2, cuda(b)))
+    c = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, 1, 2, cuda(b)))
+    assert np.array_equal(a, c)
+
+
+def test_out_of_range_codes_are_clamped_not_faulting():
+    """Codes >= K are a caller error; the kernels clamp them to K - 1, so the
+    result equals the one with clamped codes (and no access leaves the table)."""
+    N, Cs, H, W, Ct, kh, kw, Csp, K = 1, 8, 9, 9, 16, 3, 3, 4, 100
+    x, D, codes, b = conv_case(13, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    bad = codes.copy()
+    bad[::3, ::2, :] = 255
+    good = np.minimum(bad, K - 1).astype(np.uint8)
+    for algo in ("fused", "unfused"):
+        a = host(q.conv_forward(cuda(x), cuda(D), cuda(bad), kh, kw, 1, 1, cuda(b), algo=algo))
+        c = host(q.conv_forward(cuda(x), cuda(D), cuda(good), kh, kw, 1, 1, cuda(b), algo=algo))
+        assert np.array_equal(a, c)
+    xf = synth.normal((3, 32), 1.0, 1)
+    Df = synth.normal((8, 20, 4), 1.0, 2)
+    cf = np.full((8, 10), 200, np.uint8)
+    a = host(q.fc_forward(cuda(xf), cuda(Df), cuda(cf)))
+    c = host(q.fc_forward(cuda(xf), cuda(Df), cuda(np.full((8, 10), 19, np.uint8))))
+    assert np.array_equal(a, c)
+
+
+# (N, Cs, Ct, Csp, K)
+FC_SWEEP = [
+    (1, 4, 3, 4, 5),
+    (8, 512, 256, 4, 16),       # the single-layer FC workload
+    (3, 96, 7, 3, 32),          # Ct not a multiple of 4
+    (33, 128, 1030, 4, 32),     # ragged image and output tiles
+    (2, 64, 100, 8, 256),       # K = 256 (bank conflicts, still exact)
+    (5, 40, 64, 1, 2),          # Csp = 1
+    (70, 2304, 513, 4, 32),     # many chunks, splits
+    (1, 9216, 4096, 4, 32),     # fc6 at batch 1
+]
+
+
+@pytest.mark.parametrize("case", FC_SWEEP, ids=lambda c: "x".join(map(str, c)))
+def test_fc_sweep(case):
+    N, Cs, Ct, Csp, K = case
+    M = Cs // Csp
+    x = synth.normal((N, Cs), 1.0, 20, *case)
+    D = synth.normal((M, K, Csp), 0.5, 21, *case)
+    codes = synth.uniform_codes((M, Ct), K, 22, *case)
+    b = synth.normal((Ct,), 0.1, 23, *case)
+    for relu in (False, True):
+        ref = oracle.fc_forward(x, D, codes, b, relu)
+        got = q.fc_forward(cuda(x), cuda(D), cuda(codes), cuda(b), relu=relu)
+        assert rel(host(got), ref) <= TOL
+
+
+def test_fc_integer_bit_exact():
+    N, Cs, Ct, Csp, K = 17, 256, 300, 4, 32
+    M = Cs // Csp
+    x = synth.small_integers((N, Cs), -8, 8, 30)
+    D = synth.small_integers((M, K, Csp), -8, 8, 31)
+    codes = synth.uniform_codes((M, Ct), K, 32)
+    b = synth.small_integers((Ct,), -8, 8, 33)
+    ref = oracle.fc_forward(x, D, codes, b)
+    got = host(q.fc_forward(cuda(x), cuda(D), cuda(codes), cuda(b)))
+    assert np.array_equal(got.astype(np.float64), ref)
+
+
+@pytest.mark.parametrize("shape", [(2, 8, 5, 7, 4, 16), (1, 12, 1, 1, 3, 5), (3, 16, 9, 9, 8, 128),
+                                   (1, 6, 4, 4, 2, 256)])
+def test_lut_build(shape):
+    N, Cs, H, W, Csp, K = shape
+    M = Cs // Csp
+    x = synth.normal((N, Cs, H, W), 1.0, 40, *shape)
+    D = synth.normal((M, K, Csp), 1.0, 41, *shape)
+    ref = oracle.conv_lut(x, D)
+    got = host(q.lut_build(cuda(x), cuda(D)))
+    assert rel(got, ref) <= TOL
+    xf = x[:, :, 0, 0].copy()
+    assert rel(host(q.lut_build(cuda(xf), cuda(D))), oracle.fc_lut(xf, D)[:, :, None, :]) <= TOL
+
+
+@pytest.mark.parametrize("shape", [(2, 3, 55, 55, 3, 2), (1, 5, 13, 13, 3, 2), (1, 4, 8, 9, 2, 2)])
+def test_maxpool(shape):
+    N, C, H, W, k, s = shape
+    x = synth.normal((N, C, H, W), 1.0, 50, *shape)
+    assert np.array_equal(host(q.maxpool(cuda(x), k, s)).astype(np.float64), oracle.maxpool(x, k, s))
+
+
+# ---------------------------------------------------------------- networks
+def build_net(w, params, packed=False):
+    layers = []
+    for L, P in zip(w.layers, params):
+        if isinstance(L, synth.Conv):
+            codes = cuda(P["codes"])
+            if packed:
+                codes = q.conv_pack_codes(codes, L.K, L.kh, L.kw)
+            layers.append(q.ConvLayer(cuda(P["D"]), codes, cuda(P["bias"]), L.Ct, L.kh, L.kw,
+                                      L.stride, L.pad, L.relu, packed=packed))
+        elif isinstance(L, synth.FC):
+            layers.append(q.FCLayer(cuda(P["D"]), cuda(P["codes"]), cuda(P["bias"]), L.relu))
+        else:
+            layers.append(q.PoolLayer(L.k, L.s))
+    in_shape = tuple(w.in_shape) if len(w.in_shape) == 3 else (w.in_shape[0], 1, 1)
+    return q.Net(layers, in_shape)
+
+
+def oracle_layers(w, params):
+    return [synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, params)]
+
+
+def run_workload(name, N, sample):
+    w = synth.WORKLOADS[name]
+    params = w.params()
+    x = w.input(N)
+    net = build_net(w, params, packed=True)
+    xin = x if x.ndim == 4 else x.reshape(N, -1, 1, 1)
+    got = host(net.forward(cuda(xin)))
+    ol = oracle_layers(w, params)
+    ref = oracle.net_forward(x[sample], ol)
+    got_s = got[sample].reshape(ref.shape)
+    return rel(got_s, ref)
+
+
+@pytest.mark.parametrize("name,N,sample", [
+    ("fc_512x256_b8", 8, slice(None)),
+    ("conv3x3_64x56x56_b1", 1, slice(None)),
+    ("vgg16_conv_stack", 1, slice(None)),
+    ("alexnet_fc678", 1, slice(None)),
+    ("alexnet_fc678", 64, [0, 31, 63]),
+    ("alexnet_qcnn", 1, slice(None)),
+])
+def test_workload(name, N, sample):
+    assert run_workload(name, N, sample) <= TOL
+
+
+def test_vgg_stack_batch32_sampled():
+    assert run_workload("vgg16_conv_stack", 32, [0, 17, 31]) <= TOL
+
+
+def test_fc678_batch256_sampled():
+    assert run_workload("alexnet_fc678", 256, [0, 100, 255]) <= TOL
+
+
+def test_alexnet_batch128_bench_launch_sampled():
+    """The benchmark's launch configuration: AlexNet-shaped Q-CNN at batch 128
+    with packed codes; images 0, 64 and 127 against the oracle."""
+    assert run_workload("alexnet_qcnn", 128, [0, 64, 127]) <= TOL
+
+
+def test_net_forward_host_matches_device():
+    w = synth.alexnet()
+    params = w.params()
+    net = build_net(w, params, packed=True)
+    N = 4
+    x = w.input(N, 5)
+    dev = host(net.forward(cuda(x)))
+    xh = torch.from_numpy(x).pin_memory()
+    yh = torch.empty((N, 1000), dtype=torch.float32).pin_memory()
+    ws = net.alloc_workspace(N, host_io=True)
+    net.forward_host(xh, yh, ws)
+    assert np.array_equal(yh.numpy(), dev)
+
+
+def test_launch_counter_counts_kernels():
+    x = cuda(synth.normal((2, 32), 1.0, 1))
+    D = cuda(synth.normal((8, 16, 4), 1.0, 2))
+    c = cuda(synth.uniform_codes((8, 12), 16, 3))
+    before = q.launch_count()
+    q.fc_forward(x, D, c)
+    torch.cuda.synchronize()
+    assert q.launch_count() > before
