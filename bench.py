@@ -49,17 +49,27 @@ def parse():
 
 
 # ----------------------------------------------------------------- oracle
+_CACHE = {}
+
+
+def _workload_cache(batch):
+    """Per-process copy of the workload's parameters and input batch."""
+    if _CACHE.get("batch") != batch:
+        w = synth.WORKLOADS[WORKLOAD]
+        params = w.params()
+        _CACHE.update(batch=batch, x=w.input(batch),
+                      layers=[synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, params)])
+    return _CACHE
+
+
 def _oracle_worker(args):
     """Run the float64 oracle on image `i` of the workload (spawned process)."""
     i, batch = args
     sys.path.insert(0, ROOT)
     import oracle as orc
-    w = synth.WORKLOADS[WORKLOAD]
-    params = w.params()
-    layers = [synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, params)]
-    x = w.input(batch)[i:i + 1]
+    c = _workload_cache(batch)
     t = time.perf_counter()
-    orc.net_forward(x, layers)
+    orc.net_forward(c["x"][i:i + 1], c["layers"])
     return time.perf_counter() - t
 
 
@@ -75,26 +85,28 @@ def _cpu_info():
     return model
 
 
-def oracle_pool(cores):
+def oracle_pool(cores, batch):
     import oracle as orc
     orc.build()
     ctx = mp.get_context("spawn")
     pool = ctx.Pool(cores)
-    pool.map(_oracle_ping, range(cores))
+    pool.map(_oracle_ping, [batch] * cores, chunksize=1)
     return pool
 
 
-def _oracle_ping(_):
+def _oracle_ping(batch):
     sys.path.insert(0, ROOT)
-    import oracle as orc  # noqa: F401
+    import oracle as orc
     orc.default()
+    _workload_cache(batch)
+    time.sleep(0.5)  # keep every worker busy so each one gets a ping
     return 0
 
 
 def time_oracle(pool, cores, sample, batch):
     """Wall time of `sample` images through the oracle on `cores` processes."""
     t = time.perf_counter()
-    pool.map(_oracle_worker, [(i % batch, batch) for i in range(sample)])
+    pool.map(_oracle_worker, [(i % batch, batch) for i in range(sample)], chunksize=1)
     return time.perf_counter() - t
 
 
@@ -103,7 +115,7 @@ def reference_arm(a):
     if rank != 0:
         return 0
     cores = min(os.cpu_count() or 1, 16)
-    pool = oracle_pool(cores)
+    pool = oracle_pool(cores, a.batch)
     sample = cores
     for _ in range(a.warmup):
         time_oracle(pool, cores, sample, a.batch)
@@ -208,7 +220,7 @@ def main():
     pool = None
     cores = min(os.cpu_count() or 1, 16)
     if rank == 0 and world == 1 and not a.no_cpu_baseline:
-        pool = oracle_pool(cores)
+        pool = oracle_pool(cores, a.batch)
 
     import torch
     import torch.distributed as dist
