@@ -107,6 +107,31 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
                             void *stream);
 
 /*
+ * qcnn_fc_forward_noalloc -- the same result as qcnn_fc_forward, for callers
+ * that cannot hand the library any device memory: code running inside
+ * another runtime's execution step, where that runtime owns all device
+ * memory and forbids allocation, or a foreign-function caller with no device
+ * allocator.  The paper has no counterpart; it is a deployment convenience.
+ *   Scratch: a fixed array of QCNN_FC_NOALLOC_SCRATCH_BYTES compiled into
+ *   the library, held in the memory of every GPU that loads it until the
+ *   process exits.  The call allocates nothing.  The first call on each
+ *   device looks up the array's device address (cudaGetSymbolAddress), so
+ *   make that first call before any stream capture.
+ *   Limit: when qcnn_fc_workspace_size(...) for these sizes exceeds
+ *   QCNN_FC_NOALLOC_SCRATCH_BYTES the call returns QCNN_ERR_WORKSPACE and
+ *   enqueues nothing.
+ *   All calls share the array: calls that overlap on the GPU (different
+ *   streams or host threads without ordering) race and give wrong results.
+ *   Nothing in it needs clearing: each call writes what it reads back.
+ * Arguments, layouts and other errors are those of qcnn_fc_forward.
+ */
+#define QCNN_FC_NOALLOC_SCRATCH_BYTES (16u << 20)
+qcnn_status qcnn_fc_forward_noalloc(const float *x, int N, int Cs, int Ct,
+                                    const float *D, int Csp, int K,
+                                    const uint8_t *codes, const float *bias,
+                                    float *y, int relu, void *stream);
+
+/*
  * qcnn_conv_pack_codes -- re-layout conv codes once, at model-load time,
  * for the fused kernels: packed[m][pk][ct] (ct padded with code 0 to a
  * multiple of 256), every code clamped into [0, K).

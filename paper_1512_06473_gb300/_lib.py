@@ -40,6 +40,8 @@ _SIGS = {
     "qcnn_fc_workspace_size": (c_int, [c_int, c_int, c_int, c_int, c_int, ctypes.POINTER(c_size_t)]),
     "qcnn_fc_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
                                 c_void_p, c_void_p, c_int, c_void_p, c_size_t, c_void_p]),
+    "qcnn_fc_forward_noalloc": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int,
+                                        c_void_p, c_void_p, c_void_p, c_int, c_void_p]),
     "qcnn_conv_packed_codes_bytes": (c_size_t, [c_int, c_int, c_int, c_int]),
     "qcnn_conv_pack_codes": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_void_p,
                                      c_void_p]),
