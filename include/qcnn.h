@@ -55,9 +55,11 @@ typedef enum {
 } qcnn_status;
 
 typedef enum {
-    QCNN_ALGO_AUTO = 0,    /* library picks (fused whenever it applies)       */
-    QCNN_ALGO_FUSED = 1,   /* table tile built in shared memory, stride 1 only */
-    QCNN_ALGO_UNFUSED = 2  /* tables materialised in the workspace first      */
+    QCNN_ALGO_AUTO = 0,    /* library picks: fused, else chunked, else unfused */
+    QCNN_ALGO_FUSED = 1,   /* full table rows of a band in shared memory, stride 1 only */
+    QCNN_ALGO_UNFUSED = 2, /* tables materialised in the workspace first      */
+    QCNN_ALGO_CHUNKED = 3  /* table rows built KC sub-codewords at a time in
+                              shared memory, any stride                      */
 } qcnn_algo;
 
 typedef enum {

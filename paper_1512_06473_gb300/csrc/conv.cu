@@ -71,7 +71,6 @@ struct ConvFusedArgs {
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
 };
 
-constexpr int kFusedThreads = 256;
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned).
 struct FusedSmem {
@@ -114,8 +113,10 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // CTW   : output channels per warp
 // WP    : warps along positions (8 / WP warps along channels)
 // CSP4  : C'_s rounded up to 4 or 8 (register width of one sub-vector)
-template <int P, int CTW, int WP, int CSP4>
-__global__ void __launch_bounds__(kFusedThreads, 2) conv_fused_kernel(const ConvFusedArgs a) {
+// NW    : warps per CTA (8 or 16)
+template <int P, int CTW, int WP, int CSP4, int NW>
+__global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(const ConvFusedArgs a) {
+    constexpr int kFusedThreads = NW * 32;
     constexpr int QB = 16 / CSP4;  // sub-codewords per lane per build pass
     extern __shared__ __align__(16) unsigned char smem[];
     const FusedSmem L = fused_smem_layout(a.K, a.KS, a.xs_floats, CSP4, a.kh * a.kw, a.ct_cta);
@@ -184,7 +185,7 @@ __global__ void __launch_bounds__(kFusedThreads, 2) conv_fused_kernel(const Conv
         {
             const float *xb = xs + b * a.xs_floats;
             const float *db = ds + b * K * CSP4;
-            const int hpw = cdiv(HP, 8);
+            const int hpw = cdiv(HP, NW);
             const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
             for (int q0 = 0; q0 < K; q0 += 32 * QB) {
                 float dk[QB][CSP4];
@@ -270,14 +271,16 @@ __global__ void __launch_bounds__(kFusedThreads, 2) conv_fused_kernel(const Conv
 
 // ---------------------------------------------------------- variant table --
 struct FusedVariant {
-    int P, CTW, WP, CSP4;
+    int P, CTW, WP, CSP4, NW;
     void (*fn)(ConvFusedArgs);
 };
 
-#define QCNN_FUSED(P, CTW, WP, C4) {P, CTW, WP, C4, conv_fused_kernel<P, CTW, WP, C4>}
+#define QCNN_FUSED(P, CTW, WP, C4, NW) {P, CTW, WP, C4, NW, conv_fused_kernel<P, CTW, WP, C4, NW>}
 static const FusedVariant kFused[] = {
-    QCNN_FUSED(2, 32, 1, 4), QCNN_FUSED(4, 16, 1, 4), QCNN_FUSED(4, 8, 2, 4),
-    QCNN_FUSED(2, 32, 1, 8), QCNN_FUSED(4, 16, 1, 8), QCNN_FUSED(4, 8, 2, 8),
+    QCNN_FUSED(2, 32, 1, 4, 8),  QCNN_FUSED(4, 16, 1, 4, 8),  QCNN_FUSED(4, 8, 2, 4, 8),
+    QCNN_FUSED(2, 32, 1, 8, 8),  QCNN_FUSED(4, 16, 1, 8, 8),  QCNN_FUSED(4, 8, 2, 8, 8),
+    QCNN_FUSED(4, 16, 1, 4, 16), QCNN_FUSED(4, 16, 2, 4, 16), QCNN_FUSED(2, 32, 2, 4, 16),
+    QCNN_FUSED(4, 16, 1, 8, 16), QCNN_FUSED(4, 16, 2, 8, 16), QCNN_FUSED(2, 32, 2, 8, 16),
 };
 #undef QCNN_FUSED
 constexpr int kNumFused = sizeof(kFused) / sizeof(kFused[0]);
@@ -317,7 +320,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         TH = cdiv(s.Ho, row_tiles);  // balance the bands
         const int HP = (TH + s.kh - 1) * pitch;
         const int KS = ks_for(slots * 32 + (s.kh - 1) * pitch + (s.kw - 1));
-        const int ct_cta = (8 / fv.WP) * fv.CTW;
+        const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
         const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta).total;
         if (smem > (size_t)smem_optin) continue;
@@ -329,7 +332,9 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const double gather = (double)slots * ct_cta * kk * s.M;
         const double build = (double)HP * s.K * s.M * 1.5 / 32.0;
         const double per_cta = gather + build;
-        const double score = waves * per_cta / cps * (cps == 1 ? 1.15 : 1.0);
+        // fewer than 16 resident warps per SM leave the gather latency bound
+        const int warps_sm = cps * fv.NW;
+        const double score = waves * per_cta / cps * (warps_sm < 16 ? 1.4 : 1.0);
         if (!best.ok || score < best.score) {
             best.ok = true;
             best.variant = v;
@@ -385,7 +390,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
     dim3 grid(p.row_tiles, p.ct_tiles, s.N);
-    fv.fn<<<grid, kFusedThreads, p.smem, st>>>(a);
+    fv.fn<<<grid, fv.NW * 32, p.smem, st>>>(a);
     return after_launch();
 }
 

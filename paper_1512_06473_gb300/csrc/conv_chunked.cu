@@ -1,0 +1,336 @@
+// conv_chunked.cu -- PQ conv response (Eq. 7) for layers whose table rows do
+// not fit shared memory whole: any stride, any kernel size, K up to 256.
+// Built for AlexNet conv1 (11x11, stride 4, one sub-space of C'_s = 3,
+// K = 128), where the K-entry table of every input position of a band of
+// output rows would need ~1.5 MB.
+//
+// One CTA owns an image, a band of TH output rows (all columns) and CT_CTA
+// output channels.  For each sub-space m and each chunk of KC sub-codewords
+// [k0, k0 + KC) it
+//   1. builds the chunk's table of every input position the band reads, in
+//      a stride-phase-split layout  lut[kl][ay][ax][r][c]  with
+//      iy = (oy0 + r + dymin)*s + ay,  ix = (c + dxmin)*s + ax,
+//      so that for a fixed kernel offset the 32 lanes of a warp (consecutive
+//      output columns) read 32 consecutive words: conflict free;
+//   2. gathers only the (c_t, p_k) pairs whose code lies in the chunk.  Those
+//      pairs come from per-(m, c_t) entry lists, counting-sorted by chunk in
+//      the workspace by a small prep kernel, each entry being the ready
+//      shared-memory offset  kl*SK + phase*PS + (dy - dymin)*PW + (dx - dxmin).
+// A lane owns P positions of the band's output grid of pitch PW
+// (l = r*PW + c, columns c >= Wo are discarded) and CTW channels; its input
+// sub-vectors (QPT positions x CSPT channels) stay in registers across the
+// chunks of a sub-space.
+#include "qcnn_internal.cuh"
+
+#include <algorithm>
+
+namespace qcnn {
+
+constexpr int kChunkThreads = 512;
+
+struct ChunkGeom {
+    int s, pad, kh, kw, TH, PR, PW, PS, SK, NQ, dymin, dymax, dxmin, dxmax, KC, NCH;
+};
+
+__host__ __device__ inline int floor_div(int a, int b) {
+    return (a >= 0) ? a / b : -((-a + b - 1) / b);
+}
+
+// Shared-memory offset of kernel offset (ky, kx) inside one table row.
+__host__ __device__ inline int chunk_phase_off(const ChunkGeom &g, int ky, int kx) {
+    const int ty = ky - g.pad, tx = kx - g.pad;
+    const int dy = floor_div(ty, g.s), dx = floor_div(tx, g.s);
+    const int ay = ty - dy * g.s, ax = tx - dx * g.s;
+    return (ay * g.s + ax) * g.PS + (dy - g.dymin) * g.PW + (dx - g.dxmin);
+}
+
+// ------------------------------------------------------------------ prep --
+// One thread per (m, ct): entries[m][ct][*] = offsets sorted by chunk,
+// starts[m][ct][c] = first entry of chunk c (NCH + 1 values).
+__global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed, int CtP,
+                                  int Ct, int kk, int M, int K, ChunkGeom g,
+                                  uint32_t *__restrict__ entries, int *__restrict__ starts) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= M * Ct) return;
+    const int m = i / Ct, ct = i % Ct;
+    auto code_at = [&](int pk) -> int {
+        const int c = packed ? codes[((size_t)m * kk + pk) * CtP + ct]
+                             : codes[((size_t)ct * kk + pk) * M + m];
+        return min(c, K - 1);
+    };
+    int *st = starts + (size_t)i * (g.NCH + 1);
+    for (int c = 0; c <= g.NCH; ++c) st[c] = 0;
+    for (int pk = 0; pk < kk; ++pk) st[code_at(pk) / g.KC + 1] += 1;
+    for (int c = 0; c < g.NCH; ++c) st[c + 1] += st[c];
+    uint32_t *en = entries + (size_t)i * kk;
+    // stable placement: a second pass per chunk keeps p_k order inside a chunk
+    for (int c = 0; c < g.NCH; ++c) {
+        int pos = st[c];
+        for (int pk = 0; pk < kk; ++pk) {
+            const int code = code_at(pk);
+            if (code / g.KC != c) continue;
+            const int ky = pk / g.kw, kx = pk % g.kw;
+            en[pos++] = (uint32_t)((code - c * g.KC) * g.SK + chunk_phase_off(g, ky, kx));
+        }
+    }
+}
+
+// ---------------------------------------------------------------- kernel --
+struct ChunkArgs {
+    const float *__restrict__ x;
+    const float *__restrict__ D;
+    const uint32_t *__restrict__ entries;
+    const int *__restrict__ starts;
+    const float *__restrict__ bias;
+    float *__restrict__ y;
+    int N, Cs, H, W, Ct, Csp, K, M, Ho, Wo, kk, ct_cta, relu;
+    ChunkGeom g;
+};
+
+template <int P, int CTW, int QPT, int CSPT>
+__global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const ChunkArgs a) {
+    extern __shared__ __align__(16) float csm[];
+    const ChunkGeom &g = a.g;
+    float *lut = csm;                            // [KC][SK]
+    float *ds = csm + (size_t)g.KC * g.SK;       // [K][CSPT]
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int oy0 = blockIdx.x * g.TH;
+    const int ct0 = blockIdx.y * a.ct_cta;
+    const int n = blockIdx.z;
+    const int ctw0 = ct0 + warp * CTW;
+
+    float acc[CTW][P];
+#pragma unroll
+    for (int c = 0; c < CTW; ++c)
+#pragma unroll
+        for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
+
+    for (int m = 0; m < a.M; ++m) {
+        __syncthreads();  // previous sub-space finished with ds and lut
+        for (int e = tid; e < a.K * CSPT; e += kChunkThreads) {
+            const int k = e / CSPT, j = e % CSPT;
+            ds[e] = j < a.Csp ? __ldg(a.D + ((size_t)m * a.K + k) * a.Csp + j) : 0.f;
+        }
+        // this thread's input sub-vectors, kept for every chunk of m
+        float xr[QPT][CSPT];
+#pragma unroll
+        for (int qi = 0; qi < QPT; ++qi) {
+            const int q = tid + qi * kChunkThreads;
+            const int phase = q / g.PS, rem = q - phase * g.PS;
+            const int r = rem / g.PW, c = rem - r * g.PW;
+            const int ay = phase / g.s, ax = phase - ay * g.s;
+            const int iy = (oy0 + r + g.dymin) * g.s + ay, ix = (c + g.dxmin) * g.s + ax;
+            const bool ok = q < g.NQ && iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+            const float *xp = a.x + (((size_t)n * a.Cs + (size_t)m * a.Csp) * a.H +
+                                     (ok ? iy : 0)) * a.W + (ok ? ix : 0);
+#pragma unroll
+            for (int j = 0; j < CSPT; ++j) {
+                const float v = __ldg(xp + (size_t)min(j, a.Csp - 1) * a.H * a.W);
+                xr[qi][j] = (ok && j < a.Csp) ? v : 0.f;
+            }
+        }
+        __syncthreads();  // ds ready
+
+        const int *st = a.starts;
+        const uint32_t *en = a.entries;
+        for (int ch = 0; ch < g.NCH; ++ch) {
+            const int k0 = ch * g.KC, kc = min(g.KC, a.K - k0);
+            // ---- build the chunk's table rows (one codeword at a time, so its
+            // components are read once per thread and reused for QPT positions)
+            for (int kl = 0; kl < kc; ++kl) {
+                float dk[CSPT];
+#pragma unroll
+                for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
+                float *row = lut + kl * g.SK;
+#pragma unroll
+                for (int qi = 0; qi < QPT; ++qi) {
+                    const int q = tid + qi * kChunkThreads;
+                    float v = 0.f;
+#pragma unroll
+                    for (int j = 0; j < CSPT; ++j) v = fmaf(xr[qi][j], dk[j], v);
+                    if (q < g.NQ) row[q] = v;
+                }
+            }
+            __syncthreads();
+            // ---- gather the pairs whose code is in this chunk
+#pragma unroll
+            for (int c = 0; c < CTW; ++c) {
+                const int ct = ctw0 + c;
+                if (ct < a.Ct) {
+                    const size_t row = (size_t)m * a.Ct + ct;
+                    const int e0 = __ldg(st + row * (g.NCH + 1) + ch);
+                    const int e1 = __ldg(st + row * (g.NCH + 1) + ch + 1);
+                    const uint32_t *ep = en + row * a.kk;
+#pragma unroll 2
+                    for (int e = e0; e < e1; ++e) {
+                        const float *base = lut + lane + __ldg(ep + e);
+#pragma unroll
+                        for (int p = 0; p < P; ++p) acc[c][p] += base[p * 32];
+                    }
+                }
+            }
+            __syncthreads();  // table rows free for the next chunk
+        }
+    }
+
+    // ---- epilogue
+#pragma unroll
+    for (int c = 0; c < CTW; ++c) {
+        const int ct = ctw0 + c;
+        if (ct >= a.Ct) continue;
+        const float bv = a.bias ? a.bias[ct] : 0.f;
+#pragma unroll
+        for (int p = 0; p < P; ++p) {
+            const int l = p * 32 + lane;
+            const int r = l / g.PW, col = l - r * g.PW;
+            const int oy = oy0 + r;
+            if (r < g.TH && col < a.Wo && oy < a.Ho) {
+                float v = acc[c][p] + bv;
+                if (a.relu) v = fmaxf(v, 0.f);
+                a.y[(((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + col] = v;
+            }
+        }
+    }
+}
+
+struct ChunkVariant {
+    int P, CTW, QPT, CSPT;
+    void (*fn)(ChunkArgs);
+};
+#define QCNN_CHUNK(P, CTW, QPT, C) {P, CTW, QPT, C, conv_chunked_kernel<P, CTW, QPT, C>}
+static const ChunkVariant kChunk[] = {
+    QCNN_CHUNK(8, 6, 11, 3),   // AlexNet conv1: 4 rows of 57, 96 channels
+    QCNN_CHUNK(8, 8, 8, 4),
+    QCNN_CHUNK(4, 8, 4, 8),
+};
+#undef QCNN_CHUNK
+constexpr int kNumChunk = sizeof(kChunk) / sizeof(kChunk[0]);
+
+static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P) {
+    ChunkGeom g;
+    g.s = s.stride;
+    g.pad = s.pad;
+    g.kh = s.kh;
+    g.kw = s.kw;
+    g.TH = TH;
+    g.dymin = floor_div(-s.pad, s.stride);
+    g.dymax = floor_div(s.kh - 1 - s.pad, s.stride);
+    g.dxmin = floor_div(-s.pad, s.stride);
+    g.dxmax = floor_div(s.kw - 1 - s.pad, s.stride);
+    g.PR = TH + g.dymax - g.dymin;
+    g.PW = s.Wo + g.dxmax - g.dxmin;
+    g.PS = g.PR * g.PW;
+    g.NQ = s.stride * s.stride * g.PS;
+    int sk = (s.stride * s.stride - 1) * g.PS + (g.dymax - g.dymin) * g.PW + (g.dxmax - g.dxmin) +
+             P * 32;
+    sk = std::max(sk, g.NQ);
+    while (sk % 32 != 1) ++sk;
+    g.SK = sk;
+    g.KC = KC;
+    g.NCH = cdiv(s.K, KC);
+    return g;
+}
+
+ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
+    ConvChunkPlan best;
+    const int sms = num_sms();
+    int dev = 0, smem_optin = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess || smem_optin <= 0) {
+        cudaGetLastError();
+        smem_optin = 227 * 1024;
+    }
+    for (int v = 0; v < kNumChunk; ++v) {
+        const ChunkVariant &cv = kChunk[v];
+        if (s.Csp > cv.CSPT) continue;
+        const int ct_cta = 16 * cv.CTW;
+        // largest band that the variant's lanes cover
+        for (int TH = std::min(s.Ho, 64); TH >= 1; --TH) {
+            const ChunkGeom g0 = chunk_geom(s, TH, 1, cv.P);
+            if (TH * g0.PW > cv.P * 32) continue;
+            if (g0.NQ > cv.QPT * kChunkThreads) continue;
+            // balance the bands
+            const int row_tiles = cdiv(s.Ho, TH);
+            const int th = cdiv(s.Ho, row_tiles);
+            for (int KC : {16, 8, 4, 2, 1}) {
+                if (KC > s.K) continue;
+                const ChunkGeom g = chunk_geom(s, th, KC, cv.P);
+                const size_t smem = ((size_t)KC * g.SK + (size_t)s.K * cv.CSPT) * sizeof(float);
+                if (smem > (size_t)smem_optin) continue;
+                const int ct_tiles = cdiv(s.Ct, ct_cta);
+                const double ctas = (double)s.N * row_tiles * ct_tiles;
+                const double waves = std::ceil(ctas / sms);
+                // per CTA: gather wavefronts + table stores, per sub-space
+                const double gather = (double)cv.P * ct_cta * s.kh * s.kw;
+                const double build = (double)g.NQ * s.K / 32.0 + (double)g.NCH * 400.0;
+                const double score = waves * (gather + build) * s.M;
+                if (!best.ok || score < best.score) {
+                    best.ok = true;
+                    best.variant = v;
+                    best.g_TH = th;
+                    best.KC = KC;
+                    best.ct_cta = ct_cta;
+                    best.row_tiles = row_tiles;
+                    best.ct_tiles = ct_tiles;
+                    best.smem = smem;
+                    best.score = score;
+                }
+                break;  // largest KC that fits
+            }
+            break;  // largest TH that fits
+        }
+    }
+    if (best.ok) {
+        const ChunkGeom g = chunk_geom(s, best.g_TH, best.KC, kChunk[best.variant].P);
+        best.NCH = g.NCH;
+        best.entries_bytes = align_up((size_t)s.M * s.Ct * s.kh * s.kw * 4, kWsAlign);
+        best.starts_bytes = align_up((size_t)s.M * s.Ct * (g.NCH + 1) * 4, kWsAlign);
+    }
+    return best;
+}
+
+qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, const float *x,
+                                const float *D, const uint8_t *codes, int codes_packed,
+                                const float *bias, float *y, int relu, void *ws,
+                                cudaStream_t st) {
+    const ChunkVariant &cv = kChunk[p.variant];
+    const ChunkGeom g = chunk_geom(s, p.g_TH, p.KC, cv.P);
+    uint32_t *entries = static_cast<uint32_t *>(ws);
+    int *starts = reinterpret_cast<int *>(static_cast<uint8_t *>(ws) + p.entries_bytes);
+    const int kk = s.kh * s.kw;
+    const int nthreads = s.M * s.Ct;
+    chunk_prep_kernel<<<cdiv(nthreads, 128), 128, 0, st>>>(codes, codes_packed, packed_ct(s.Ct),
+                                                          s.Ct, kk, s.M, s.K, g, entries, starts);
+    qcnn_status rc = after_launch();
+    if (rc != QCNN_OK) return rc;
+    ChunkArgs a;
+    a.x = x;
+    a.D = D;
+    a.entries = entries;
+    a.starts = starts;
+    a.bias = bias;
+    a.y = y;
+    a.N = s.N;
+    a.Cs = s.Cs;
+    a.H = s.H;
+    a.W = s.W;
+    a.Ct = s.Ct;
+    a.Csp = s.Csp;
+    a.K = s.K;
+    a.M = s.M;
+    a.Ho = s.Ho;
+    a.Wo = s.Wo;
+    a.kk = kk;
+    a.ct_cta = p.ct_cta;
+    a.relu = relu;
+    a.g = g;
+    cudaError_t e =
+        cudaFuncSetAttribute(cv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    if (e != cudaSuccess) return cuda_status(e);
+    dim3 grid(p.row_tiles, p.ct_tiles, s.N);
+    cv.fn<<<grid, kChunkThreads, p.smem, st>>>(a);
+    return after_launch();
+}
+
+}  // namespace qcnn

@@ -84,8 +84,9 @@ bool fc_shape(int N, int Cs, int Ct, int Csp, int K, FcShape *s) {
 // ------------------------------------------------------------ conv plan ---
 struct ConvCall {
     ConvShape s;
-    bool fused;
+    int algo;  // resolved: FUSED, CHUNKED or UNFUSED
     ConvFusedPlan fp;
+    ConvChunkPlan cp;
     ConvUnfusedPlan up;
     size_t packed_off, lut_off, total;
 };
@@ -93,22 +94,33 @@ struct ConvCall {
 qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvCall *c) {
     if (codes_layout != QCNN_CODES_CANONICAL && codes_layout != QCNN_CODES_PACKED)
         return QCNN_ERR_INVALID_ARG;
-    if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED)
+    if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED &&
+        algo != QCNN_ALGO_CHUNKED)
         return QCNN_ERR_INVALID_ARG;
     c->s = s;
-    c->fused = false;
-    if (algo != QCNN_ALGO_UNFUSED) {
+    c->algo = QCNN_ALGO_UNFUSED;
+    if (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_FUSED) {
         c->fp = plan_conv_fused(s);
-        c->fused = c->fp.ok;
-        if (algo == QCNN_ALGO_FUSED && !c->fused) return QCNN_ERR_UNSUPPORTED;
+        if (c->fp.ok) c->algo = QCNN_ALGO_FUSED;
+        else if (algo == QCNN_ALGO_FUSED) return QCNN_ERR_UNSUPPORTED;
     }
-    if (!c->fused) c->up = plan_conv_unfused(s);
+    if (c->algo == QCNN_ALGO_UNFUSED && (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_CHUNKED)) {
+        c->cp = plan_conv_chunked(s);
+        if (c->cp.ok) c->algo = QCNN_ALGO_CHUNKED;
+        else if (algo == QCNN_ALGO_CHUNKED) return QCNN_ERR_UNSUPPORTED;
+    }
     size_t off = 0;
     c->packed_off = off;
-    if (codes_layout == QCNN_CODES_CANONICAL)
+    // the chunked path reads either code layout directly
+    if (codes_layout == QCNN_CODES_CANONICAL && c->algo != QCNN_ALGO_CHUNKED)
         off += align_up(packed_codes_bytes(s.Ct, s.kh * s.kw, s.M), kWsAlign);
     c->lut_off = off;
-    if (!c->fused) off += align_up(c->up.lut_bytes, kWsAlign);
+    if (c->algo == QCNN_ALGO_UNFUSED) {
+        c->up = plan_conv_unfused(s);
+        off += align_up(c->up.lut_bytes, kWsAlign);
+    } else if (c->algo == QCNN_ALGO_CHUNKED) {
+        off += c->cp.entries_bytes + c->cp.starts_bytes;
+    }
     c->total = off;
     return QCNN_OK;
 }
@@ -116,6 +128,9 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
 qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const uint8_t *codes,
                      int codes_layout, const float *bias, float *y, int relu, void *ws,
                      cudaStream_t st) {
+    if (c.algo == QCNN_ALGO_CHUNKED)
+        return launch_conv_chunked(c.s, c.cp, x, D, codes, codes_layout == QCNN_CODES_PACKED, bias,
+                                   y, relu, static_cast<uint8_t *>(ws) + c.lut_off, st);
     const uint8_t *packed = codes;
     if (codes_layout == QCNN_CODES_CANONICAL) {
         uint8_t *p = static_cast<uint8_t *>(ws) + c.packed_off;
@@ -124,7 +139,8 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
         if (rc != QCNN_OK) return rc;
         packed = p;
     }
-    if (c.fused) return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, st);
+    if (c.algo == QCNN_ALGO_FUSED)
+        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, st);
     float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
     return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
 }

@@ -55,6 +55,20 @@ struct ConvUnfusedPlan {
 };
 ConvUnfusedPlan plan_conv_unfused(const ConvShape &s);
 
+// Chunked plan (conv_chunked.cu): table rows of KC sub-codewords at a time.
+struct ConvChunkPlan {
+    bool ok = false;
+    int variant = -1;
+    int g_TH, KC, NCH, ct_cta, row_tiles, ct_tiles;
+    size_t smem, entries_bytes, starts_bytes;
+    double score;
+};
+ConvChunkPlan plan_conv_chunked(const ConvShape &s);
+qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, const float *x,
+                                const float *D, const uint8_t *codes, int codes_packed,
+                                const float *bias, float *y, int relu, void *ws,
+                                cudaStream_t st);
+
 size_t packed_codes_bytes(int Ct, int kk, int M);
 int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
 

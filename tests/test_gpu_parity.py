@@ -63,7 +63,7 @@ CONV_SWEEP = [
 
 
 @pytest.mark.parametrize("case", CONV_SWEEP, ids=lambda c: "x".join(map(str, c)))
-@pytest.mark.parametrize("algo", ["auto", "unfused"])
+@pytest.mark.parametrize("algo", ["auto", "unfused", "chunked"])
 def test_conv_sweep(case, algo):
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
     x, D, codes, b = conv_case(hash(case) % 1000, N, Cs, H, W, Ct, kh, kw, Csp, K)
@@ -84,7 +84,7 @@ def test_conv_fused_forced(case):
     assert rel(host(got), ref) <= TOL
 
 
-@pytest.mark.parametrize("algo", ["fused", "unfused"])
+@pytest.mark.parametrize("algo", ["fused", "unfused", "chunked"])
 def test_conv_integer_bit_exact(algo):
     case = (2, 16, 14, 13, 36, 3, 3, 1, 1, 4, 32)
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
@@ -134,7 +134,7 @@ def test_out_of_range_codes_are_clamped_not_faulting():
     bad = codes.copy()
     bad[::3, ::2, :] = 255
     good = np.minimum(bad, K - 1).astype(np.uint8)
-    for algo in ("fused", "unfused"):
+    for algo in ("fused", "unfused", "chunked"):
         a = host(q.conv_forward(cuda(x), cuda(D), cuda(bad), kh, kw, 1, 1, cuda(b), algo=algo))
         c = host(q.conv_forward(cuda(x), cuda(D), cuda(good), kh, kw, 1, 1, cuda(b), algo=algo))
         assert np.array_equal(a, c)
