@@ -23,6 +23,8 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdio>
+#include <cstdlib>
 
 namespace qcnn {
 
@@ -67,23 +69,23 @@ struct ConvFusedArgs {
     const float *__restrict__ bias;
     float *__restrict__ y;
     int N, Cs, H, W, Ct, kh, kw, pad, Csp, K, M, Ho, Wo;
-    int pitch, TH, KS, HP, ct_cta, CtP, relu;
+    int pitch, TH, KS, HP, CtP, relu;
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
 };
 
-
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned).
 struct FusedSmem {
-    size_t lut, xs, ds, cs, total;
+    size_t lut, xs, ds, cs, hoff, total;
 };
-__host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats,
-                                                       int csp4, int kk, int ct_cta) {
+__host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats, int csp4,
+                                                       int kk, int ct_cta, int HP) {
     FusedSmem s;
     s.lut = 0;
     s.xs = ((size_t)K * KS * 4 + 15) / 16 * 16;
     s.ds = s.xs + (size_t)2 * xs_floats * 4;
     s.cs = s.ds + (size_t)2 * K * csp4 * 4;
-    s.total = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
+    s.hoff = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
+    s.total = s.hoff + ((size_t)HP * 4 + 15) / 16 * 16;
     return s;
 }
 
@@ -111,53 +113,68 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 
 // P     : 32-position slots per warp
 // CTW   : output channels per warp
-// WP    : warps along positions (8 / WP warps along channels)
+// WP    : warps along positions (NW / WP warps along channels)
 // CSP4  : C'_s rounded up to 4 or 8 (register width of one sub-vector)
-// NW    : warps per CTA (8 or 16)
-template <int P, int CTW, int WP, int CSP4, int NW>
-__global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(const ConvFusedArgs a) {
-    constexpr int kFusedThreads = NW * 32;
-    constexpr int QB = 16 / CSP4;  // sub-codewords per lane per build pass
+// NW    : warps per CTA (8, 16 or 32)
+// MINB  : CTAs per SM the register budget is sized for (2 lets one CTA's
+//         table build and barriers overlap the other CTA's gather)
+template <int P, int CTW, int WP, int CSP4, int NW, int MINB>
+__global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
+    constexpr int NT = NW * 32;
+    constexpr int CT_CTA = (NW / WP) * CTW;
+    constexpr int Q16 = CT_CTA / 16;
+    // sub-codewords per lane per build pass (fewer under a 64-register budget)
+    constexpr int QB = (NW * MINB >= 32 ? 8 : 16) / CSP4;
+    static_assert(CT_CTA % 16 == 0, "channel tile must be a multiple of 16");
     extern __shared__ __align__(16) unsigned char smem[];
-    const FusedSmem L = fused_smem_layout(a.K, a.KS, a.xs_floats, CSP4, a.kh * a.kw, a.ct_cta);
+    const int kk = a.kh * a.kw;
+    const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
+    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, HP);
     float *lut = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
+    int *hoff = reinterpret_cast<int *>(smem + L.hoff);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
     const int oy0 = blockIdx.x * a.TH;
-    const int ct0 = blockIdx.y * a.ct_cta;
+    const int ct0 = blockIdx.y * CT_CTA;
     const int n = blockIdx.z;
-    const int kk = a.kh * a.kw;
-    const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
+    const int HW = a.H * a.W;
+
+    // Halo position h -> offset iy*W + ix inside one input plane, or -1 where
+    // the zero padding is; sub-vector slots j >= C'_s stay zero.
+    for (int h = tid; h < HP; h += NT) {
+        const int r = h / pitch, c = h - r * pitch;
+        const int iy = oy0 - a.pad + r, ix = c - a.pad;
+        hoff[h] = (iy >= 0 && iy < a.H && ix >= 0 && ix < a.W) ? iy * a.W + ix : -1;
+    }
+    if (a.Csp < CSP4) {
+        for (int e = tid; e < 2 * a.xs_floats; e += NT) xs[e] = 0.f;
+        for (int e = tid; e < 2 * K * CSP4; e += NT) ds[e] = 0.f;
+    }
+    __syncthreads();
 
     // ---- asynchronous staging of sub-space m into buffer b ---------------
     auto stage = [&](int m, int b) {
         float *xb = xs + b * a.xs_floats;
-        const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * a.H * a.W;
-        for (int e = tid; e < HP * CSP4; e += kFusedThreads) {
-            const int h = e % HP, j = e / HP;
-            const int r = h / pitch, c = h - r * pitch;
-            const int iy = oy0 - a.pad + r, ix = c - a.pad;
-            const bool ok = j < a.Csp && iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
-            const float *src = ok ? xn + ((size_t)j * a.H + iy) * a.W + ix : a.x;
-            cp_async4(xb + h * CSP4 + j, src, ok);
+        const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * HW;
+        for (int j = 0; j < a.Csp; ++j) {
+            for (int h = tid; h < HP; h += NT) {
+                const int off = hoff[h];
+                cp_async4(xb + h * CSP4 + j, off >= 0 ? xn + (size_t)j * HW + off : a.x, off >= 0);
+            }
         }
         float *db = ds + b * K * CSP4;
         const float *dm = a.D + (size_t)m * K * a.Csp;
-        for (int e = tid; e < K * CSP4; e += kFusedThreads) {
-            const int k = e / CSP4, j = e - k * CSP4;
-            const bool ok = j < a.Csp;
-            cp_async4(db + e, ok ? dm + k * a.Csp + j : a.D, ok);
-        }
-        uint8_t *cb = cs + (size_t)b * kk * a.ct_cta;
-        const int q16 = a.ct_cta / 16;
+        for (int k = tid; k < K; k += NT)
+            for (int j = 0; j < a.Csp; ++j) cp_async4(db + k * CSP4 + j, dm + k * a.Csp + j, true);
+        uint8_t *cb = cs + (size_t)b * kk * CT_CTA;
         const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
-        for (int e = tid; e < kk * q16; e += kFusedThreads) {
-            const int pk = e / q16, q = e - pk * q16;
-            cp_async16(cb + pk * a.ct_cta + q * 16, cm + (size_t)pk * a.CtP + q * 16);
+        for (int e = tid; e < kk * Q16; e += NT) {
+            const int pk = e / Q16, q = e % Q16;
+            cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
         }
         cp_async_commit();
     };
@@ -173,6 +190,8 @@ __global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(co
     const int KS4 = KS * 4;
     const unsigned char *lutb = reinterpret_cast<const unsigned char *>(lut);
     const unsigned kmax4 = (unsigned)(K - 1) * 0x01010101u;  // clamp codes into [0, K)
+    const int hpw = cdiv(HP, NW);
+    const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
 
     stage(0, 0);
     for (int m = 0; m < a.M; ++m) {
@@ -181,21 +200,18 @@ __global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(co
         __syncthreads();  // stage m visible; gather of m-1 finished everywhere
         if (m + 1 < a.M) stage(m + 1, b ^ 1);
 
-        // ---- build: lut[k][h] = <x(h), D[m][k]> ----------------------------
+        // ---- build: lut[k][h] = <x(h), D[m][k]>; lanes on k, warps on h ----
         {
             const float *xb = xs + b * a.xs_floats;
             const float *db = ds + b * K * CSP4;
-            const int hpw = cdiv(HP, NW);
-            const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
             for (int q0 = 0; q0 < K; q0 += 32 * QB) {
                 float dk[QB][CSP4];
 #pragma unroll
                 for (int i = 0; i < QB; ++i) {
-                    const int k = q0 + 32 * i + lane;
+                    const int k = min(q0 + 32 * i + lane, K - 1);
 #pragma unroll
                     for (int j = 0; j < CSP4; j += 4) {
-                        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-                        if (k < K) v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
+                        const float4 v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
                         dk[i][j] = v.x;
                         dk[i][j + 1] = v.y;
                         dk[i][j + 2] = v.z;
@@ -227,12 +243,12 @@ __global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(co
 
         // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
         {
-            const uint8_t *cb = cs + (size_t)b * kk * a.ct_cta + wc * CTW;
+            const uint8_t *cb = cs + (size_t)b * kk * CT_CTA + wc * CTW;
             for (int ky = 0; ky < a.kh; ++ky) {
                 for (int kx = 0; kx < a.kw; ++kx) {
                     const int pk = ky * a.kw + kx;
                     unsigned w[CTW / 4];
-                    load_code_words<CTW>(cb + pk * a.ct_cta, w);
+                    load_code_words<CTW>(cb + pk * CT_CTA, w);
 #pragma unroll
                     for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
                     const int base4 = lane_off4 + (ky * pitch + kx) * 4;
@@ -270,18 +286,25 @@ __global__ void __launch_bounds__(NW * 32, NW == 8 ? 2 : 1) conv_fused_kernel(co
 }
 
 // ---------------------------------------------------------- variant table --
+// eff: measured gather throughput of the variant relative to the best one
+// (GB300, AlexNet conv2-5 and VGG-16 conv3-5 shapes, all lanes counted).
 struct FusedVariant {
-    int P, CTW, WP, CSP4, NW;
+    int P, CTW, WP, CSP4, NW, MINB;
+    double eff;
     void (*fn)(ConvFusedArgs);
 };
 
-#define QCNN_FUSED(P, CTW, WP, C4, NW) {P, CTW, WP, C4, NW, conv_fused_kernel<P, CTW, WP, C4, NW>}
-static const FusedVariant kFused[] = {
-    QCNN_FUSED(2, 32, 1, 4, 8),  QCNN_FUSED(4, 16, 1, 4, 8),  QCNN_FUSED(4, 8, 2, 4, 8),
-    QCNN_FUSED(2, 32, 1, 8, 8),  QCNN_FUSED(4, 16, 1, 8, 8),  QCNN_FUSED(4, 8, 2, 8, 8),
-    QCNN_FUSED(4, 16, 1, 4, 16), QCNN_FUSED(4, 16, 2, 4, 16), QCNN_FUSED(2, 32, 2, 4, 16),
-    QCNN_FUSED(4, 16, 1, 8, 16), QCNN_FUSED(4, 16, 2, 8, 16), QCNN_FUSED(2, 32, 2, 8, 16),
-};
+#define QCNN_FUSED(P, CTW, WP, C4, NW, MB, EFF) \
+    {P, CTW, WP, C4, NW, MB, EFF, conv_fused_kernel<P, CTW, WP, C4, NW, MB>}
+#define QCNN_FUSED_SET(C4)                                                                  \
+    QCNN_FUSED(4, 8, 2, C4, 8, 2, 0.45),  /* small tiles: many CTAs for small batches */  \
+    QCNN_FUSED(4, 16, 1, C4, 16, 1, 1.0), /* 16 warps, 128 registers */                    \
+    QCNN_FUSED(7, 8, 1, C4, 16, 1, 1.0),                                                    \
+    QCNN_FUSED(4, 8, 1, C4, 16, 2, 0.83), /* 2 x 16 warps, 64 registers */                 \
+    QCNN_FUSED(8, 4, 1, C4, 32, 1, 0.82), /* 32 warps, 64 registers */                     \
+    QCNN_FUSED(7, 4, 1, C4, 32, 1, 0.89), QCNN_FUSED(4, 8, 1, C4, 32, 1, 0.98)
+static const FusedVariant kFused[] = {QCNN_FUSED_SET(4), QCNN_FUSED_SET(8)};
+#undef QCNN_FUSED_SET
 #undef QCNN_FUSED
 constexpr int kNumFused = sizeof(kFused) / sizeof(kFused[0]);
 
@@ -303,14 +326,25 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
     int smem_optin = 0;
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
             cudaSuccess ||
-        smem_optin <= 0)
+        smem_optin <= 0) {
+        cudaGetLastError();
         smem_optin = 227 * 1024;
+    }
     int smem_sm = 0;
     if (cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
             cudaSuccess ||
-        smem_sm <= 0)
+        smem_sm <= 0) {
+        cudaGetLastError();
         smem_sm = 228 * 1024;
+    }
+#ifdef QCNN_TUNING  // tuning builds only: force a variant from the environment
+    const char *force_env = getenv("QCNN_FUSED_VARIANT");
+    const int force = force_env ? atoi(force_env) : -1;
+#endif
     for (int v = 0; v < kNumFused; ++v) {
+#ifdef QCNN_TUNING
+        if (force >= 0 && v != force) continue;
+#endif
         const FusedVariant &fv = kFused[v];
         if (fv.CSP4 != csp4) continue;
         const int slots = fv.WP * fv.P;
@@ -322,19 +356,18 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const int KS = ks_for(slots * 32 + (s.kh - 1) * pitch + (s.kw - 1));
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
-        const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta).total;
+        const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, HP).total;
         if (smem > (size_t)smem_optin) continue;
-        const int cps = std::max(1, std::min(2, (int)(smem_sm / (smem + 1024))));
+        const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
         const int ct_tiles = cdiv(s.Ct, ct_cta);
         const double ctas = (double)s.N * row_tiles * ct_tiles;
         const double waves = std::ceil(ctas / (sms * cps));
-        // work per CTA in shared-memory wavefronts: gather + table build
+        // work per CTA in shared-memory wavefronts: gather (incl. lanes on
+        // discarded positions and channels past Ct) over the variant's measured
+        // efficiency, plus the table build
         const double gather = (double)slots * ct_cta * kk * s.M;
         const double build = (double)HP * s.K * s.M * 1.5 / 32.0;
-        const double per_cta = gather + build;
-        // fewer than 16 resident warps per SM leave the gather latency bound
-        const int warps_sm = cps * fv.NW;
-        const double score = waves * per_cta / cps * (warps_sm < 16 ? 1.4 : 1.0);
+        const double score = waves * (gather / fv.eff + build) * cps;
         if (!best.ok || score < best.score) {
             best.ok = true;
             best.variant = v;
@@ -352,6 +385,12 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
             best.score = score;
         }
     }
+#ifdef QCNN_TUNING
+    if (best.ok && getenv("QCNN_PLAN_VERBOSE"))
+        fprintf(stderr, "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d TH=%d KS=%d ct_cta=%d smem=%zu\n",
+                best.variant, best.P, best.CTW, best.WP, kFused[best.variant].NW, best.TH, best.KS,
+                best.ct_cta, best.smem);
+#endif
     return best;
 }
 
@@ -382,7 +421,6 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.TH = p.TH;
     a.KS = p.KS;
     a.HP = p.HP;
-    a.ct_cta = p.ct_cta;
     a.CtP = packed_ct(s.Ct);
     a.relu = relu;
     a.xs_floats = cdiv(p.HP, 4) * 4 * fv.CSP4;

@@ -8,8 +8,10 @@
 // NW images -- adds lut[mm][code][n] for its codes.  Lanes of a warp hold
 // different codes for the same (mm, n): with the odd pitch, distinct codes
 // below 32 land in distinct banks and equal codes broadcast, so the gather is
-// conflict free for K <= 32.  Codes are read straight from device memory,
-// four per 32-bit load, coalesced along c_t; each code serves NW images.
+// conflict free for K <= 32.  The chunk's codes, inputs and sub-codebooks are
+// copied to shared memory with cp.async one chunk ahead (double buffered), so
+// their device-memory latency overlaps the previous chunk's gather; each
+// code then serves NW images.
 // When the sub-space range is split over several CTAs (to fill the GPU),
 // the partial sums go to the workspace and a second kernel adds them in a
 // fixed order (deterministic), then applies bias and ReLU.
@@ -17,6 +19,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 
 namespace qcnn {
 
@@ -29,62 +32,51 @@ struct FcArgs {
     float *__restrict__ partial;  // [splits][N][Ct] when splits > 1
     int N, Cs, Ct, Csp, K, M;
     int NT, CT_CTA, MCH, n_chunks, chunks_per_split, splits, relu;
-    int NTP;  // odd pitch of a table row (>= NT)
-    int NTX;  // odd pitch of a staged x row (>= NT)
+    int NTP;     // odd pitch of a table row (>= NT)
+    int NTX;     // odd pitch of a staged x row (>= NT)
+    int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
 };
 
 constexpr int kFcThreads = 256;
-constexpr int kCPL = 4;  // outputs per lane
+constexpr int kCPL = 4;       // outputs per lane
+constexpr int kMchMax = 16;   // sub-spaces per chunk, at most
 
 struct FcSmem {
-    size_t lut, xs, ds, total;
+    size_t lut, xs, ds, cs, total;
 };
-__host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int NTP, int NTX, int Csp) {
+__host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int NTP, int NTX, int Csp,
+                                                 int CT_CTA) {
     FcSmem s;
     s.lut = 0;
     s.xs = ((size_t)MCH * K * NTP * 4 + 15) / 16 * 16;
     s.ds = s.xs + ((size_t)2 * MCH * Csp * NTX * 4 + 15) / 16 * 16;
-    s.total = s.ds + (size_t)2 * MCH * K * Csp * 4;
+    s.cs = s.ds + ((size_t)2 * MCH * K * Csp * 4 + 15) / 16 * 16;
+    s.total = s.cs + (size_t)2 * MCH * CT_CTA;
     return s;
 }
 
-// Four consecutive codes of row m starting at output ct (zero past Ct),
-// clamped into [0, K).
-__device__ __forceinline__ unsigned load_codes4(const uint8_t *__restrict__ codes, int Ct,
-                                                int m, int ct, bool vec, unsigned kmax4) {
-    unsigned w = 0;
-    const uint8_t *p = codes + (size_t)m * Ct + ct;
-    if (vec && ct + 3 < Ct) {
-        w = __ldg(reinterpret_cast<const unsigned *>(p));
-    } else {
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            if (ct + i < Ct) w |= (unsigned)__ldg(p + i) << (8 * i);
-    }
-    return __vminu4(w, kmax4);
-}
-
 // NW : images per lane;  WN : warps along images (8 / WN along outputs)
-template <int NW, int WN>
-__global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a) {
-    constexpr int MCH_MAX = 16;
+// MINB : CTAs per SM the register budget is sized for
+template <int NW, int WN, int MINB>
+__global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs a) {
+    constexpr int CT_CTA = (8 / WN) * 32 * kCPL;
     extern __shared__ __align__(16) unsigned char smem[];
-    const FcSmem L = fc_smem_layout(a.MCH, a.K, a.NTP, a.NTX, a.Csp);
+    const FcSmem L = fc_smem_layout(a.MCH, a.K, a.NTP, a.NTX, a.Csp, CT_CTA);
     float *lut = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
+    uint8_t *cs = smem + L.cs;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wn = warp % WN, wc = warp / WN;
-    const int ct0 = blockIdx.x * a.CT_CTA;
+    const int ct0 = blockIdx.x * CT_CTA;
     const int n0 = blockIdx.y * a.NT;
     const int split = blockIdx.z;
     const int c_begin = split * a.chunks_per_split;
     const int c_end = min(a.n_chunks, c_begin + a.chunks_per_split);
-    const int ct_lane = ct0 + (wc * 32 + lane) * kCPL;
+    const int lane_ct = (wc * 32 + lane) * kCPL;  // first output of this lane in the tile
     const int nbase = wn * NW;
     const int CCH = a.MCH * a.Csp;  // staged x floats per image
-    const bool vec = (a.Ct & 3) == 0;
     const unsigned kmax4 = (unsigned)(a.K - 1) * 0x01010101u;
 
     auto stage = [&](int c, int b) {
@@ -101,6 +93,32 @@ __global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a)
         const int dn = a.MCH * a.K * a.Csp, dv = mch * a.K * a.Csp;
         const float *dsrc = a.D + (size_t)m0 * a.K * a.Csp;
         for (int e = tid; e < dn; e += kFcThreads) cp_async4(db + e, e < dv ? dsrc + e : a.D, e < dv);
+        // codes[m0 + mm][ct0 .. ct0 + CT_CTA) -> cs[b][mm][.]; zero outside
+        uint8_t *cb = cs + (size_t)b * a.MCH * CT_CTA;
+        if (a.cvec > 0) {
+            const int per_row = CT_CTA / a.cvec;
+            for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
+                const int mm = e / per_row, q = e % per_row;
+                const int ct = ct0 + q * a.cvec;
+                const bool ok = mm < mch && ct < a.Ct;  // Ct % cvec == 0: all or nothing
+                const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
+                void *dst = cb + mm * CT_CTA + q * a.cvec;
+                const unsigned d = smem_addr(dst);
+                const int sz = ok ? a.cvec : 0;
+                if (a.cvec == 16)
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                else if (a.cvec == 8)
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                else
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+            }
+        } else {  // rows not 4-byte aligned: plain byte copies
+            for (int e = tid; e < a.MCH * CT_CTA; e += kFcThreads) {
+                const int mm = e / CT_CTA, q = e % CT_CTA;
+                const int ct = ct0 + q;
+                cb[e] = (mm < mch && ct < a.Ct) ? a.codes[(size_t)(m0 + mm) * a.Ct + ct] : 0;
+            }
+        }
         cp_async_commit();
     };
 
@@ -113,18 +131,10 @@ __global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a)
     if (c_begin < c_end) stage(c_begin, 0);
     for (int c = c_begin; c < c_end; ++c) {
         const int b = (c - c_begin) & 1;
-        const int m0 = c * a.MCH;
-        const int mch = min(a.MCH, a.M - m0);
+        const int mch = min(a.MCH, a.M - c * a.MCH);
         cp_async_wait<0>();
         __syncthreads();  // chunk c staged; gather of c-1 finished
         if (c + 1 < c_end) stage(c + 1, b ^ 1);
-
-        // codes of this chunk for this lane (latency hidden by the build)
-        unsigned cw[MCH_MAX];
-#pragma unroll
-        for (int mm = 0; mm < MCH_MAX; ++mm)
-            cw[mm] = (mm < mch && ct_lane < a.Ct) ? load_codes4(a.codes, a.Ct, m0 + mm, ct_lane, vec, kmax4)
-                                                  : 0u;
 
         // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>
         {
@@ -147,12 +157,15 @@ __global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a)
         __syncthreads();
 
         // gather
+        const uint8_t *cb = cs + (size_t)b * a.MCH * CT_CTA + lane_ct;
 #pragma unroll
-        for (int mm = 0; mm < MCH_MAX; ++mm) {
+        for (int mm = 0; mm < kMchMax; ++mm) {
             if (mm < mch) {
+                const unsigned w =
+                    __vminu4(*reinterpret_cast<const unsigned *>(cb + mm * CT_CTA), kmax4);
 #pragma unroll
                 for (int q = 0; q < kCPL; ++q) {
-                    const int code = (int)byte_of(cw[mm], q);
+                    const int code = (int)byte_of(w, q);
                     const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
 #pragma unroll
                     for (int i = 0; i < NW; ++i) acc[q][i] += row[i];
@@ -162,6 +175,7 @@ __global__ void __launch_bounds__(kFcThreads, 2) fc_fused_kernel(const FcArgs a)
     }
 
     // epilogue
+    const int ct_lane = ct0 + lane_ct;
 #pragma unroll
     for (int i = 0; i < NW; ++i) {
         const int n = n0 + nbase + i;
@@ -194,13 +208,17 @@ __global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, 
     }
 }
 
+// eff: measured gather throughput relative to the best variant (GB300,
+// AlexNet fc6-fc8 at batch 128).
 struct FcVariant {
-    int NW, WN;
+    int NW, WN, MINB;
+    double eff;
     void (*fn)(FcArgs);
 };
-#define QCNN_FC(NW, WN) {NW, WN, fc_fused_kernel<NW, WN>}
-static const FcVariant kFcVariants[] = {QCNN_FC(16, 2), QCNN_FC(8, 2), QCNN_FC(4, 1),
-                                        QCNN_FC(1, 1)};
+#define QCNN_FC(NW, WN, MB, EFF) {NW, WN, MB, EFF, fc_fused_kernel<NW, WN, MB>}
+static const FcVariant kFcVariants[] = {QCNN_FC(16, 2, 2, 0.8), QCNN_FC(8, 2, 3, 0.84),
+                                        QCNN_FC(8, 4, 3, 0.6), QCNN_FC(4, 1, 3, 1.0),
+                                        QCNN_FC(1, 1, 3, 0.5)};
 #undef QCNN_FC
 constexpr int kNumFc = sizeof(kFcVariants) / sizeof(kFcVariants[0]);
 
@@ -208,26 +226,40 @@ FcPlan plan_fc(const FcShape &s) {
     FcPlan best{};
     double best_t = 1e300;
     const int sms = num_sms();
-    const int MCH = s.K <= 32 ? 16 : std::max(1, 512 / s.K);
-    const int n_chunks = cdiv(s.M, MCH);
+    const size_t sm_bytes = 228 * 1024;
+#ifdef QCNN_TUNING  // tuning builds only: force a variant from the environment
+    const char *force_env = getenv("QCNN_FC_VARIANT");
+    const int force = force_env ? atoi(force_env) : -1;
+#endif
     for (int v = 0; v < kNumFc; ++v) {
+#ifdef QCNN_TUNING
+        if (force >= 0 && v != force) continue;
+#endif
         const FcVariant &fv = kFcVariants[v];
         const int NT = fv.NW * fv.WN;
         const int CT_CTA = (8 / fv.WN) * 32 * kCPL;
         const int NTP = NT | 1, NTX = NT | 1;
-        const size_t smem = fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp).total;
-        if (smem > 110 * 1024) continue;
+        // largest chunk that lets MINB CTAs share an SM
+        int MCH = std::min(kMchMax, std::max(1, 512 / s.K));
+        while (MCH > 1 &&
+               (fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp, CT_CTA).total + 1024) * fv.MINB > sm_bytes)
+            --MCH;
+        const size_t smem = fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp, CT_CTA).total;
+        if (smem > 200 * 1024) continue;
+        const int cps_sm = std::max(1, std::min(fv.MINB, (int)(sm_bytes / (smem + 1024))));
+        const int n_chunks = cdiv(s.M, MCH);
         const int n_tiles = cdiv(s.N, NT), ct_tiles = cdiv(s.Ct, CT_CTA);
         const int tiles = n_tiles * ct_tiles;
-        const int target = 2 * sms * 2;
+        const int target = 2 * sms * cps_sm;
         int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
-        const int cps = cdiv(n_chunks, splits);
-        splits = cdiv(n_chunks, cps);
+        const int cpsplit = cdiv(n_chunks, splits);
+        splits = cdiv(n_chunks, cpsplit);
         const double ctas = (double)tiles * splits;
-        const double waves = std::ceil(ctas / (2.0 * sms));
-        // one CTA: shared-memory wavefronts (gather + build) per chunk
+        const double waves = std::ceil(ctas / ((double)cps_sm * sms));
+        // one CTA: shared-memory wavefronts (gather + build) per chunk; a wave
+        // of cps_sm co-resident CTAs shares one SM
         const double per_chunk = (double)MCH * NT * CT_CTA / 32.0 + (double)MCH * s.K * NT / 32.0 * 2;
-        const double t_smem = waves * cps * per_chunk / 2.0 / 1.9e9;
+        const double t_smem = waves * cpsplit * per_chunk * cps_sm / 1.2e9 / fv.eff;
         const double bytes = (double)s.M * s.Ct * n_tiles + 4.0 * s.N * s.Cs * ct_tiles +
                              (splits > 1 ? 8.0 * splits * s.N * s.Ct : 0.0);
         const double t = std::max(t_smem, bytes / 6.0e12) + (splits > 1 ? 3e-6 : 0.0);
@@ -239,7 +271,7 @@ FcPlan plan_fc(const FcShape &s) {
             best.MCH = MCH;
             best.n_chunks = n_chunks;
             best.splits = splits;
-            best.chunks_per_split = cps;
+            best.chunks_per_split = cpsplit;
             best.n_tiles = n_tiles;
             best.ct_tiles = ct_tiles;
             best.smem = smem;
@@ -275,6 +307,11 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.relu = relu;
     a.NTP = p.NT | 1;
     a.NTX = p.NT | 1;
+    const uintptr_t base = reinterpret_cast<uintptr_t>(codes);
+    a.cvec = (s.Ct % 16 == 0 && base % 16 == 0) ? 16
+             : (s.Ct % 8 == 0 && base % 8 == 0) ? 8
+             : (s.Ct % 4 == 0 && base % 4 == 0) ? 4
+                                                 : 0;
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
