@@ -73,15 +73,16 @@ struct ConvFusedArgs {
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
 };
 
-// Shared memory carve-up of the fused kernel (byte offsets, 16-aligned).
+// Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
+// nlut = 2 table buffers when the sub-spaces are software pipelined.
 struct FusedSmem {
     size_t lut, xs, ds, cs, hoff, total;
 };
 __host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats, int csp4,
-                                                       int kk, int ct_cta, int HP) {
+                                                       int kk, int ct_cta, int HP, int nlut) {
     FusedSmem s;
     s.lut = 0;
-    s.xs = ((size_t)K * KS * 4 + 15) / 16 * 16;
+    s.xs = ((size_t)nlut * K * KS * 4 + 15) / 16 * 16;
     s.ds = s.xs + (size_t)2 * xs_floats * 4;
     s.cs = s.ds + (size_t)2 * K * csp4 * 4;
     s.hoff = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
@@ -116,9 +117,10 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // WP    : warps along positions (NW / WP warps along channels)
 // CSP4  : C'_s rounded up to 4 or 8 (register width of one sub-vector)
 // NW    : warps per CTA (8, 16 or 32)
-// MINB  : CTAs per SM the register budget is sized for (2 lets one CTA's
-//         table build and barriers overlap the other CTA's gather)
-template <int P, int CTW, int WP, int CSP4, int NW, int MINB>
+// MINB  : CTAs per SM the register budget is sized for
+// PIPE  : two table buffers; sub-space m+1's table is built while m is
+//         gathered, with one barrier per sub-space instead of two
+template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
     constexpr int NT = NW * 32;
     constexpr int CT_CTA = (NW / WP) * CTW;
@@ -129,8 +131,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     extern __shared__ __align__(16) unsigned char smem[];
     const int kk = a.kh * a.kw;
     const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
-    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, HP);
-    float *lut = reinterpret_cast<float *>(smem + L.lut);
+    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, HP, PIPE ? 2 : 1);
+    float *lut0 = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
@@ -156,8 +158,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     }
     __syncthreads();
 
-    // ---- asynchronous staging of sub-space m into buffer b ---------------
-    auto stage = [&](int m, int b) {
+    // ---- asynchronous staging (callers commit) --------------------------
+    auto stage_xd = [&](int m, int b) {  // inputs and sub-codebook of sub-space m
         float *xb = xs + b * a.xs_floats;
         const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * HW;
         for (int j = 0; j < a.Csp; ++j) {
@@ -170,98 +172,135 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         const float *dm = a.D + (size_t)m * K * a.Csp;
         for (int k = tid; k < K; k += NT)
             for (int j = 0; j < a.Csp; ++j) cp_async4(db + k * CSP4 + j, dm + k * a.Csp + j, true);
+    };
+    auto stage_codes = [&](int m, int b) {
         uint8_t *cb = cs + (size_t)b * kk * CT_CTA;
         const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
         for (int e = tid; e < kk * Q16; e += NT) {
             const int pk = e / Q16, q = e % Q16;
             cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
         }
-        cp_async_commit();
     };
 
+    // ---- build: lut[k][h] = <x(h), D[m][k]>; lanes on k, warps on h -------
+    const int hpw = cdiv(HP, NW);
+    const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
+    auto build = [&](int b, float *lut) {
+        const float *xb = xs + b * a.xs_floats;
+        const float *db = ds + b * K * CSP4;
+        for (int q0 = 0; q0 < K; q0 += 32 * QB) {
+            float dk[QB][CSP4];
+#pragma unroll
+            for (int i = 0; i < QB; ++i) {
+                const int k = min(q0 + 32 * i + lane, K - 1);
+#pragma unroll
+                for (int j = 0; j < CSP4; j += 4) {
+                    const float4 v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
+                    dk[i][j] = v.x;
+                    dk[i][j + 1] = v.y;
+                    dk[i][j + 2] = v.z;
+                    dk[i][j + 3] = v.w;
+                }
+            }
+            for (int h = h0; h < h1; ++h) {
+                float xv[CSP4];
+#pragma unroll
+                for (int j = 0; j < CSP4; j += 4) {
+                    const float4 v = *reinterpret_cast<const float4 *>(xb + h * CSP4 + j);
+                    xv[j] = v.x;
+                    xv[j + 1] = v.y;
+                    xv[j + 2] = v.z;
+                    xv[j + 3] = v.w;
+                }
+#pragma unroll
+                for (int i = 0; i < QB; ++i) {
+                    const int k = q0 + 32 * i + lane;
+                    float v = 0.f;
+#pragma unroll
+                    for (int j = 0; j < CSP4; ++j) v = fmaf(xv[j], dk[i][j], v);
+                    if (k < K) lut[k * KS + h] = v;
+                }
+            }
+        }
+    };
+
+    // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
     float acc[CTW][P];
 #pragma unroll
     for (int c = 0; c < CTW; ++c)
 #pragma unroll
         for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
-
-    // Byte offset of this lane's first position inside a table row.
-    const int lane_off4 = (wp * P * 32 + lane) * 4;
+    const int lane_off4 = (wp * P * 32 + lane) * 4;  // byte offset of the first position
     const int KS4 = KS * 4;
-    const unsigned char *lutb = reinterpret_cast<const unsigned char *>(lut);
     const unsigned kmax4 = (unsigned)(K - 1) * 0x01010101u;  // clamp codes into [0, K)
-    const int hpw = cdiv(HP, NW);
-    const int h0 = warp * hpw, h1 = min(HP, h0 + hpw);
-
-    stage(0, 0);
-    for (int m = 0; m < a.M; ++m) {
-        const int b = m & 1;
-        cp_async_wait<0>();
-        __syncthreads();  // stage m visible; gather of m-1 finished everywhere
-        if (m + 1 < a.M) stage(m + 1, b ^ 1);
-
-        // ---- build: lut[k][h] = <x(h), D[m][k]>; lanes on k, warps on h ----
-        {
-            const float *xb = xs + b * a.xs_floats;
-            const float *db = ds + b * K * CSP4;
-            for (int q0 = 0; q0 < K; q0 += 32 * QB) {
-                float dk[QB][CSP4];
+    auto gather = [&](int b, const float *lut) {
+        const unsigned char *lutb = reinterpret_cast<const unsigned char *>(lut);
+        const uint8_t *cb = cs + (size_t)b * kk * CT_CTA + wc * CTW;
+        for (int ky = 0; ky < a.kh; ++ky) {
+            for (int kx = 0; kx < a.kw; ++kx) {
+                const int pk = ky * a.kw + kx;
+                unsigned w[CTW / 4];
+                load_code_words<CTW>(cb + pk * CT_CTA, w);
 #pragma unroll
-                for (int i = 0; i < QB; ++i) {
-                    const int k = min(q0 + 32 * i + lane, K - 1);
+                for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
+                const int base4 = lane_off4 + (ky * pitch + kx) * 4;
 #pragma unroll
-                    for (int j = 0; j < CSP4; j += 4) {
-                        const float4 v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
-                        dk[i][j] = v.x;
-                        dk[i][j + 1] = v.y;
-                        dk[i][j + 2] = v.z;
-                        dk[i][j + 3] = v.w;
-                    }
-                }
-                for (int h = h0; h < h1; ++h) {
-                    float xv[CSP4];
-#pragma unroll
-                    for (int j = 0; j < CSP4; j += 4) {
-                        const float4 v = *reinterpret_cast<const float4 *>(xb + h * CSP4 + j);
-                        xv[j] = v.x;
-                        xv[j + 1] = v.y;
-                        xv[j + 2] = v.z;
-                        xv[j + 3] = v.w;
-                    }
-#pragma unroll
-                    for (int i = 0; i < QB; ++i) {
-                        const int k = q0 + 32 * i + lane;
-                        float v = 0.f;
-#pragma unroll
-                        for (int j = 0; j < CSP4; ++j) v = fmaf(xv[j], dk[i][j], v);
-                        if (k < K) lut[k * KS + h] = v;
-                    }
+                for (int c = 0; c < CTW; ++c) {
+                    const unsigned code = byte_of(w[c >> 2], c & 3);
+                    const unsigned char *row = lutb + (int)code * KS4 + base4;
+                    accumulate<P>(acc[c], [&](int p) {
+                        return *reinterpret_cast<const float *>(row + p * 128);
+                    });
                 }
             }
         }
-        __syncthreads();
+    };
 
-        // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
-        {
-            const uint8_t *cb = cs + (size_t)b * kk * CT_CTA + wc * CTW;
-            for (int ky = 0; ky < a.kh; ++ky) {
-                for (int kx = 0; kx < a.kw; ++kx) {
-                    const int pk = ky * a.kw + kx;
-                    unsigned w[CTW / 4];
-                    load_code_words<CTW>(cb + pk * CT_CTA, w);
-#pragma unroll
-                    for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
-                    const int base4 = lane_off4 + (ky * pitch + kx) * 4;
-#pragma unroll
-                    for (int c = 0; c < CTW; ++c) {
-                        const unsigned code = byte_of(w[c >> 2], c & 3);
-                        const unsigned char *row = lutb + (int)code * KS4 + base4;
-#pragma unroll
-                        for (int p = 0; p < P; ++p)
-                            acc[c][p] += *reinterpret_cast<const float *>(row + p * 128);
-                    }
-                }
+    if constexpr (!PIPE) {
+        stage_xd(0, 0);
+        stage_codes(0, 0);
+        cp_async_commit();
+        for (int m = 0; m < a.M; ++m) {
+            const int b = m & 1;
+            cp_async_wait<0>();
+            __syncthreads();  // stage m visible; gather of m-1 finished everywhere
+            if (m + 1 < a.M) {
+                stage_xd(m + 1, b ^ 1);
+                stage_codes(m + 1, b ^ 1);
+                cp_async_commit();
             }
+            build(b, lut0);
+            __syncthreads();
+            gather(b, lut0);
+        }
+    } else {
+        float *lut1 = lut0 + (size_t)K * KS;
+        stage_xd(0, 0);
+        if (a.M > 1) stage_xd(1, 1);
+        stage_codes(0, 0);
+        cp_async_commit();
+        cp_async_wait<0>();
+        __syncthreads();
+        build(0, lut0);
+        __syncthreads();
+        // Iteration m: table m ready in buffer m&1, codes m in code buffer m&1,
+        // inputs of m+1 in staging buffer (m+1)&1.
+        for (int m = 0; m < a.M; ++m) {
+            const int b = m & 1;
+            if (m + 2 < a.M) stage_xd(m + 2, b);
+            if (m + 1 < a.M) stage_codes(m + 1, b ^ 1);
+            cp_async_commit();
+            // even warps build first, odd warps gather first: the latency-bound
+            // table build of one half overlaps the other half's gather
+            if (warp & 1) {
+                gather(b, b ? lut1 : lut0);
+                if (m + 1 < a.M) build(b ^ 1, b ? lut0 : lut1);
+            } else {
+                if (m + 1 < a.M) build(b ^ 1, b ? lut0 : lut1);
+                gather(b, b ? lut1 : lut0);
+            }
+            cp_async_wait<0>();
+            __syncthreads();
         }
     }
 
@@ -287,22 +326,28 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 
 // ---------------------------------------------------------- variant table --
 // eff: measured gather throughput of the variant relative to the best one
-// (GB300, AlexNet conv2-5 and VGG-16 conv3-5 shapes, all lanes counted).
+// (GB300, AlexNet conv2-5 and VGG-16 conv3-5 shapes, all lanes counted);
+// build: share of the table-build time left exposed (1 = not overlapped).
 struct FusedVariant {
-    int P, CTW, WP, CSP4, NW, MINB;
-    double eff;
+    int P, CTW, WP, CSP4, NW, MINB, PIPE;
+    double eff, build;
     void (*fn)(ConvFusedArgs);
 };
 
-#define QCNN_FUSED(P, CTW, WP, C4, NW, MB, EFF) \
-    {P, CTW, WP, C4, NW, MB, EFF, conv_fused_kernel<P, CTW, WP, C4, NW, MB>}
-#define QCNN_FUSED_SET(C4)                                                                  \
-    QCNN_FUSED(4, 8, 2, C4, 8, 2, 0.45),  /* small tiles: many CTAs for small batches */  \
-    QCNN_FUSED(4, 16, 1, C4, 16, 1, 1.0), /* 16 warps, 128 registers */                    \
-    QCNN_FUSED(7, 8, 1, C4, 16, 1, 1.0),                                                    \
-    QCNN_FUSED(4, 8, 1, C4, 16, 2, 0.83), /* 2 x 16 warps, 64 registers */                 \
-    QCNN_FUSED(8, 4, 1, C4, 32, 1, 0.82), /* 32 warps, 64 registers */                     \
-    QCNN_FUSED(7, 4, 1, C4, 32, 1, 0.89), QCNN_FUSED(4, 8, 1, C4, 32, 1, 0.98)
+#define QCNN_FUSED(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
+    {P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD, conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE>}
+#define QCNN_FUSED_SET(C4)                                                                       \
+    QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
+    QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
+    QCNN_FUSED(7, 8, 1, C4, 16, 1, false, 1.0, 1.0),                                             \
+    QCNN_FUSED(4, 8, 1, C4, 16, 2, false, 0.83, 1.0), /* 2 x 16 warps, 64 registers */          \
+    QCNN_FUSED(8, 4, 1, C4, 32, 1, false, 0.82, 1.0), /* 32 warps, 64 registers */              \
+    QCNN_FUSED(7, 4, 1, C4, 32, 1, false, 0.89, 1.0),                                            \
+    QCNN_FUSED(4, 8, 1, C4, 32, 1, false, 0.98, 1.0),                                            \
+    QCNN_FUSED(2, 32, 1, C4, 16, 1, true, 0.75, 0.3), /* pipelined: two table buffers */         \
+    QCNN_FUSED(4, 16, 1, C4, 16, 1, true, 0.85, 0.3),                                             \
+    QCNN_FUSED(2, 16, 2, C4, 16, 1, true, 0.7, 0.3),                                             \
+    QCNN_FUSED(4, 8, 1, C4, 16, 1, true, 0.8, 0.3)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4), QCNN_FUSED_SET(8)};
 #undef QCNN_FUSED_SET
 #undef QCNN_FUSED
@@ -356,7 +401,8 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const int KS = ks_for(slots * 32 + (s.kh - 1) * pitch + (s.kw - 1));
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
-        const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, HP).total;
+        const size_t smem =
+            fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, HP, fv.PIPE ? 2 : 1).total;
         if (smem > (size_t)smem_optin) continue;
         const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
         const int ct_tiles = cdiv(s.Ct, ct_cta);
@@ -364,10 +410,11 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const double waves = std::ceil(ctas / (sms * cps));
         // work per CTA in shared-memory wavefronts: gather (incl. lanes on
         // discarded positions and channels past Ct) over the variant's measured
-        // efficiency, plus the table build
+        // efficiency, plus the exposed part of the table build (which costs
+        // about 4 wavefronts of time per 32 entries: latency-bound FMA chains)
         const double gather = (double)slots * ct_cta * kk * s.M;
-        const double build = (double)HP * s.K * s.M * 1.5 / 32.0;
-        const double score = waves * (gather / fv.eff + build) * cps;
+        const double build = (double)HP * s.K * s.M * 4.0 / 32.0;
+        const double score = waves * (gather / fv.eff + build * fv.build) * cps;
         if (!best.ok || score < best.score) {
             best.ok = true;
             best.variant = v;
@@ -387,9 +434,10 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
     }
 #ifdef QCNN_TUNING
     if (best.ok && getenv("QCNN_PLAN_VERBOSE"))
-        fprintf(stderr, "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d TH=%d KS=%d ct_cta=%d smem=%zu\n",
-                best.variant, best.P, best.CTW, best.WP, kFused[best.variant].NW, best.TH, best.KS,
-                best.ct_cta, best.smem);
+        fprintf(stderr,
+                "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d pipe=%d TH=%d KS=%d ct_cta=%d smem=%zu\n",
+                best.variant, best.P, best.CTW, best.WP, kFused[best.variant].NW,
+                kFused[best.variant].PIPE, best.TH, best.KS, best.ct_cta, best.smem);
 #endif
     return best;
 }

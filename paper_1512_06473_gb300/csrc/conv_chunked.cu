@@ -164,8 +164,7 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
 #pragma unroll 2
                     for (int e = e0; e < e1; ++e) {
                         const float *base = lut + lane + __ldg(ep + e);
-#pragma unroll
-                        for (int p = 0; p < P; ++p) acc[c][p] += base[p * 32];
+                        accumulate<P>(acc[c], [&](int p) { return base[p * 32]; });
                     }
                 }
             }
@@ -200,7 +199,7 @@ struct ChunkVariant {
 #define QCNN_CHUNK(P, CTW, QPT, C) {P, CTW, QPT, C, conv_chunked_kernel<P, CTW, QPT, C>}
 static const ChunkVariant kChunk[] = {
     QCNN_CHUNK(8, 6, 11, 3),   // AlexNet conv1: 4 rows of 57, 96 channels
-    QCNN_CHUNK(8, 8, 8, 4),
+    QCNN_CHUNK(8, 8, 6, 4),
     QCNN_CHUNK(4, 8, 4, 8),
 };
 #undef QCNN_CHUNK

@@ -167,8 +167,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 for (int q = 0; q < kCPL; ++q) {
                     const int code = (int)byte_of(w, q);
                     const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
-#pragma unroll
-                    for (int i = 0; i < NW; ++i) acc[q][i] += row[i];
+                    accumulate<NW>(acc[q], [&](int i) { return row[i]; });
                 }
             }
         }

@@ -6,7 +6,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
-#include "../../include/qcnn.h"
+#include "qcnn.h"  // include/ is on the include path of the build
 
 namespace qcnn {
 
@@ -146,6 +146,22 @@ __device__ __forceinline__ void cp_async_wait() {
 // Byte b (0..3) of w, zero-extended.
 __device__ __forceinline__ unsigned byte_of(unsigned w, int b) {
     return __byte_perm(w, 0u, 0x4440u | (unsigned)b);
+}
+
+// a += x; b += y with one packed fp32x2 add: two independent IEEE
+// round-to-nearest additions, bit-identical to two scalar adds.
+__device__ __forceinline__ void add2(float &a, float &b, float x, float y) {
+    const float2 r = __fadd2_rn(make_float2(a, b), make_float2(x, y));
+    a = r.x;
+    b = r.y;
+}
+
+// acc[p] += v(p) for p < P, pairing the adds where possible.
+template <int P, typename F>
+__device__ __forceinline__ void accumulate(float (&acc)[P], F v) {
+#pragma unroll
+    for (int p = 0; p + 1 < P; p += 2) add2(acc[p], acc[p + 1], v(p), v(p + 1));
+    if constexpr (P % 2 == 1) acc[P - 1] += v(P - 1);
 }
 
 }  // namespace qcnn
