@@ -15,7 +15,7 @@
 //   2. gathers only the (c_t, p_k) pairs whose code lies in the chunk.  Those
 //      pairs come from per-(m, c_t) entry lists, counting-sorted by chunk in
 //      the workspace by a small prep kernel, each entry being the ready
-//      shared-memory offset  kl*SK + phase*PS + (dy - dymin)*PW + (dx - dxmin).
+//      byte offset  4 * (kl*SK + phase*PS + (dy - dymin)*PW + (dx - dxmin)).
 // A lane owns P positions of the band's output grid of pitch PW
 // (l = r*PW + c, columns c >= Wo are discarded) and CTW channels; its input
 // sub-vectors (QPT positions x CSPT channels) stay in registers across the
@@ -23,6 +23,7 @@
 #include "qcnn_internal.cuh"
 
 #include <algorithm>
+#include <cmath>
 
 namespace qcnn {
 
@@ -36,7 +37,7 @@ __host__ __device__ inline int floor_div(int a, int b) {
     return (a >= 0) ? a / b : -((-a + b - 1) / b);
 }
 
-// Shared-memory offset of kernel offset (ky, kx) inside one table row.
+// Offset (in floats) of kernel offset (ky, kx) inside one table row.
 __host__ __device__ inline int chunk_phase_off(const ChunkGeom &g, int ky, int kx) {
     const int ty = ky - g.pad, tx = kx - g.pad;
     const int dy = floor_div(ty, g.s), dx = floor_div(tx, g.s);
@@ -45,7 +46,7 @@ __host__ __device__ inline int chunk_phase_off(const ChunkGeom &g, int ky, int k
 }
 
 // ------------------------------------------------------------------ prep --
-// One thread per (m, ct): entries[m][ct][*] = offsets sorted by chunk,
+// One thread per (m, ct): entries[m][ct][*] = byte offsets sorted by chunk,
 // starts[m][ct][c] = first entry of chunk c (NCH + 1 values).
 __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed, int CtP,
                                   int Ct, int kk, int M, int K, ChunkGeom g,
@@ -63,14 +64,14 @@ __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed,
     for (int pk = 0; pk < kk; ++pk) st[code_at(pk) / g.KC + 1] += 1;
     for (int c = 0; c < g.NCH; ++c) st[c + 1] += st[c];
     uint32_t *en = entries + (size_t)i * kk;
-    // stable placement: a second pass per chunk keeps p_k order inside a chunk
+    // stable placement: a pass per chunk keeps p_k order inside a chunk
     for (int c = 0; c < g.NCH; ++c) {
         int pos = st[c];
         for (int pk = 0; pk < kk; ++pk) {
             const int code = code_at(pk);
             if (code / g.KC != c) continue;
             const int ky = pk / g.kw, kx = pk % g.kw;
-            en[pos++] = (uint32_t)((code - c * g.KC) * g.SK + chunk_phase_off(g, ky, kx));
+            en[pos++] = (uint32_t)(4 * ((code - c * g.KC) * g.SK + chunk_phase_off(g, ky, kx)));
         }
     }
 }
@@ -91,8 +92,8 @@ template <int P, int CTW, int QPT, int CSPT>
 __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const ChunkArgs a) {
     extern __shared__ __align__(16) float csm[];
     const ChunkGeom &g = a.g;
-    float *lut = csm;                            // [KC][SK]
-    float *ds = csm + (size_t)g.KC * g.SK;       // [K][CSPT]
+    float *lut = csm;                             // [KC][SK]
+    float *ds = csm + (size_t)g.KC * g.SK;        // [K][CSPT]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int oy0 = blockIdx.x * g.TH;
     const int ct0 = blockIdx.y * a.ct_cta;
@@ -105,14 +106,73 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
 #pragma unroll
         for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
 
+    float xr[QPT][CSPT];  // input sub-vectors of positions tid + qi * 512
+
+    // rows [kl] of chunk ch: lut[kl][q] = <x(q), D[m][k0 + kl]>; every thread
+    // writes its QPT positions (SK >= QPT * 512, positions past NQ hold 0)
+    auto build = [&](int ch, float *L) {
+        const int k0 = ch * g.KC, kc = min(g.KC, a.K - k0);
+        for (int kl = 0; kl < kc; ++kl) {
+            float dk[CSPT];
+#pragma unroll
+            for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
+            float *row = L + kl * g.SK + tid;
+#pragma unroll
+            for (int qi = 0; qi + 1 < QPT; qi += 2) {
+                float2 v = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int j = 0; j < CSPT; ++j)
+                    v = __ffma2_rn(make_float2(xr[qi][j], xr[qi + 1][j]), make_float2(dk[j], dk[j]), v);
+                row[qi * kChunkThreads] = v.x;
+                row[(qi + 1) * kChunkThreads] = v.y;
+            }
+            if constexpr (QPT % 2 == 1) {
+                float v = 0.f;
+#pragma unroll
+                for (int j = 0; j < CSPT; ++j) v = fmaf(xr[QPT - 1][j], dk[j], v);
+                row[(QPT - 1) * kChunkThreads] = v;
+            }
+        }
+    };
+
+    // the (c_t, p_k) pairs of this warp's channels whose code is in chunk ch
+    auto gather = [&](int m, int ch, const float *L) {
+        const unsigned char *lb = reinterpret_cast<const unsigned char *>(L) + lane * 4;
+#pragma unroll
+        for (int c = 0; c < CTW; ++c) {
+            const int ct = ctw0 + c;
+            if (ct < a.Ct) {
+                const size_t row = (size_t)m * a.Ct + ct;
+                const int e0 = __ldg(a.starts + row * (g.NCH + 1) + ch);
+                const int e1 = __ldg(a.starts + row * (g.NCH + 1) + ch + 1);
+                const uint32_t *ep = a.entries + row * a.kk;
+                int e = e0;
+                for (; e + 1 < e1; e += 2) {
+                    const unsigned o0 = __ldg(ep + e), o1 = __ldg(ep + e + 1);
+                    const unsigned char *b0 = lb + o0, *b1 = lb + o1;
+                    accumulate<P>(acc[c], [&](int p) {
+                        return *reinterpret_cast<const float *>(b0 + p * 128);
+                    });
+                    accumulate<P>(acc[c], [&](int p) {
+                        return *reinterpret_cast<const float *>(b1 + p * 128);
+                    });
+                }
+                if (e < e1) {
+                    const unsigned char *b0 = lb + __ldg(ep + e);
+                    accumulate<P>(acc[c], [&](int p) {
+                        return *reinterpret_cast<const float *>(b0 + p * 128);
+                    });
+                }
+            }
+        }
+    };
+
     for (int m = 0; m < a.M; ++m) {
-        __syncthreads();  // previous sub-space finished with ds and lut
+        __syncthreads();  // previous sub-space finished with ds and the tables
         for (int e = tid; e < a.K * CSPT; e += kChunkThreads) {
             const int k = e / CSPT, j = e % CSPT;
             ds[e] = j < a.Csp ? __ldg(a.D + ((size_t)m * a.K + k) * a.Csp + j) : 0.f;
         }
-        // this thread's input sub-vectors, kept for every chunk of m
-        float xr[QPT][CSPT];
 #pragma unroll
         for (int qi = 0; qi < QPT; ++qi) {
             const int q = tid + qi * kChunkThreads;
@@ -131,43 +191,10 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
         }
         __syncthreads();  // ds ready
 
-        const int *st = a.starts;
-        const uint32_t *en = a.entries;
         for (int ch = 0; ch < g.NCH; ++ch) {
-            const int k0 = ch * g.KC, kc = min(g.KC, a.K - k0);
-            // ---- build the chunk's table rows (one codeword at a time, so its
-            // components are read once per thread and reused for QPT positions)
-            for (int kl = 0; kl < kc; ++kl) {
-                float dk[CSPT];
-#pragma unroll
-                for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
-                float *row = lut + kl * g.SK;
-#pragma unroll
-                for (int qi = 0; qi < QPT; ++qi) {
-                    const int q = tid + qi * kChunkThreads;
-                    float v = 0.f;
-#pragma unroll
-                    for (int j = 0; j < CSPT; ++j) v = fmaf(xr[qi][j], dk[j], v);
-                    if (q < g.NQ) row[q] = v;
-                }
-            }
+            build(ch, lut);
             __syncthreads();
-            // ---- gather the pairs whose code is in this chunk
-#pragma unroll
-            for (int c = 0; c < CTW; ++c) {
-                const int ct = ctw0 + c;
-                if (ct < a.Ct) {
-                    const size_t row = (size_t)m * a.Ct + ct;
-                    const int e0 = __ldg(st + row * (g.NCH + 1) + ch);
-                    const int e1 = __ldg(st + row * (g.NCH + 1) + ch + 1);
-                    const uint32_t *ep = en + row * a.kk;
-#pragma unroll 2
-                    for (int e = e0; e < e1; ++e) {
-                        const float *base = lut + lane + __ldg(ep + e);
-                        accumulate<P>(acc[c], [&](int p) { return base[p * 32]; });
-                    }
-                }
-            }
+            gather(m, ch, lut);
             __syncthreads();  // table rows free for the next chunk
         }
     }
@@ -198,14 +225,15 @@ struct ChunkVariant {
 };
 #define QCNN_CHUNK(P, CTW, QPT, C) {P, CTW, QPT, C, conv_chunked_kernel<P, CTW, QPT, C>}
 static const ChunkVariant kChunk[] = {
-    QCNN_CHUNK(8, 6, 11, 3),   // AlexNet conv1: 4 rows of 57, 96 channels
+    QCNN_CHUNK(8, 6, 11, 3),  // AlexNet conv1: 4 rows of 57, 96 channels per CTA
+    QCNN_CHUNK(8, 1, 11, 3),  // same band, 16 channels per CTA: small batches
     QCNN_CHUNK(8, 8, 6, 4),
     QCNN_CHUNK(4, 8, 4, 8),
 };
 #undef QCNN_CHUNK
 constexpr int kNumChunk = sizeof(kChunk) / sizeof(kChunk[0]);
 
-static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P) {
+static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P, int QPT) {
     ChunkGeom g;
     g.s = s.stride;
     g.pad = s.pad;
@@ -222,7 +250,7 @@ static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P) {
     g.NQ = s.stride * s.stride * g.PS;
     int sk = (s.stride * s.stride - 1) * g.PS + (g.dymax - g.dymin) * g.PW + (g.dxmax - g.dxmin) +
              P * 32;
-    sk = std::max(sk, g.NQ);
+    sk = std::max(sk, QPT * kChunkThreads);  // every thread's positions fit a row
     while (sk % 32 != 1) ++sk;
     g.SK = sk;
     g.KC = KC;
@@ -240,30 +268,38 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
         cudaGetLastError();
         smem_optin = 227 * 1024;
     }
+#ifdef QCNN_TUNING  // tuning builds only: force a variant from the environment
+    const char *force_env = getenv("QCNN_CHUNK_VARIANT");
+    const int force = force_env ? atoi(force_env) : -1;
+#endif
     for (int v = 0; v < kNumChunk; ++v) {
+#ifdef QCNN_TUNING
+        if (force >= 0 && v != force) continue;
+#endif
         const ChunkVariant &cv = kChunk[v];
         if (s.Csp > cv.CSPT) continue;
         const int ct_cta = 16 * cv.CTW;
-        // largest band that the variant's lanes cover
+        // largest band that the variant's lanes and registers cover
         for (int TH = std::min(s.Ho, 64); TH >= 1; --TH) {
-            const ChunkGeom g0 = chunk_geom(s, TH, 1, cv.P);
+            const ChunkGeom g0 = chunk_geom(s, TH, 1, cv.P, cv.QPT);
             if (TH * g0.PW > cv.P * 32) continue;
             if (g0.NQ > cv.QPT * kChunkThreads) continue;
-            // balance the bands
             const int row_tiles = cdiv(s.Ho, TH);
-            const int th = cdiv(s.Ho, row_tiles);
+            const int th = cdiv(s.Ho, row_tiles);  // balance the bands
             for (int KC : {16, 8, 4, 2, 1}) {
                 if (KC > s.K) continue;
-                const ChunkGeom g = chunk_geom(s, th, KC, cv.P);
+                const ChunkGeom g = chunk_geom(s, th, KC, cv.P, cv.QPT);
                 const size_t smem = ((size_t)KC * g.SK + (size_t)s.K * cv.CSPT) * sizeof(float);
                 if (smem > (size_t)smem_optin) continue;
                 const int ct_tiles = cdiv(s.Ct, ct_cta);
                 const double ctas = (double)s.N * row_tiles * ct_tiles;
                 const double waves = std::ceil(ctas / sms);
-                // per CTA: gather wavefronts + table stores, per sub-space
+                // per CTA and sub-space: gather wavefronts + table stores + a
+                // barrier cost per chunk
                 const double gather = (double)cv.P * ct_cta * s.kh * s.kw;
-                const double build = (double)g.NQ * s.K / 32.0 + (double)g.NCH * 400.0;
-                const double score = waves * (gather + build) * s.M;
+                const double build = (double)g.NQ * s.K / 32.0;
+                const double sync = (double)g.NCH * 1200.0;
+                const double score = waves * (gather + build + sync) * s.M;
                 if (!best.ok || score < best.score) {
                     best.ok = true;
                     best.variant = v;
@@ -281,7 +317,8 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
         }
     }
     if (best.ok) {
-        const ChunkGeom g = chunk_geom(s, best.g_TH, best.KC, kChunk[best.variant].P);
+        const ChunkVariant &cv = kChunk[best.variant];
+        const ChunkGeom g = chunk_geom(s, best.g_TH, best.KC, cv.P, cv.QPT);
         best.NCH = g.NCH;
         best.entries_bytes = align_up((size_t)s.M * s.Ct * s.kh * s.kw * 4, kWsAlign);
         best.starts_bytes = align_up((size_t)s.M * s.Ct * (g.NCH + 1) * 4, kWsAlign);
@@ -294,7 +331,7 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
                                 const float *bias, float *y, int relu, void *ws,
                                 cudaStream_t st) {
     const ChunkVariant &cv = kChunk[p.variant];
-    const ChunkGeom g = chunk_geom(s, p.g_TH, p.KC, cv.P);
+    const ChunkGeom g = chunk_geom(s, p.g_TH, p.KC, cv.P, cv.QPT);
     uint32_t *entries = static_cast<uint32_t *>(ws);
     int *starts = reinterpret_cast<int *>(static_cast<uint8_t *>(ws) + p.entries_bytes);
     const int kk = s.kh * s.kw;
