@@ -207,6 +207,44 @@ def load_peaks():
         return {}
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest value of x over all ranks (the slowest rank's time)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(images_per_rank: int, world: int, steps: int, seconds: float) -> float:
+    """Whole-job images/s: every rank processes its own batch each step
+    (independent replicas, weak scaling), timed by the slowest rank."""
+    return images_per_rank * world * steps / seconds
+
+
+def recorded_traffic(workload, batch, layer):
+    """DRAM bytes per launch of a layer's kernel from the ncu record in
+    profiles/dram_traffic.txt, or None when there is no record or the
+    kernel's sources changed since it was taken."""
+    import hashlib
+    try:
+        lines = open(os.path.join(ROOT, "profiles", "dram_traffic.txt")).read().splitlines()
+    except OSError:
+        return None
+    for line in lines:
+        if not line.strip() or line.startswith("#"):
+            continue
+        r = json.loads(line)
+        if (r["workload"], r["batch"], r["layer"]) != (workload, batch, layer):
+            continue
+        h = hashlib.sha256()
+        for s in r["sources"]:
+            h.update(open(os.path.join(ROOT, s), "rb").read())
+        if h.hexdigest() == r["sha256"]:
+            return r["dram_read_bytes"] + r["dram_write_bytes"]
+    return None
+
+
 def main():
     a = parse()
     if a.impl == "reference":
@@ -288,11 +326,9 @@ def main():
     clk = clocks.stop(t0, t1)
     ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
     if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+        ms = max_over_ranks(ms, dev)
     ms_per_step = ms / a.steps
-    value = N * world * a.steps / (ms / 1e3)
+    value = job_throughput(N, world, a.steps, ms / 1e3)
 
     # ---- per-stage timing: the same layers launched one by one, events between
     conv_costs, per_layer = [], []
@@ -354,7 +390,9 @@ def main():
         "achieved": round(dom_alg / (dom["ms"] / 1e3) / 1e9, 1),
         "peak": round(smem_peak_gbs, 1), "unit": "GB/s",
         "frac": round(dom_alg / (dom["ms"] / 1e3) / 1e9 / smem_peak_gbs, 4),
-        "traffic": None,
+        "traffic": recorded_traffic(WORKLOAD, N, dom["layer"]),
+        "traffic_note": "DRAM read+write bytes per launch (ncu, profiles/dram_traffic.txt); "
+                        "the kernel's algorithmic traffic is shared-memory, not DRAM",
         "peak_basis": f"{nsm} SMs x 128 B/clk shared-memory loads x {sm_max:.0f} MHz max SM clock",
         "alg_bytes_per_launch": dom_alg,
     }
@@ -372,10 +410,8 @@ def main():
         net.forward_host(x_host, y_host, ws_h)
         e2e_t += time.perf_counter() - t
     if world > 1:
-        t = torch.tensor([e2e_t], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_t = float(t.item())
-    e2e = {"value": N * world * a.steps / e2e_t, "unit": "images/s",
+        e2e_t = max_over_ranks(e2e_t, dev)
+    e2e = {"value": job_throughput(N, world, a.steps, e2e_t), "unit": "images/s",
            "h2d_bytes_per_step": x_host.numel() * 4, "d2h_bytes_per_step": y_host.numel() * 4}
 
     # ---- batch 1 latency (plain launches)

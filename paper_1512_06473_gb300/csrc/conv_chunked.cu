@@ -46,34 +46,54 @@ __host__ __device__ inline int chunk_phase_off(const ChunkGeom &g, int ky, int k
 }
 
 // ------------------------------------------------------------------ prep --
-// One thread per (m, ct): entries[m][ct][*] = byte offsets sorted by chunk,
-// starts[m][ct][c] = first entry of chunk c (NCH + 1 values).
+// One CTA per (m, ct), one thread per kernel offset p_k (kk <= kMaxPrepKK):
+// entries[m][ct][*] = byte offsets grouped by chunk, in p_k order inside a
+// chunk (a stable counting sort, so the gather order -- and the rounding --
+// is the same on every call); starts[m][ct][c] = first entry of chunk c.
+constexpr int kMaxPrepKK = 1024;
+
 __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed, int CtP,
                                   int Ct, int kk, int M, int K, ChunkGeom g,
                                   uint32_t *__restrict__ entries, int *__restrict__ starts) {
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= M * Ct) return;
+    extern __shared__ int psh[];  // wcount[NW][NCH], bstart[NCH + 1]
+    const int nw = blockDim.x / 32;
+    int *wcount = psh, *bstart = psh + nw * g.NCH;
+    const int i = blockIdx.x;
     const int m = i / Ct, ct = i % Ct;
-    auto code_at = [&](int pk) -> int {
-        const int c = packed ? codes[((size_t)m * kk + pk) * CtP + ct]
-                             : codes[((size_t)ct * kk + pk) * M + m];
-        return min(c, K - 1);
-    };
-    int *st = starts + (size_t)i * (g.NCH + 1);
-    for (int c = 0; c <= g.NCH; ++c) st[c] = 0;
-    for (int pk = 0; pk < kk; ++pk) st[code_at(pk) / g.KC + 1] += 1;
-    for (int c = 0; c < g.NCH; ++c) st[c + 1] += st[c];
-    uint32_t *en = entries + (size_t)i * kk;
-    // stable placement: a pass per chunk keeps p_k order inside a chunk
-    for (int c = 0; c < g.NCH; ++c) {
-        int pos = st[c];
-        for (int pk = 0; pk < kk; ++pk) {
-            const int code = code_at(pk);
-            if (code / g.KC != c) continue;
-            const int ky = pk / g.kw, kx = pk % g.kw;
-            en[pos++] = (uint32_t)(4 * ((code - c * g.KC) * g.SK + chunk_phase_off(g, ky, kx)));
-        }
+    const int pk = threadIdx.x, lane = pk & 31, warp = pk >> 5;
+    int code = 0, b = -1;
+    if (pk < kk) {
+        code = packed ? codes[((size_t)m * kk + pk) * CtP + ct] : codes[((size_t)ct * kk + pk) * M + m];
+        code = min(code, K - 1);
+        b = code / g.KC;
     }
+    for (int e = threadIdx.x; e < nw * g.NCH; e += blockDim.x) wcount[e] = 0;
+    __syncthreads();
+    const unsigned same = __match_any_sync(0xffffffffu, b);  // lanes of this warp in chunk b
+    const int rank = __popc(same & ((1u << lane) - 1u));
+    if (b >= 0 && rank == 0) wcount[warp * g.NCH + b] = __popc(same);
+    __syncthreads();
+    if (threadIdx.x == 0) {  // exclusive prefix over (chunk, warp)
+        int run = 0;
+        for (int c = 0; c < g.NCH; ++c) {
+            bstart[c] = run;
+            for (int w = 0; w < nw; ++w) {
+                const int v = wcount[w * g.NCH + c];
+                wcount[w * g.NCH + c] = run;
+                run += v;
+            }
+        }
+        bstart[g.NCH] = run;
+    }
+    __syncthreads();
+    if (b >= 0) {
+        const int pos = wcount[warp * g.NCH + b] + rank;
+        const int ky = pk / g.kw, kx = pk % g.kw;
+        entries[(size_t)i * kk + pos] =
+            (uint32_t)(4 * ((code - b * g.KC) * g.SK + chunk_phase_off(g, ky, kx)));
+    }
+    for (int c = threadIdx.x; c <= g.NCH; c += blockDim.x)
+        starts[(size_t)i * (g.NCH + 1) + c] = bstart[c];
 }
 
 // ---------------------------------------------------------------- kernel --
@@ -277,7 +297,7 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
         if (force >= 0 && v != force) continue;
 #endif
         const ChunkVariant &cv = kChunk[v];
-        if (s.Csp > cv.CSPT) continue;
+        if (s.Csp > cv.CSPT || s.kh * s.kw > kMaxPrepKK) continue;
         const int ct_cta = 16 * cv.CTW;
         // largest band that the variant's lanes and registers cover
         for (int TH = std::min(s.Ho, 64); TH >= 1; --TH) {
@@ -335,8 +355,9 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
     uint32_t *entries = static_cast<uint32_t *>(ws);
     int *starts = reinterpret_cast<int *>(static_cast<uint8_t *>(ws) + p.entries_bytes);
     const int kk = s.kh * s.kw;
-    const int nthreads = s.M * s.Ct;
-    chunk_prep_kernel<<<cdiv(nthreads, 128), 128, 0, st>>>(codes, codes_packed, packed_ct(s.Ct),
+    const int pthreads = cdiv(kk, 32) * 32;
+    const size_t psmem = ((size_t)(pthreads / 32) * g.NCH + g.NCH + 1) * sizeof(int);
+    chunk_prep_kernel<<<s.M * s.Ct, pthreads, psmem, st>>>(codes, codes_packed, packed_ct(s.Ct),
                                                           s.Ct, kk, s.M, s.K, g, entries, starts);
     qcnn_status rc = after_launch();
     if (rc != QCNN_OK) return rc;
