@@ -35,6 +35,8 @@ struct FcArgs {
     int NTP;     // odd pitch of a table row (>= NT)
     int NTX;     // odd pitch of a staged x row (>= NT)
     int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
+    int cvec_log2;
+    int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
 };
 
 constexpr int kFcThreads = 256;
@@ -60,6 +62,9 @@ __host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int NTP, int NT
 template <int NW, int WN, int MINB>
 __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs a) {
     constexpr int CT_CTA = (8 / WN) * 32 * kCPL;
+    constexpr int kCtCtaLog2 = CT_CTA == 1024 ? 10 : (CT_CTA == 512 ? 9 : 8);
+    static_assert((1 << kCtCtaLog2) == CT_CTA, "output tile must be 256, 512 or 1024");
+    constexpr int NT = NW * WN;  // images per CTA (== a.NT)
     extern __shared__ __align__(16) unsigned char smem[];
     const FcSmem L = fc_smem_layout(a.MCH, a.K, a.NTP, a.NTX, a.Csp, CT_CTA);
     float *lut = reinterpret_cast<float *>(smem + L.lut);
@@ -83,8 +88,11 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         const int m0 = c * a.MCH;
         const int mch = min(a.MCH, a.M - m0);
         float *xb = xs + (size_t)b * CCH * a.NTX;
-        for (int e = tid; e < CCH * a.NT; e += kFcThreads) {
-            const int cc = e % CCH, nn = e / CCH;
+        // (image nn, float cc) with cc on a power-of-two stride: no division
+        const int cmask = (1 << a.cch_log2) - 1;
+        for (int e = tid; e < (NT << a.cch_log2); e += kFcThreads) {
+            const int cc = e & cmask, nn = e >> a.cch_log2;
+            if (cc >= CCH) continue;
             const bool ok = cc < mch * a.Csp && n0 + nn < a.N;
             const float *src = ok ? a.x + (size_t)(n0 + nn) * a.Cs + (size_t)m0 * a.Csp + cc : a.x;
             cp_async4(xb + cc * a.NTX + nn, src, ok);
@@ -96,9 +104,10 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         // codes[m0 + mm][ct0 .. ct0 + CT_CTA) -> cs[b][mm][.]; zero outside
         uint8_t *cb = cs + (size_t)b * a.MCH * CT_CTA;
         if (a.cvec > 0) {
-            const int per_row = CT_CTA / a.cvec;
+            const int row_log2 = kCtCtaLog2 - a.cvec_log2;  // copies per code row
+            const int per_row = 1 << row_log2;
             for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
-                const int mm = e / per_row, q = e % per_row;
+                const int mm = e >> row_log2, q = e & (per_row - 1);
                 const int ct = ct0 + q * a.cvec;
                 const bool ok = mm < mch && ct < a.Ct;  // Ct % cvec == 0: all or nothing
                 const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
@@ -136,22 +145,22 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         __syncthreads();  // chunk c staged; gather of c-1 finished
         if (c + 1 < c_end) stage(c + 1, b ^ 1);
 
-        // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>
+        // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>; (k, nn) with nn
+        // fastest over the compile-time image tile: no division
         {
             const float *xb = xs + (size_t)b * CCH * a.NTX;
             const float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
-            const int tot = a.MCH * a.K * a.NT;
-            for (int e = tid; e < tot; e += kFcThreads) {
-                const int nn = e % a.NT;
-                const int r = e / a.NT;
-                const int k = r % a.K, mm = r / a.K;
-                const float *xp = xb + mm * a.Csp * a.NTX + nn;
-                const float *dp = db + (mm * a.K + k) * a.Csp;
-                float v = 0.f;
+            for (int mm = 0; mm < mch; ++mm) {
+                for (int e = tid; e < a.K * NT; e += kFcThreads) {
+                    const int nn = e % NT, k = e / NT;
+                    const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                    const float *dp = db + (mm * a.K + k) * a.Csp;
+                    float v = 0.f;
 #pragma unroll
-                for (int j = 0; j < kMaxCsp; ++j)
-                    if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
-                lut[(mm * a.K + k) * a.NTP + nn] = v;
+                    for (int j = 0; j < kMaxCsp; ++j)
+                        if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
+                    lut[(mm * a.K + k) * a.NTP + nn] = v;
+                }
             }
         }
         __syncthreads();
@@ -311,6 +320,9 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
              : (s.Ct % 8 == 0 && base % 8 == 0) ? 8
              : (s.Ct % 4 == 0 && base % 4 == 0) ? 4
                                                  : 0;
+    a.cvec_log2 = a.cvec == 16 ? 4 : a.cvec == 8 ? 3 : 2;
+    a.cch_log2 = 0;
+    while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
