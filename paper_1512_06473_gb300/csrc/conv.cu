@@ -71,6 +71,8 @@ struct ConvFusedArgs {
     int N, Cs, H, W, Ct, kh, kw, pad, Csp, K, M, Ho, Wo;
     int pitch, TH, KS, HP, CtP, relu;
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
+    int splits, m_per_split;    // sub-space ranges over several CTAs (small batches)
+    float *__restrict__ partial;  // [splits][N][Ct][Ho][Wo] when splits > 1
 };
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
@@ -142,7 +144,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     const int wp = warp % WP, wc = warp / WP;
     const int oy0 = blockIdx.x * a.TH;
     const int ct0 = blockIdx.y * CT_CTA;
-    const int n = blockIdx.z;
+    const int n = blockIdx.z / a.splits, split = blockIdx.z % a.splits;
     const int HW = a.H * a.W;
 
     // Halo position h -> offset iy*W + ix inside one input plane, or -1 where
@@ -256,15 +258,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     };
 
+    // sub-spaces [mb, me) of this CTA (all of them unless M is split)
+    const int mb = split * a.m_per_split, me = min(a.M, mb + a.m_per_split);
     if constexpr (!PIPE) {
-        stage_xd(0, 0);
-        stage_codes(0, 0);
+        stage_xd(mb, 0);
+        stage_codes(mb, 0);
         cp_async_commit();
-        for (int m = 0; m < a.M; ++m) {
-            const int b = m & 1;
+        for (int m = mb; m < me; ++m) {
+            const int b = (m - mb) & 1;
             cp_async_wait<0>();
             __syncthreads();  // stage m visible; gather of m-1 finished everywhere
-            if (m + 1 < a.M) {
+            if (m + 1 < me) {
                 stage_xd(m + 1, b ^ 1);
                 stage_codes(m + 1, b ^ 1);
                 cp_async_commit();
@@ -275,28 +279,28 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     } else {
         float *lut1 = lut0 + (size_t)K * KS;
-        stage_xd(0, 0);
-        if (a.M > 1) stage_xd(1, 1);
-        stage_codes(0, 0);
+        stage_xd(mb, 0);
+        if (mb + 1 < me) stage_xd(mb + 1, 1);
+        stage_codes(mb, 0);
         cp_async_commit();
         cp_async_wait<0>();
         __syncthreads();
         build(0, lut0);
         __syncthreads();
-        // Iteration m: table m ready in buffer m&1, codes m in code buffer m&1,
-        // inputs of m+1 in staging buffer (m+1)&1.
-        for (int m = 0; m < a.M; ++m) {
-            const int b = m & 1;
-            if (m + 2 < a.M) stage_xd(m + 2, b);
-            if (m + 1 < a.M) stage_codes(m + 1, b ^ 1);
+        // Iteration m (b = (m - mb) & 1): table m ready in buffer b, codes m in
+        // code buffer b, inputs of m+1 in staging buffer b^1.
+        for (int m = mb; m < me; ++m) {
+            const int b = (m - mb) & 1;
+            if (m + 2 < me) stage_xd(m + 2, b);
+            if (m + 1 < me) stage_codes(m + 1, b ^ 1);
             cp_async_commit();
             // even warps build first, odd warps gather first: the latency-bound
             // table build of one half overlaps the other half's gather
             if (warp & 1) {
                 gather(b, b ? lut1 : lut0);
-                if (m + 1 < a.M) build(b ^ 1, b ? lut0 : lut1);
+                if (m + 1 < me) build(b ^ 1, b ? lut0 : lut1);
             } else {
-                if (m + 1 < a.M) build(b ^ 1, b ? lut0 : lut1);
+                if (m + 1 < me) build(b ^ 1, b ? lut0 : lut1);
                 gather(b, b ? lut1 : lut0);
             }
             cp_async_wait<0>();
@@ -304,7 +308,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     }
 
-    // ---- epilogue: bias, ReLU, store --------------------------------------
+    // ---- epilogue: bias, ReLU, store (or raw partial sums of a split) -----
 #pragma unroll
     for (int c = 0; c < CTW; ++c) {
         const int ct = ct0 + wc * CTW + c;
@@ -316,11 +320,31 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             const int r = l / pitch, col = l - r * pitch;
             const int oy = oy0 + r;
             if (r < a.TH && col < a.Wo && oy < a.Ho) {
-                float v = acc[c][p] + bv;
-                if (a.relu) v = fmaxf(v, 0.f);
-                a.y[(((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + col] = v;
+                const size_t o = (((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
+                if (a.splits > 1) {
+                    a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
+                } else {
+                    float v = acc[c][p] + bv;
+                    if (a.relu) v = fmaxf(v, 0.f);
+                    a.y[o] = v;
+                }
             }
         }
+    }
+}
+
+// y = bias + sum over splits of the partial sums, in split order; then ReLU.
+__global__ void conv_split_reduce_kernel(const float *__restrict__ partial, int splits,
+                                         size_t total, int Ct, int HoWo,
+                                         const float *__restrict__ bias, int relu,
+                                         float *__restrict__ y) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        float v = 0.f;
+        for (int s = 0; s < splits; ++s) v += partial[(size_t)s * total + i];
+        if (bias) v += bias[(i / HoWo) % Ct];
+        if (relu) v = fmaxf(v, 0.f);
+        y[i] = v;
     }
 }
 
@@ -407,15 +431,35 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
         const int ct_tiles = cdiv(s.Ct, ct_cta);
         const double ctas = (double)s.N * row_tiles * ct_tiles;
-        const double waves = std::ceil(ctas / (sms * cps));
-        // work per CTA in shared-memory wavefronts: gather (incl. lanes on
-        // discarded positions and channels past Ct) over the variant's measured
-        // efficiency, plus the exposed part of the table build (which costs
-        // about 4 wavefronts of time per 32 entries: latency-bound FMA chains)
-        const double gather = (double)slots * ct_cta * kk * s.M;
-        const double build = (double)HP * s.K * s.M * 4.0 / 32.0;
-        const double score = waves * (gather / fv.eff + build * fv.build) * cps;
+        // work per CTA and sub-space in shared-memory wavefronts (~cycles):
+        // gather (incl. lanes on discarded positions and channels past Ct)
+        // over the variant's measured efficiency, plus the exposed part of the
+        // table build (about 4 wavefronts of time per 32 entries:
+        // latency-bound FMA chains)
+        const double per_m = (double)slots * ct_cta * kk / fv.eff +
+                             (double)HP * s.K * 4.0 / 32.0 * fv.build;
+        // Small batches: split the sub-spaces of each tile over `splits` CTAs
+        // (partial sums through the workspace, then a reduction) when the
+        // grid would leave SMs idle.
+        int splits = 1;
+        double score = 0;
+        for (int sp = 1; sp <= std::min(s.M, 64); sp *= 2) {
+            const int mps = cdiv(s.M, sp);
+            const int sp_eff = cdiv(s.M, mps);
+            const double waves = std::ceil(ctas * sp_eff / (sms * cps));
+            const double part = sp_eff > 1 ? 2.0 * sp_eff * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
+            const double sc = waves * per_m * mps * cps + part / 3000.0 + (sp_eff > 1 ? 6000.0 : 0.0);
+            if (sp == 1 || sc < score) {
+                score = sc;
+                splits = sp_eff;
+            }
+            if (ctas * sp >= 2.0 * sms * cps) break;
+        }
         if (!best.ok || score < best.score) {
+            best.splits = splits;
+            best.m_per_split = cdiv(s.M, splits);
+            best.partial_bytes =
+                splits > 1 ? (size_t)splits * s.N * s.Ct * s.Ho * s.Wo * sizeof(float) : 0;
             best.ok = true;
             best.variant = v;
             best.P = fv.P;
@@ -444,7 +488,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
 
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias,
-                              float *y, int relu, cudaStream_t st) {
+                              float *y, int relu, float *partial_ws, cudaStream_t st) {
     const FusedVariant &fv = kFused[p.variant];
     ConvFusedArgs a;
     a.x = x;
@@ -472,11 +516,20 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.CtP = packed_ct(s.Ct);
     a.relu = relu;
     a.xs_floats = cdiv(p.HP, 4) * 4 * fv.CSP4;
+    a.splits = p.splits;
+    a.m_per_split = p.m_per_split;
+    a.partial = partial_ws;
     cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
-    dim3 grid(p.row_tiles, p.ct_tiles, s.N);
+    dim3 grid(p.row_tiles, p.ct_tiles, s.N * p.splits);
     fv.fn<<<grid, fv.NW * 32, p.smem, st>>>(a);
+    qcnn_status rc = after_launch();
+    if (rc != QCNN_OK || p.splits == 1) return rc;
+    const size_t total = (size_t)s.N * s.Ct * s.Ho * s.Wo;
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
+    conv_split_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, total, s.Ct,
+                                                     s.Ho * s.Wo, bias, relu, y);
     return after_launch();
 }
 

@@ -120,6 +120,8 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         off += align_up(c->up.lut_bytes, kWsAlign);
     } else if (c->algo == QCNN_ALGO_CHUNKED) {
         off += c->cp.entries_bytes + c->cp.starts_bytes;
+    } else {
+        off += align_up(c->fp.partial_bytes, kWsAlign);
     }
     c->total = off;
     return QCNN_OK;
@@ -140,7 +142,9 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
         packed = p;
     }
     if (c.algo == QCNN_ALGO_FUSED)
-        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, st);
+        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu,
+                                 reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off),
+                                 st);
     float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
     return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
 }

@@ -42,6 +42,9 @@ struct ConvFusedPlan {
     int HP;             // halo positions with data: (TH + kh - 1) * pitch
     int ct_cta;         // channels per CTA
     int row_tiles, ct_tiles;
+    int splits = 1;     // CTAs sharing one tile's sub-spaces (small batches)
+    int m_per_split;
+    size_t partial_bytes = 0;  // workspace for split partial sums
     size_t smem;        // dynamic shared memory bytes
     double score;       // estimated cost (lower is better)
 };
@@ -74,10 +77,11 @@ int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
 
 qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K,
                               uint8_t *packed, cudaStream_t st);
+// partial_ws: p.partial_bytes of workspace (unused when p.splits == 1)
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p,
                               const float *x, const float *D,
                               const uint8_t *packed, const float *bias, float *y,
-                              int relu, cudaStream_t st);
+                              int relu, float *partial_ws, cudaStream_t st);
 qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
                                 const float *x, const float *D,
                                 const uint8_t *packed, const float *bias,
