@@ -14,6 +14,9 @@ Paper: Wu et al., "Quantized Convolutional Neural Networks for Mobile Devices"
   - FC layer response: Sec. 3.1, Eq. 5 and the look-up-table paragraph after it.
   - Conv layer response: Sec. 3.2, Eq. 7 and the paragraph after it.
   - Whole network (conv/pool/FC stack): Sec. 4.2.3, Table 8.
+  - ``lut_bf16=True``: every table entry rounded to bfloat16 (nearest, ties to
+    even) before the sums, the rounding model of the library's reduced-precision
+    table variant; ``round_bf16`` exposes that rounding.
 
 Array conventions (all numpy):
   fc:   x [N, Cs], codebooks D [M, K, Csp], codes [M, Ct] uint8, bias [Ct]
@@ -44,7 +47,7 @@ def compile_c(src: str, out: str) -> str:
     no fast-math, no fused multiply-add contraction, so x86 and Arm agree)."""
     os.makedirs(os.path.dirname(out) or ".", exist_ok=True)
     tmp = out + f".tmp{os.getpid()}"
-    subprocess.run(["gcc", *GCC_FLAGS, "-o", tmp, src], check=True)
+    subprocess.run(["gcc", *GCC_FLAGS, "-o", tmp, src, "-lm"], check=True)
     os.replace(tmp, out)
     return out
 
@@ -88,28 +91,36 @@ class Oracle:
     def __init__(self, so_path: str):
         lib = ctypes.CDLL(so_path)
         i = ctypes.c_int
-        lib.qo_fc_lut.argtypes = [_D, i, i, _D, i, i, _D]
-        lib.qo_fc_forward.argtypes = [_D, i, i, i, _D, i, i, _U8, _D, i, _D]
-        lib.qo_conv_lut.argtypes = [_D, i, i, i, i, _D, i, i, _D]
+        lib.qo_fc_lut.argtypes = [_D, i, i, _D, i, i, i, _D]
+        lib.qo_fc_forward.argtypes = [_D, i, i, i, _D, i, i, _U8, _D, i, i, _D]
+        lib.qo_conv_lut.argtypes = [_D, i, i, i, i, _D, i, i, i, _D]
         lib.qo_conv_forward.argtypes = [_D, i, i, i, i, i, i, i, i, i, _D,
-                                        i, i, _U8, _D, i, _D]
+                                        i, i, _U8, _D, i, i, _D]
+        lib.qo_round_bf16.argtypes = [ctypes.c_double]
+        lib.qo_round_bf16.restype = ctypes.c_double
         lib.qo_maxpool.argtypes = [_D, i, i, i, i, i, i, _D]
         for f in (lib.qo_fc_lut, lib.qo_fc_forward, lib.qo_conv_lut,
                   lib.qo_conv_forward, lib.qo_maxpool):
             f.restype = ctypes.c_int
         self.lib = lib
 
-    def fc_lut(self, x, D):
+    def round_bf16(self, v):
+        """Each value rounded to the nearest bfloat16 (ties to even)."""
+        v = _f64(v)
+        return np.array([self.lib.qo_round_bf16(float(e)) for e in v.ravel()],
+                        np.float64).reshape(v.shape)
+
+    def fc_lut(self, x, D, lut_bf16=False):
         """LUT[n, m, k] = <x[n, m*Csp:(m+1)*Csp], D[m, k, :]> (Sec. 3.1)."""
         x, D = _f64(x), _f64(D)
         N, Cs = x.shape
         M, K, Csp = D.shape
         out = np.empty((N, M, K), np.float64)
         _check(self.lib.qo_fc_lut(_p(x, _D), N, Cs, _p(D, _D), Csp, K,
-                                  _p(out, _D)), "fc_lut")
+                                  int(bool(lut_bf16)), _p(out, _D)), "fc_lut")
         return out
 
-    def fc_forward(self, x, D, codes, bias=None, relu=False):
+    def fc_forward(self, x, D, codes, bias=None, relu=False, lut_bf16=False):
         """Eq. 5: y[n, ct] = bias[ct] + sum_m LUT[n, m, codes[m, ct]]."""
         x, D, codes = _f64(x), _f64(D), _u8(codes)
         N, Cs = x.shape
@@ -121,11 +132,11 @@ class Oracle:
         y = np.empty((N, Ct), np.float64)
         _check(self.lib.qo_fc_forward(
             _p(x, _D), N, Cs, Ct, _p(D, _D), Csp, K, _p(codes, _U8),
-            None if b is None else _p(b, _D), int(bool(relu)), _p(y, _D)),
-            "fc_forward")
+            None if b is None else _p(b, _D), int(bool(relu)),
+            int(bool(lut_bf16)), _p(y, _D)), "fc_forward")
         return y
 
-    def conv_lut(self, x, D):
+    def conv_lut(self, x, D, lut_bf16=False):
         """LUT[n, m, iy*W+ix, k] = <x[n, m*Csp:(m+1)*Csp, iy, ix], D[m, k]>
         (Sec. 3.2: one table per input position)."""
         x, D = _f64(x), _f64(D)
@@ -133,11 +144,11 @@ class Oracle:
         M, K, Csp = D.shape
         out = np.empty((N, M, H * W, K), np.float64)
         _check(self.lib.qo_conv_lut(_p(x, _D), N, Cs, H, W, _p(D, _D), Csp, K,
-                                    _p(out, _D)), "conv_lut")
+                                    int(bool(lut_bf16)), _p(out, _D)), "conv_lut")
         return out
 
     def conv_forward(self, x, D, codes, kh, kw, stride=1, pad=0, bias=None,
-                     relu=False):
+                     relu=False, lut_bf16=False):
         """Eq. 7: y[n, ct, oy, ox] = bias[ct] + sum_{(pk, ps)} sum_m
         LUT[n, m, ps, codes[ct, pk, m]], ps = (oy*s - pad + ky, ox*s - pad + kx)."""
         x, D, codes = _f64(x), _f64(D), _u8(codes)
@@ -153,7 +164,7 @@ class Oracle:
         _check(self.lib.qo_conv_forward(
             _p(x, _D), N, Cs, H, W, Ct, kh, kw, stride, pad, _p(D, _D), Csp, K,
             _p(codes, _U8), None if b is None else _p(b, _D), int(bool(relu)),
-            _p(y, _D)), "conv_forward")
+            int(bool(lut_bf16)), _p(y, _D)), "conv_forward")
         return y
 
     def maxpool(self, x, k, s):
@@ -173,6 +184,7 @@ class Oracle:
           {"kind": "conv", "D", "codes", "bias", "kh", "kw", "stride", "pad", "relu"}
           {"kind": "maxpool", "k", "s"}
           {"kind": "fc", "D", "codes", "bias", "relu"}
+        plus an optional "lut_bf16" on conv and fc layers.
         A conv/pool output feeding an FC layer is flattened in C*H*W order.
         """
         h = _f64(x)
@@ -182,14 +194,15 @@ class Oracle:
             if kind == "conv":
                 h = self.conv_forward(h, L["D"], L["codes"], L["kh"], L["kw"],
                                       L.get("stride", 1), L.get("pad", 0),
-                                      L.get("bias"), L.get("relu", False))
+                                      L.get("bias"), L.get("relu", False),
+                                      L.get("lut_bf16", False))
             elif kind == "maxpool":
                 h = self.maxpool(h, L["k"], L["s"])
             elif kind == "fc":
                 if h.ndim != 2:
                     h = h.reshape(h.shape[0], -1)
                 h = self.fc_forward(h, L["D"], L["codes"], L.get("bias"),
-                                    L.get("relu", False))
+                                    L.get("relu", False), L.get("lut_bf16", False))
             else:
                 raise OracleError(f"unknown layer kind {kind!r}")
             outs.append(h)
@@ -209,20 +222,26 @@ def default() -> Oracle:
     return _default
 
 
-def fc_lut(x, D):
-    return default().fc_lut(x, D)
+def round_bf16(v):
+    return default().round_bf16(v)
 
 
-def fc_forward(x, D, codes, bias=None, relu=False):
-    return default().fc_forward(x, D, codes, bias, relu)
+def fc_lut(x, D, lut_bf16=False):
+    return default().fc_lut(x, D, lut_bf16)
 
 
-def conv_lut(x, D):
-    return default().conv_lut(x, D)
+def fc_forward(x, D, codes, bias=None, relu=False, lut_bf16=False):
+    return default().fc_forward(x, D, codes, bias, relu, lut_bf16)
 
 
-def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False):
-    return default().conv_forward(x, D, codes, kh, kw, stride, pad, bias, relu)
+def conv_lut(x, D, lut_bf16=False):
+    return default().conv_lut(x, D, lut_bf16)
+
+
+def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False,
+                 lut_bf16=False):
+    return default().conv_forward(x, D, codes, kh, kw, stride, pad, bias, relu,
+                                  lut_bf16)
 
 
 def maxpool(x, k, s):

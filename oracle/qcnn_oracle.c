@@ -31,10 +31,17 @@
  * All arithmetic is IEEE double; build with -ffp-contract=off so that the
  * result does not depend on whether the host fuses multiply-adds.
  *
+ * Reduced-precision tables: with lut_bf16 = 1 every table entry is rounded
+ * to bfloat16 (8 significant bits, round to nearest, ties to even) before
+ * it is summed; the sums stay exact in double.  The paper builds its tables
+ * in full precision; this models the reduced-precision table variant of
+ * the library.  The entry is rounded from its exact value.
+ *
  * Every function returns 0 on success and a negative value on an invalid
  * argument (non-positive size, C_s not a multiple of C'_s, K outside
  * [1, 256], a code >= K) or an allocation failure.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 
@@ -45,13 +52,31 @@
 
 typedef long long i64;
 
+/*
+ * Round v to the nearest bfloat16 value, ties to even.  bfloat16 keeps the
+ * 8-bit exponent of binary32 and 8 significant bits (7 stored): write
+ * v = f * 2^e with 0.5 <= |f| < 1, scale f to an integer significand
+ * f * 2^8 in [128, 256), round that to an integer (nearbyint rounds to
+ * nearest, ties to even, in the default rounding mode) and scale back.
+ * Values below the binary32 normal range are not handled (the tests keep
+ * far from them).
+ */
+double qo_round_bf16(double v)
+{
+    if (v == 0.0 || !isfinite(v)) return v;
+    int e;
+    const double f = frexp(v, &e);
+    return ldexp(nearbyint(ldexp(f, 8)), e - 8);
+}
+
 /* ------------------------------------------------------------------ */
 /* Look-up table of one input vector (Sec. 3.1, the paragraph after    */
 /* Eq. 5): for every sub-space m and every sub-codeword k,             */
 /*     LUT[m][k] = < S^(m), D^(m)_k > = sum_j S[m*C'_s + j] * D[m][k][j] */
 /* ------------------------------------------------------------------ */
 static void lut_of_vector(const double *s, i64 s_stride, int M, int Csp,
-                          int K, const double *D, double *lut /* [M][K] */)
+                          int K, const double *D, int lut_bf16,
+                          double *lut /* [M][K] */)
 {
     for (int m = 0; m < M; ++m) {
         for (int k = 0; k < K; ++k) {
@@ -59,7 +84,7 @@ static void lut_of_vector(const double *s, i64 s_stride, int M, int Csp,
             double acc = 0.0;
             for (int j = 0; j < Csp; ++j)
                 acc += s[(i64)(m * Csp + j) * s_stride] * dk[j];
-            lut[(i64)m * K + k] = acc;
+            lut[(i64)m * K + k] = lut_bf16 ? qo_round_bf16(acc) : acc;
         }
     }
 }
@@ -83,13 +108,14 @@ static int check_codes(const uint8_t *codes, i64 n, int K)
  * x: [N][Cs]; D: [M][K][Csp]; lut: [N][M][K].
  */
 int qo_fc_lut(const double *x, int N, int Cs, const double *D, int Csp, int K,
-              double *lut)
+              int lut_bf16, double *lut)
 {
     int rc = check_pq(Cs, Csp, K);
     if (rc || N <= 0) return QO_EINVAL;
     const int M = Cs / Csp;
     for (int n = 0; n < N; ++n)
-        lut_of_vector(x + (i64)n * Cs, 1, M, Csp, K, D, lut + (i64)n * M * K);
+        lut_of_vector(x + (i64)n * Cs, 1, M, Csp, K, D, lut_bf16,
+                      lut + (i64)n * M * K);
     return QO_OK;
 }
 
@@ -102,7 +128,7 @@ int qo_fc_lut(const double *x, int N, int Cs, const double *D, int Csp, int K,
  */
 int qo_fc_forward(const double *x, int N, int Cs, int Ct, const double *D,
                   int Csp, int K, const uint8_t *codes, const double *bias,
-                  int relu, double *y)
+                  int relu, int lut_bf16, double *y)
 {
     int rc = check_pq(Cs, Csp, K);
     if (rc || N <= 0 || Ct <= 0) return QO_EINVAL;
@@ -111,7 +137,7 @@ int qo_fc_forward(const double *x, int N, int Cs, int Ct, const double *D,
     double *lut = (double *)malloc(sizeof(double) * (size_t)M * K);
     if (!lut) return QO_ENOMEM;
     for (int n = 0; n < N; ++n) {
-        lut_of_vector(x + (i64)n * Cs, 1, M, Csp, K, D, lut);
+        lut_of_vector(x + (i64)n * Cs, 1, M, Csp, K, D, lut_bf16, lut);
         for (int ct = 0; ct < Ct; ++ct) {
             double t = 0.0;
             for (int m = 0; m < M; ++m)
@@ -132,7 +158,7 @@ int qo_fc_forward(const double *x, int N, int Cs, int Ct, const double *D,
  * x: [N][Cs][H][W] (NCHW); lut: [N][M][H*W][K].
  */
 int qo_conv_lut(const double *x, int N, int Cs, int H, int W, const double *D,
-                int Csp, int K, double *lut)
+                int Csp, int K, int lut_bf16, double *lut)
 {
     int rc = check_pq(Cs, Csp, K);
     if (rc || N <= 0 || H <= 0 || W <= 0) return QO_EINVAL;
@@ -143,7 +169,7 @@ int qo_conv_lut(const double *x, int N, int Cs, int H, int W, const double *D,
     for (int n = 0; n < N; ++n) {
         const double *xn = x + (i64)n * Cs * P;
         for (i64 p = 0; p < P; ++p) {
-            lut_of_vector(xn + p, P, M, Csp, K, D, row);
+            lut_of_vector(xn + p, P, M, Csp, K, D, lut_bf16, row);
             for (int m = 0; m < M; ++m)
                 for (int k = 0; k < K; ++k)
                     lut[(((i64)n * M + m) * P + p) * K + k] = row[(i64)m * K + k];
@@ -166,7 +192,7 @@ int qo_conv_lut(const double *x, int N, int Cs, int H, int W, const double *D,
 int qo_conv_forward(const double *x, int N, int Cs, int H, int W, int Ct,
                     int kh, int kw, int stride, int pad, const double *D,
                     int Csp, int K, const uint8_t *codes, const double *bias,
-                    int relu, double *y)
+                    int relu, int lut_bf16, double *y)
 {
     int rc = check_pq(Cs, Csp, K);
     if (rc || N <= 0 || H <= 0 || W <= 0 || Ct <= 0 || kh <= 0 || kw <= 0 ||
@@ -184,7 +210,8 @@ int qo_conv_forward(const double *x, int N, int Cs, int H, int W, int Ct,
     double *lut = (double *)malloc(sizeof(double) * (size_t)M * P * K);
     if (!lut) return QO_ENOMEM;
     for (int n = 0; n < N; ++n) {
-        rc = qo_conv_lut(x + (i64)n * Cs * P, 1, Cs, H, W, D, Csp, K, lut);
+        rc = qo_conv_lut(x + (i64)n * Cs * P, 1, Cs, H, W, D, Csp, K, lut_bf16,
+                         lut);
         if (rc) { free(lut); return rc; }
         for (int ct = 0; ct < Ct; ++ct) {
             for (int oy = 0; oy < Ho; ++oy) {

@@ -380,9 +380,92 @@ def pin_tiny_net(o):
     return [] if relerr(got, h.numpy()) < 1e-12 else [f"tiny net err {relerr(got, h.numpy())}"]
 
 
+def torch_bf16(v):
+    """torch's CPU float32 -> bfloat16 conversion (round to nearest even)."""
+    t = torch.from_numpy(np.asarray(v, np.float32)).to(torch.bfloat16)
+    return t.to(torch.float64).numpy()
+
+
+def pin_bf16_rounding(o):
+    """The bfloat16 rounding of the reduced-precision table model: equal to
+    torch's float32 -> bfloat16 conversion on float32 values of every scale,
+    and to hand-worked ties (8 significant bits, ties to even)."""
+    fails = []
+    r = _rng(31)
+    v = (r.standard_normal(3000) * 2.0 ** r.integers(-40, 40, 3000)).astype(np.float32)
+    v = np.concatenate([v, np.float32([0.0, 1.0, -1.0, 255.0, 1e30, -3e-30])])
+    got, ref = o.round_bf16(v.astype(np.float64)), torch_bf16(v)
+    if not np.array_equal(got, ref):
+        bad = int(np.sum(got != ref))
+        fails.append(f"{bad} values differ from torch's bfloat16 conversion")
+    e8 = 2.0 ** -8
+    worked = [
+        (1 + e8, 1.0),                         # tie: 1 has an even last bit
+        (1 + 3 * e8, 1 + 4 * e8),              # tie: 1 + 2^-7 has an odd last bit
+        (-(1 + e8), -1.0),
+        (1 + e8 + 2.0 ** -40, 1 + 2 * e8),     # just above the tie (not a float32)
+        (257.0, 256.0), (259.0, 260.0), (258.0, 258.0),
+        (0.1, 0.10009765625),                  # 0x3DCD
+        (-1000.0, -1000.0), (1001.0, 1000.0), (1003.0, 1004.0),
+    ]
+    for x, want in worked:
+        g = float(o.round_bf16(np.float64([x]))[0])
+        if g != want:
+            fails.append(f"round_bf16({x!r}) = {g!r}, expected {want!r}")
+    return fails
+
+
+def pin_bf16_tables(o):
+    """Reduced-precision tables, on integer data whose table entries (up to a
+    few thousand) are exact in double and in float32 but not in bfloat16:
+    the FC response must equal (rounded tables) @ (one-hot code matrix) and the
+    conv response a float64 conv2d of the rounded table maps with one-hot
+    code kernels (Eq. 7 read as a convolution over the (m, k) table
+    channels); tables built by torch, rounded by torch."""
+    fails = []
+    r = _rng(37)
+    for (N, Cs, Ct, Csp, K) in [(3, 24, 7, 4, 16), (2, 16, 5, 8, 3)]:
+        M = Cs // Csp
+        x = r.integers(-20, 21, (N, Cs)).astype(np.float64)
+        D = r.integers(-20, 21, (M, K, Csp)).astype(np.float64)
+        codes = r.integers(0, K, (M, Ct), dtype=np.uint8)
+        T = torch.einsum("nmj,mkj->nmk", torch.from_numpy(x.reshape(N, M, Csp)),
+                         torch.from_numpy(D)).numpy()
+        Tr = torch_bf16(T)
+        if np.array_equal(Tr, T):
+            fails.append("test data too small to exercise rounding")
+        onehot = np.zeros((M, K, Ct))
+        onehot[np.arange(M)[:, None], codes.astype(np.int64), np.arange(Ct)[None, :]] = 1.0
+        ref = Tr.reshape(N, M * K) @ onehot.reshape(M * K, Ct)
+        got = o.fc_forward(x, D, codes, lut_bf16=True)
+        if not np.array_equal(got, ref):
+            fails.append(f"fc bf16 tables: err {relerr(got, ref)}")
+    for (N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K) in [
+            (2, 8, 6, 7, 3, 3, 3, 1, 1, 4, 6), (1, 6, 9, 8, 2, 5, 3, 2, 2, 3, 5)]:
+        M = Cs // Csp
+        x = r.integers(-20, 21, (N, Cs, H, W)).astype(np.float64)
+        D = r.integers(-20, 21, (M, K, Csp)).astype(np.float64)
+        codes = r.integers(0, K, (Ct, kh * kw, M), dtype=np.uint8)
+        T = torch.einsum("nmjhw,mkj->nmkhw",
+                         torch.from_numpy(x.reshape(N, M, Csp, H, W)),
+                         torch.from_numpy(D)).numpy()
+        Tr = torch_bf16(T).reshape(N, M * K, H, W)
+        Wk = np.zeros((Ct, M, K, kh * kw))
+        ct_i, pk_i, m_i = np.meshgrid(np.arange(Ct), np.arange(kh * kw), np.arange(M),
+                                      indexing="ij")
+        Wk[ct_i, m_i, codes.astype(np.int64), pk_i] = 1.0
+        Wk = Wk.reshape(Ct, M * K, kh, kw)
+        ref = F.conv2d(torch.from_numpy(Tr), torch.from_numpy(Wk), stride=stride,
+                       padding=pad).numpy()
+        got = o.conv_forward(x, D, codes, kh, kw, stride, pad, lut_bf16=True)
+        if got.shape != ref.shape or not np.array_equal(got, ref):
+            fails.append(f"conv bf16 tables: err {relerr(got, ref)}")
+    return fails
+
+
 ALL_PINS = [pin_conv_vs_dense, pin_fc_vs_dense, pin_integer_exact, pin_exactness,
             pin_linearity, pin_permutation, pin_k1_closed_form, pin_conv_fc_equivalence,
-            pin_lut_one_hot, pin_maxpool, pin_tiny_net]
+            pin_lut_one_hot, pin_maxpool, pin_tiny_net, pin_bf16_rounding, pin_bf16_tables]
 
 
 def run_all(o):

@@ -46,6 +46,13 @@ MUTANTS = {
         "if (iy < 0 || iy >= H) continue;", "if (iy <= 0 || iy >= H) continue;"),
     "pool_window_short": (
         "for (int dy = 0; dy < k; ++dy)", "for (int dy = 0; dy < k - 1; ++dy)"),
+    "bf16_rounding_truncates": (
+        "ldexp(nearbyint(ldexp(f, 8)), e - 8)", "ldexp(trunc(ldexp(f, 8)), e - 8)"),
+    "bf16_keeps_nine_bits": (
+        "ldexp(nearbyint(ldexp(f, 8)), e - 8)", "ldexp(nearbyint(ldexp(f, 9)), e - 9)"),
+    "bf16_flag_ignored": (
+        "lut[(i64)m * K + k] = lut_bf16 ? qo_round_bf16(acc) : acc;",
+        "lut[(i64)m * K + k] = acc;"),
     "lut_dot_product_drops_last_dim": (
         "for (int j = 0; j < Csp; ++j)\n                acc +=",
         "for (int j = 0; j < Csp - 1; ++j)\n                acc +="),
