@@ -278,19 +278,25 @@ def main():
     x = x_host.to(dev)
 
     # model load: codes re-laid out once, outside the timed region
-    layers, shapes = [], w.shapes()
-    for L, P in zip(w.layers, params):
-        if isinstance(L, synth.Conv):
-            codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
-            layers.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
-                                      torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
-                                      L.stride, L.pad, L.relu, packed=True))
-        elif isinstance(L, synth.FC):
-            layers.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
-                                    torch.from_numpy(P["codes"]).to(dev),
-                                    torch.from_numpy(P["bias"]).to(dev), L.relu))
-        else:
-            layers.append(q.PoolLayer(L.k, L.s))
+    shapes = w.shapes()
+
+    def make_layers(lut):
+        layers = []
+        for L, P in zip(w.layers, params):
+            if isinstance(L, synth.Conv):
+                codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
+                layers.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
+                                          torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
+                                          L.stride, L.pad, L.relu, packed=True, lut=lut))
+            elif isinstance(L, synth.FC):
+                layers.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
+                                        torch.from_numpy(P["codes"]).to(dev),
+                                        torch.from_numpy(P["bias"]).to(dev), L.relu, lut=lut))
+            else:
+                layers.append(q.PoolLayer(L.k, L.s))
+        return layers
+
+    layers = make_layers("fp32")
     net = q.Net(layers, tuple(w.in_shape))
     ws = net.alloc_workspace(N, dev)
     out = net._out(N, dev)
@@ -331,58 +337,62 @@ def main():
     value = job_throughput(N, world, a.steps, ms / 1e3)
 
     # ---- per-stage timing: the same layers launched one by one, events between
-    conv_costs, per_layer = [], []
-    hshape = tuple(w.in_shape)
-    bufs = []
-    h = x
-    for L, qL, (sin, sout) in zip(w.layers, layers, shapes):
-        o = torch.empty((N, *sout), dtype=torch.float32, device=dev)
-        bufs.append(o)
-    stage_ms = [0.0] * len(layers)
+    bufs = [torch.empty((N, *sout), dtype=torch.float32, device=dev) for (sin, sout) in shapes]
     lws = torch.empty(ws.numel(), dtype=torch.uint8, device=dev)
-    for it in range(a.steps + 2):
-        flush.zero_()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(layers) + 1)]
-        ev[0].record(stream)
-        h = x
-        for j, (L, qL) in enumerate(zip(w.layers, layers)):
-            o = bufs[j]
-            if isinstance(qL, q.ConvLayer):
-                q.conv_forward(h, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias,
-                               qL.relu, packed=True, Ct=qL.Ct, out=o, workspace=lws)
-            elif isinstance(qL, q.FCLayer):
-                q.fc_forward(h.reshape(N, -1), qL.D, qL.codes, qL.bias, qL.relu, out=o.reshape(N, -1),
-                             workspace=lws)
-            else:
-                q.maxpool(h, qL.k, qL.s, out=o)
-            ev[j + 1].record(stream)
-            h = o
-        torch.cuda.synchronize(dev)
-        if it >= 2:
-            for j in range(len(layers)):
-                stage_ms[j] += ev[j].elapsed_time(ev[j + 1])
-    stage_ms = [s / a.steps for s in stage_ms]
+
+    def stage_times(qlayers, lut):
+        stage_ms = [0.0] * len(qlayers)
+        for it in range(a.steps + 2):
+            flush.zero_()
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(qlayers) + 1)]
+            ev[0].record(stream)
+            h = x
+            for j, qL in enumerate(qlayers):
+                o = bufs[j]
+                if isinstance(qL, q.ConvLayer):
+                    q.conv_forward(h, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias,
+                                   qL.relu, packed=True, Ct=qL.Ct, out=o, workspace=lws, lut=lut)
+                elif isinstance(qL, q.FCLayer):
+                    q.fc_forward(h.reshape(N, -1), qL.D, qL.codes, qL.bias, qL.relu,
+                                 out=o.reshape(N, -1), workspace=lws, lut=lut)
+                else:
+                    q.maxpool(h, qL.k, qL.s, out=o)
+                ev[j + 1].record(stream)
+                h = o
+            torch.cuda.synchronize(dev)
+            if it >= 2:
+                for j in range(len(qlayers)):
+                    stage_ms[j] += ev[j].elapsed_time(ev[j + 1])
+        return [t / a.steps for t in stage_ms]
 
     peaks = load_peaks()
     sm_max = float(peaks.get("sm_max_mhz") or 2070.0)
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
     smem_peak_gbs = nsm * 128 * sm_max * 1e6 / 1e9
-    stages = []
-    dense_macs = 0.0
-    for j, (L, (sin, sout)) in enumerate(zip(w.layers, shapes)):
-        if isinstance(L, synth.Conv):
-            c = cm.conv_cost(L.Cs, L.Ct, sin[1], sin[2], L.kh, L.kw, sout[1], sout[2], L.Csp, L.K)
-        elif isinstance(L, synth.FC):
-            c = cm.fc_cost(L.Cs, L.Ct, L.Csp, L.K)
-        else:
-            stages.append({"layer": j, "kind": "maxpool", "ms": round(stage_ms[j], 4)})
-            continue
-        dense_macs += c.dense_macs
-        alg_bytes = 4.0 * (c.lookups + c.lut_entries) * N
-        ach = alg_bytes / (stage_ms[j] / 1e3) / 1e9
-        stages.append({"layer": j, "kind": L.kind, "ms": round(stage_ms[j], 4),
-                       "lookups": c.lookups * N, "lut_entries": c.lut_entries * N,
-                       "smem_alg_GBs": round(ach, 1), "frac_smem": round(ach / smem_peak_gbs, 4)})
+
+    def stage_report(stage_ms, entry_bytes):
+        """Per-layer ms and shared-memory roofline fraction; algorithmic bytes =
+        entry_bytes x (look-ups + table entries) (Table 1 counts)."""
+        stages, dense = [], 0.0
+        for j, (L, (sin, sout)) in enumerate(zip(w.layers, shapes)):
+            if isinstance(L, synth.Conv):
+                c = cm.conv_cost(L.Cs, L.Ct, sin[1], sin[2], L.kh, L.kw, sout[1], sout[2], L.Csp,
+                                 L.K)
+            elif isinstance(L, synth.FC):
+                c = cm.fc_cost(L.Cs, L.Ct, L.Csp, L.K)
+            else:
+                stages.append({"layer": j, "kind": "maxpool", "ms": round(stage_ms[j], 4)})
+                continue
+            dense += c.dense_macs
+            alg_bytes = entry_bytes * (c.lookups + c.lut_entries) * N
+            ach = alg_bytes / (stage_ms[j] / 1e3) / 1e9
+            stages.append({"layer": j, "kind": L.kind, "ms": round(stage_ms[j], 4),
+                           "lookups": c.lookups * N, "lut_entries": c.lut_entries * N,
+                           "smem_alg_GBs": round(ach, 1),
+                           "frac_smem": round(ach / smem_peak_gbs, 4)})
+        return stages, dense
+
+    stages, dense_macs = stage_report(stage_times(layers, "fp32"), 4.0)
     dom = max((s for s in stages if s["kind"] != "maxpool"), key=lambda s: s["ms"])
     dom_alg = 4.0 * (dom["lookups"] + dom["lut_entries"])
     roofline = {
@@ -414,23 +424,70 @@ def main():
     e2e = {"value": job_throughput(N, world, a.steps, e2e_t), "unit": "images/s",
            "h2d_bytes_per_step": x_host.numel() * 4, "d2h_bytes_per_step": y_host.numel() * 4}
 
-    # ---- batch 1 latency (plain launches)
+    # ---- batch 1 latency: plain launches, and one CUDA graph of the whole stack
     x1 = x[:1].contiguous()
-    ws1 = net.alloc_workspace(1, dev)
-    o1 = net._out(1, dev)
-    for _ in range(5):
-        net.forward(x1, out=o1, workspace=ws1)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    lat = []
-    for _ in range(20):
-        flush.zero_()
-        e0.record(stream)
-        net.forward(x1, out=o1, workspace=ws1)
-        e1.record(stream)
+
+    def batch1(bnet):
+        ws1 = bnet.alloc_workspace(1, dev)
+        o1 = bnet._out(1, dev)
+        for _ in range(5):
+            bnet.forward(x1, out=o1, workspace=ws1)
         torch.cuda.synchronize(dev)
-        lat.append(e0.elapsed_time(e1))
-    b1_ms = float(np.median(lat))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+        def median_ms(fn):
+            lat = []
+            for _ in range(20):
+                flush.zero_()
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+                torch.cuda.synchronize(dev)
+                lat.append(e0.elapsed_time(e1))
+            return float(np.median(lat))
+
+        res = {"latency_ms": round(median_ms(lambda: bnet.forward(x1, out=o1, workspace=ws1)), 4)}
+        res["images_per_s"] = round(1e3 / res["latency_ms"], 1)
+        try:
+            g = torch.cuda.CUDAGraph()
+            side = torch.cuda.Stream(dev)
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                with torch.cuda.graph(g, stream=side):
+                    bnet.forward(x1, out=o1, workspace=ws1)
+            stream.wait_stream(side)
+            g.replay()
+            torch.cuda.synchronize(dev)
+            res["graph_latency_ms"] = round(median_ms(g.replay), 4)
+        except Exception as e:  # capture refused: report it, keep the plain number
+            res["graph_error"] = f"{type(e).__name__}: {e}"[:200]
+        return res
+
+    b1 = batch1(net)
+
+    # ---- bfloat16 tables: the same workload and timing, lut="bf16"
+    bf_layers = make_layers("bf16")
+    bf_net = q.Net(bf_layers, tuple(w.in_shape))
+    bf_ws = bf_net.alloc_workspace(N, dev)
+    for _ in range(max(a.warmup, 3)):
+        bf_net.forward(x, out=out, workspace=bf_ws)
+    torch.cuda.synchronize(dev)
+    bf_ms = 0.0
+    for i in range(a.steps):
+        flush.zero_()
+        starts[i].record(stream)
+        bf_net.forward(x, out=out, workspace=bf_ws)
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    bf_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
+    if world > 1:
+        bf_ms = max_over_ranks(bf_ms, dev)
+    bf_stages, _ = stage_report(stage_times(bf_layers, "bf16"), 2.0)
+    bf16 = {"value": round(job_throughput(N, world, a.steps, bf_ms / 1e3), 1),
+            "unit": "images/s", "ms_per_step": round(bf_ms / a.steps, 4),
+            "note": "table entries rounded to bfloat16, sums in fp32; smem roofline at 2 B "
+                    "per look-up and per table entry; not the headline (fp32) number",
+            "batch1": batch1(bf_net), "stages": bf_stages}
 
     cpu = None
     if pool is not None:
@@ -455,8 +512,8 @@ def main():
                    "l2": "flushed (256 MB write) before every timed step",
                    "codes": "packed once at model load (outside the timed region)"},
         "dense_equiv_gflops": round(2 * dense_macs * value / 1e9, 1),
-        "batch1": {"latency_ms": round(b1_ms, 4), "images_per_s": round(1e3 / b1_ms, 1)},
-        "roofline": roofline, "stages": stages,
+        "batch1": b1,
+        "roofline": roofline, "stages": stages, "bf16_lut": bf16,
         "cpu_baseline": cpu, "e2e": {k: (round(v, 1) if isinstance(v, float) else v)
                                      for k, v in e2e.items()},
         "gpu_launches": int(launches), "clocks": clk,

@@ -62,6 +62,19 @@ typedef enum {
                               shared memory, any stride                      */
 } qcnn_algo;
 
+/*
+ * Precision of the look-up-table entries.  FP32: each entry is the fp32 dot
+ * product of Sec. 3.1 / 3.2.  BF16: each entry is that fp32 value rounded to
+ * bfloat16 (round to nearest, ties to even), which halves the shared-memory
+ * bytes of every look-up; the sums of Eq. 5 / Eq. 7 are still accumulated
+ * in fp32.  The paper's tables are full precision; BF16 is an option of
+ * this library (expected relative error around 1e-3 of the output range).
+ */
+typedef enum {
+    QCNN_LUT_FP32 = 0,
+    QCNN_LUT_BF16 = 1
+} qcnn_lut_type;
+
 typedef enum {
     QCNN_CODES_CANONICAL = 0, /* conv codes [Ct][kh*kw][M]                   */
     QCNN_CODES_PACKED = 1     /* output of qcnn_conv_pack_codes              */
@@ -83,11 +96,13 @@ uint64_t qcnn_launch_count(void);
  * for every input position p = y*W + x (H = W = 1 for an FC input).
  *   x    [N][Cs][H][W]   fp32, device
  *   D    [M][K][Csp]     fp32, device
- *   lut  [N][M][H*W][K]  fp32, device, written
+ *   lut  [N][M][H*W][K]  device, written: fp32 (lut_type QCNN_LUT_FP32) or
+ *                        the bit patterns of bfloat16 values, 2 bytes each
+ *                        (QCNN_LUT_BF16)
  */
 qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W,
-                           const float *D, int Csp, int K, float *lut,
-                           void *stream);
+                           const float *D, int Csp, int K, void *lut,
+                           int lut_type, void *stream);
 
 /*
  * qcnn_fc_forward -- PQ fully-connected layer, Eq. 5:
@@ -97,16 +112,17 @@ qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W,
  *   x      [N][Cs]   fp32       D [M][K][Csp] fp32
  *   codes  [M][Ct]   uint8      bias [Ct] fp32, or NULL for none
  *   y      [N][Ct]   fp32, written
+ *   lut_type: qcnn_lut_type of the table entries
  *   workspace: at least qcnn_fc_workspace_size(...) bytes, 256-byte aligned
  *   (may be NULL when that size is 0).
  */
 qcnn_status qcnn_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K,
-                                   size_t *bytes);
+                                   int lut_type, size_t *bytes);
 qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
                             const float *D, int Csp, int K,
                             const uint8_t *codes, const float *bias, float *y,
-                            int relu, void *workspace, size_t workspace_bytes,
-                            void *stream);
+                            int relu, int lut_type, void *workspace,
+                            size_t workspace_bytes, void *stream);
 
 /*
  * qcnn_fc_forward_noalloc -- the same result as qcnn_fc_forward, for callers
@@ -125,7 +141,8 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
  *   All calls share the array: calls that overlap on the GPU (different
  *   streams or host threads without ordering) race and give wrong results.
  *   Nothing in it needs clearing: each call writes what it reads back.
- * Arguments, layouts and other errors are those of qcnn_fc_forward.
+ * Arguments, layouts and other errors are those of qcnn_fc_forward with
+ * lut_type QCNN_LUT_FP32.
  */
 #define QCNN_FC_NOALLOC_SCRATCH_BYTES (16u << 20)
 qcnn_status qcnn_fc_forward_noalloc(const float *x, int N, int Cs, int Ct,
@@ -155,19 +172,22 @@ qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw,
  *          qcnn_conv_pack_codes (PACKED)
  *   bias   [Ct] or NULL;   y [N][Ct][Ho][Wo] fp32, written
  *   algo:  QCNN_ALGO_FUSED needs stride 1, else QCNN_ERR_UNSUPPORTED.
+ *   lut_type: qcnn_lut_type of the table entries; QCNN_LUT_BF16 is served
+ *          by the fused and chunked algorithms (UNFUSED returns
+ *          QCNN_ERR_UNSUPPORTED).
  *   workspace: at least qcnn_conv_workspace_size(...) bytes, 256-byte aligned.
  */
 qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct,
                                      int kh, int kw, int stride, int pad,
                                      int Csp, int K, int codes_layout,
-                                     int algo, size_t *bytes);
+                                     int algo, int lut_type, size_t *bytes);
 qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W,
                               int Ct, int kh, int kw, int stride, int pad,
                               const float *D, int Csp, int K,
                               const uint8_t *codes, int codes_layout,
                               const float *bias, float *y, int relu, int algo,
-                              void *workspace, size_t workspace_bytes,
-                              void *stream);
+                              int lut_type, void *workspace,
+                              size_t workspace_bytes, void *stream);
 
 /*
  * qcnn_maxpool -- k x k max-pool, stride s, no padding, floor output size
@@ -194,6 +214,7 @@ typedef struct {
     int relu;           /* CONV / FC: 1 = ReLU after the bias                */
     int algo;           /* CONV: qcnn_algo                                   */
     int codes_layout;   /* CONV: qcnn_codes_layout of `codes`                */
+    int lut_type;       /* CONV / FC: qcnn_lut_type of the table entries     */
     const float *D;     /* CONV / FC: [M][K][Csp], device                    */
     const uint8_t *codes; /* CONV: see qcnn_conv_forward; FC: [M][Ct]; device */
     const float *bias;  /* [Ct] or NULL, device                              */

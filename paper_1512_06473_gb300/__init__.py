@@ -9,6 +9,9 @@ library cannot be built or loaded, every call raises.
 Layouts (fp32 unless stated, all CUDA tensors, contiguous):
   FC   : x [N, Cs], D [M, K, Csp], codes [M, Ct] uint8, bias [Ct]  -> [N, Ct]
   conv : x [N, Cs, H, W], D [M, K, Csp], codes [Ct, kh*kw, M] uint8 -> [N, Ct, Ho, Wo]
+
+``lut="bf16"`` rounds every table entry to bfloat16 (nearest, ties to even)
+and still sums in fp32; ``lut="fp32"`` (default) keeps fp32 entries.
 """
 from __future__ import annotations
 
@@ -59,9 +62,11 @@ def launch_count() -> int:
     return int(load().qcnn_launch_count())
 
 
-def lut_build(x: torch.Tensor, D: torch.Tensor, out: Optional[torch.Tensor] = None, stream=None):
+def lut_build(x: torch.Tensor, D: torch.Tensor, out: Optional[torch.Tensor] = None, stream=None,
+              lut: str = "fp32"):
     """Tables lut[n, m, p, k] = <x[n, m*Csp:(m+1)*Csp, p], D[m, k]> (Sec. 3.1 / 3.2).
-    x is [N, Cs] (FC input) or [N, Cs, H, W]; returns [N, M, H*W, K]."""
+    x is [N, Cs] (FC input) or [N, Cs, H, W]; returns [N, M, H*W, K], float32
+    or (lut="bf16") bfloat16."""
     if x.dim() == 2:
         N, Cs = x.shape
         H = W = 1
@@ -71,15 +76,18 @@ def lut_build(x: torch.Tensor, D: torch.Tensor, out: Optional[torch.Tensor] = No
     _need(x, "x", torch.float32, x.dim())
     _need(D, "D", torch.float32, 3)
     M, K, Csp = D.shape
+    lt = _lib.LUT[lut]
+    dt = torch.bfloat16 if lt else torch.float32
     if out is None:
-        out = torch.empty((N, M, H * W, K), dtype=torch.float32, device=x.device)
-    _need(out, "out", torch.float32, 4)
-    _lib.check(load().qcnn_lut_build(_ptr(x), N, Cs, H, W, _ptr(D), Csp, K, _ptr(out),
+        out = torch.empty((N, M, H * W, K), dtype=dt, device=x.device)
+    _need(out, "out", dt, 4)
+    _lib.check(load().qcnn_lut_build(_ptr(x), N, Cs, H, W, _ptr(D), Csp, K, _ptr(out), lt,
                                      _stream(stream)), "qcnn_lut_build")
     return out
 
 
-def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, stream=None):
+def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, stream=None,
+               lut="fp32"):
     """Eq. 5: y[n, ct] = bias[ct] + sum_m LUT_n[m, codes[m, ct]] (then ReLU)."""
     _need(x, "x", torch.float32, 2)
     _need(D, "D", torch.float32, 3)
@@ -90,14 +98,15 @@ def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, str
     if bias is not None:
         _need(bias, "bias", torch.float32, 1)
     lib = load()
+    lt = _lib.LUT[lut]
     nb = ctypes.c_size_t()
-    _lib.check(lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)),
+    _lib.check(lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, lt, ctypes.byref(nb)),
                "qcnn_fc_workspace_size")
     ws, wsb = _workspace(nb.value, x.device, workspace)
     if out is None:
         out = torch.empty((N, Ct), dtype=torch.float32, device=x.device)
     _lib.check(lib.qcnn_fc_forward(_ptr(x), N, Cs, Ct, _ptr(D), Csp, K, _ptr(codes),
-                                   _ptr(bias), _ptr(out), int(bool(relu)), _ptr(ws), wsb,
+                                   _ptr(bias), _ptr(out), int(bool(relu)), lt, _ptr(ws), wsb,
                                    _stream(stream)), "qcnn_fc_forward")
     return out
 
@@ -119,7 +128,7 @@ def conv_pack_codes(codes: torch.Tensor, K: int, kh: int, kw: int, stream=None) 
 
 
 def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, algo="auto",
-                 packed=False, Ct=None, out=None, workspace=None, stream=None):
+                 packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32"):
     """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,
     then ``Ct`` is required) the output of conv_pack_codes."""
     _need(x, "x", torch.float32, 4)
@@ -137,10 +146,11 @@ def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, al
         _need(bias, "bias", torch.float32, 1)
     layout = _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL
     a = _lib.ALGO[algo]
+    lt = _lib.LUT[lut]
     lib = load()
     nb = ctypes.c_size_t()
     _lib.check(lib.qcnn_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, layout,
-                                            a, ctypes.byref(nb)), "qcnn_conv_workspace_size")
+                                            a, lt, ctypes.byref(nb)), "qcnn_conv_workspace_size")
     ws, wsb = _workspace(nb.value, x.device, workspace)
     Ho = (H + 2 * pad - kh) // stride + 1
     Wo = (W + 2 * pad - kw) // stride + 1
@@ -148,7 +158,7 @@ def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, al
         out = torch.empty((N, Ct, Ho, Wo), dtype=torch.float32, device=x.device)
     _lib.check(lib.qcnn_conv_forward(_ptr(x), N, Cs, H, W, Ct, kh, kw, stride, pad, _ptr(D), Csp,
                                      K, _ptr(codes), layout, _ptr(bias), _ptr(out),
-                                     int(bool(relu)), a, _ptr(ws), wsb, _stream(stream)),
+                                     int(bool(relu)), a, lt, _ptr(ws), wsb, _stream(stream)),
                "qcnn_conv_forward")
     return out
 
@@ -178,6 +188,7 @@ class ConvLayer:
     relu: bool = True
     algo: str = "auto"
     packed: bool = False
+    lut: str = "fp32"
 
 
 @dataclass
@@ -186,6 +197,7 @@ class FCLayer:
     codes: torch.Tensor         # [M, Ct]
     bias: Optional[torch.Tensor]
     relu: bool = True
+    lut: str = "fp32"
 
 
 @dataclass
@@ -208,10 +220,12 @@ class Net:
                 d.kind, d.Ct, d.kh, d.kw, d.stride, d.pad = _lib.LAYER_CONV, L.Ct, L.kh, L.kw, L.stride, L.pad
                 d.Csp, d.K, d.relu, d.algo = Csp, K, int(L.relu), _lib.ALGO[L.algo]
                 d.codes_layout = _lib.CODES_PACKED if L.packed else _lib.CODES_CANONICAL
+                d.lut_type = _lib.LUT[L.lut]
                 d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
             elif isinstance(L, FCLayer):
                 M, K, Csp = L.D.shape
                 d.kind, d.Ct, d.Csp, d.K, d.relu = _lib.LAYER_FC, L.codes.shape[1], Csp, K, int(L.relu)
+                d.lut_type = _lib.LUT[L.lut]
                 d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
             elif isinstance(L, PoolLayer):
                 d.kind, d.kh, d.kw, d.stride = _lib.LAYER_MAXPOOL, L.k, L.k, L.s

@@ -14,6 +14,7 @@ c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_vo
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
 ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3}
 CODES_CANONICAL, CODES_PACKED = 0, 1
+LUT = {"fp32": 0, "bf16": 1}
 LAYER_CONV, LAYER_FC, LAYER_MAXPOOL = 0, 1, 2
 
 
@@ -28,7 +29,7 @@ class Layer(ctypes.Structure):
     _fields_ = [("kind", c_int), ("Ct", c_int), ("kh", c_int), ("kw", c_int),
                 ("stride", c_int), ("pad", c_int), ("Csp", c_int), ("K", c_int),
                 ("relu", c_int), ("algo", c_int), ("codes_layout", c_int),
-                ("D", c_void_p), ("codes", c_void_p), ("bias", c_void_p)]
+                ("lut_type", c_int), ("D", c_void_p), ("codes", c_void_p), ("bias", c_void_p)]
 
 
 _SIGS = {
@@ -36,19 +37,20 @@ _SIGS = {
     "qcnn_last_cuda_error": (c_int, []),
     "qcnn_launch_count": (c_uint64, []),
     "qcnn_lut_build": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
-                               c_void_p, c_void_p]),
-    "qcnn_fc_workspace_size": (c_int, [c_int, c_int, c_int, c_int, c_int, ctypes.POINTER(c_size_t)]),
+                               c_void_p, c_int, c_void_p]),
+    "qcnn_fc_workspace_size": (c_int, [c_int, c_int, c_int, c_int, c_int, c_int,
+                                       ctypes.POINTER(c_size_t)]),
     "qcnn_fc_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
-                                c_void_p, c_void_p, c_int, c_void_p, c_size_t, c_void_p]),
+                                c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t, c_void_p]),
     "qcnn_fc_forward_noalloc": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int,
                                         c_void_p, c_void_p, c_void_p, c_int, c_void_p]),
     "qcnn_conv_packed_codes_bytes": (c_size_t, [c_int, c_int, c_int, c_int]),
     "qcnn_conv_pack_codes": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_void_p,
                                      c_void_p]),
-    "qcnn_conv_workspace_size": (c_int, [c_int] * 13 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_conv_workspace_size": (c_int, [c_int] * 14 + [ctypes.POINTER(c_size_t)]),
     "qcnn_conv_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_int,
                                   c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int,
-                                  c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t,
+                                  c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_size_t,
                                   c_void_p]),
     "qcnn_maxpool": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_void_p,
                              c_void_p]),

@@ -13,6 +13,13 @@
 //    bank-conflict free, and the kernel offset (ky, kx) is a plain shift
 //    ky*pitch + kx of the read address.  Lanes that fall on the padding
 //    columns compute values that are discarded.
+//    bfloat16 tables (BF): every 32-bit word holds the entries of two
+//    neighbouring positions, (h, h+1), so one load serves two look-ups.  A
+//    kernel offset can be odd, so the table is kept twice: copy 0 holds the
+//    pairs that start at even h (word h/2), copy 1 those that start at odd h
+//    (word (h-1)/2).  A lane takes two neighbouring positions and reads copy
+//    (offset & 1); the two copies of 2-byte entries fill the space of one
+//    fp32 table.
 //  * conv_unfused (any stride): tables are first written to the workspace
 //    in a stride-phase-split layout lut[nb][m][k][ay][ax][py][px] with
 //    (iy, ix) = (py*s + ay, px*s + ax), so that consecutive output columns
@@ -122,9 +129,11 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // MINB  : CTAs per SM the register budget is sized for
 // PIPE  : two table buffers; sub-space m+1's table is built while m is
 //         gathered, with one barrier per sub-space instead of two
-template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE>
+// BF    : bfloat16 pair tables; a slot is then 64 positions (2 per lane)
+template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
     constexpr int NT = NW * 32;
+    constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     constexpr int CT_CTA = (NW / WP) * CTW;
     constexpr int Q16 = CT_CTA / 16;
     // sub-codewords per lane per build pass (fewer under a 64-register budget)
@@ -225,15 +234,68 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             }
         }
     };
+    // bfloat16 pair tables: a lane walks its warp's positions in order and,
+    // at position h, writes the word (t[h-1], t[h]) into copy (h-1) & 1.  The
+    // walk starts one position early (the left neighbour of the range) and
+    // the last range runs one past HP with a zero entry, so every pair
+    // (q, q+1), 0 <= q < HP, is written exactly once.
+    auto build_bf16 = [&](int b, float *lut) {
+        if (h0 >= HP) return;
+        const float *xb = xs + b * a.xs_floats;
+        const float *db = ds + b * K * CSP4;
+        unsigned *w = reinterpret_cast<unsigned *>(lut);
+        const int RW = KS >> 1;  // words per row of one copy (odd)
+        const int hs = max(h0 - 1, 0), he = h1 == HP ? HP + 1 : h1;
+        for (int q0 = 0; q0 < K; q0 += 32 * QB) {
+            float dk[QB][CSP4];
+#pragma unroll
+            for (int i = 0; i < QB; ++i) {
+                const int k = min(q0 + 32 * i + lane, K - 1);
+#pragma unroll
+                for (int j = 0; j < CSP4; j += 4) {
+                    const float4 v = *reinterpret_cast<const float4 *>(db + k * CSP4 + j);
+                    dk[i][j] = v.x;
+                    dk[i][j + 1] = v.y;
+                    dk[i][j + 2] = v.z;
+                    dk[i][j + 3] = v.w;
+                }
+            }
+            float prev[QB];
+            for (int h = hs; h < he; ++h) {
+                float xv[CSP4];
+#pragma unroll
+                for (int j = 0; j < CSP4; j += 4) {
+                    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (h < HP) v = *reinterpret_cast<const float4 *>(xb + h * CSP4 + j);
+                    xv[j] = v.x;
+                    xv[j + 1] = v.y;
+                    xv[j + 2] = v.z;
+                    xv[j + 3] = v.w;
+                }
+                const int q = h - 1;
+                unsigned *wq = w + (q & 1) * K * RW + (q >> 1);
+#pragma unroll
+                for (int i = 0; i < QB; ++i) {
+                    const int k = q0 + 32 * i + lane;
+                    float v = 0.f;
+#pragma unroll
+                    for (int j = 0; j < CSP4; ++j) v = fmaf(xv[j], dk[i][j], v);
+                    if (h > hs && k < K) wq[k * RW] = pack_bf16x2(prev[i], v);
+                    prev[i] = v;
+                }
+            }
+        }
+    };
 
     // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
-    float acc[CTW][P];
+    float acc[CTW][P * E];
 #pragma unroll
     for (int c = 0; c < CTW; ++c)
 #pragma unroll
-        for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
-    const int lane_off4 = (wp * P * 32 + lane) * 4;  // byte offset of the first position
-    const int KS4 = KS * 4;
+        for (int p = 0; p < P * E; ++p) acc[c][p] = 0.f;
+    // byte offset of the lane's first word (fp32: position; bf16: pair)
+    const int lane_off4 = (wp * P * 32 + lane) * 4;
+    const int KS4 = (BF ? KS >> 1 : KS) * 4;  // bytes between rows k and k+1
     const unsigned kmax4 = (unsigned)(K - 1) * 0x01010101u;  // clamp codes into [0, K)
     auto gather = [&](int b, const float *lut) {
         const unsigned char *lutb = reinterpret_cast<const unsigned char *>(lut);
@@ -245,14 +307,23 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 load_code_words<CTW>(cb + pk * CT_CTA, w);
 #pragma unroll
                 for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
-                const int base4 = lane_off4 + (ky * pitch + kx) * 4;
+                const int off = ky * pitch + kx;
+                const int base4 =
+                    BF ? lane_off4 + (off >> 1) * 4 + (off & 1) * K * KS4 : lane_off4 + off * 4;
 #pragma unroll
                 for (int c = 0; c < CTW; ++c) {
                     const unsigned code = byte_of(w[c >> 2], c & 3);
                     const unsigned char *row = lutb + (int)code * KS4 + base4;
-                    accumulate<P>(acc[c], [&](int p) {
-                        return *reinterpret_cast<const float *>(row + p * 128);
-                    });
+                    if constexpr (BF) {
+#pragma unroll
+                        for (int p = 0; p < P; ++p)
+                            add_bf16x2(acc[c][2 * p], acc[c][2 * p + 1],
+                                       *reinterpret_cast<const unsigned *>(row + p * 128));
+                    } else {
+                        accumulate<P>(acc[c], [&](int p) {
+                            return *reinterpret_cast<const float *>(row + p * 128);
+                        });
+                    }
                 }
             }
         }
@@ -273,7 +344,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 stage_codes(m + 1, b ^ 1);
                 cp_async_commit();
             }
-            build(b, lut0);
+            if constexpr (BF) build_bf16(b, lut0);
+            else build(b, lut0);
             __syncthreads();
             gather(b, lut0);
         }
@@ -285,7 +357,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         cp_async_commit();
         cp_async_wait<0>();
         __syncthreads();
-        build(0, lut0);
+        if constexpr (BF) build_bf16(0, lut0);
+        else build(0, lut0);
         __syncthreads();
         // Iteration m (b = (m - mb) & 1): table m ready in buffer b, codes m in
         // code buffer b, inputs of m+1 in staging buffer b^1.
@@ -296,11 +369,16 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             cp_async_commit();
             // even warps build first, odd warps gather first: the latency-bound
             // table build of one half overlaps the other half's gather
+            auto build_next = [&]() {
+                if (m + 1 >= me) return;
+                if constexpr (BF) build_bf16(b ^ 1, b ? lut0 : lut1);
+                else build(b ^ 1, b ? lut0 : lut1);
+            };
             if (warp & 1) {
                 gather(b, b ? lut1 : lut0);
-                if (m + 1 < me) build(b ^ 1, b ? lut0 : lut1);
+                build_next();
             } else {
-                if (m + 1 < me) build(b ^ 1, b ? lut0 : lut1);
+                build_next();
                 gather(b, b ? lut1 : lut0);
             }
             cp_async_wait<0>();
@@ -315,8 +393,9 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         if (ct >= a.Ct) continue;
         const float bv = a.bias ? a.bias[ct] : 0.f;
 #pragma unroll
-        for (int p = 0; p < P; ++p) {
-            const int l = (wp * P + p) * 32 + lane;
+        for (int p = 0; p < P * E; ++p) {
+            const int l = BF ? (wp * P + (p >> 1)) * 64 + 2 * lane + (p & 1)
+                             : (wp * P + p) * 32 + lane;
             const int r = l / pitch, col = l - r * pitch;
             const int oy = oy0 + r;
             if (r < a.TH && col < a.Wo && oy < a.Ho) {
@@ -353,13 +432,17 @@ __global__ void conv_split_reduce_kernel(const float *__restrict__ partial, int 
 // (GB300, AlexNet conv2-5 and VGG-16 conv3-5 shapes, all lanes counted);
 // build: share of the table-build time left exposed (1 = not overlapped).
 struct FusedVariant {
-    int P, CTW, WP, CSP4, NW, MINB, PIPE;
+    int P, CTW, WP, CSP4, NW, MINB, PIPE, BF;
     double eff, build;
     void (*fn)(ConvFusedArgs);
 };
 
 #define QCNN_FUSED(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
-    {P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD, conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE>}
+    {P, CTW, WP, C4, NW, MB, PIPE, 0, EFF, BLD,             \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, false>}
+#define QCNN_FUSED_BF(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
+    {P, CTW, WP, C4, NW, MB, PIPE, 1, EFF, BLD,                \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, true>}
 #define QCNN_FUSED_SET(C4)                                                                       \
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
@@ -372,8 +455,22 @@ struct FusedVariant {
     QCNN_FUSED(4, 16, 1, C4, 16, 1, true, 0.85, 0.3),                                             \
     QCNN_FUSED(2, 16, 2, C4, 16, 1, true, 0.7, 0.3),                                             \
     QCNN_FUSED(4, 8, 1, C4, 16, 1, true, 0.8, 0.3)
-static const FusedVariant kFused[] = {QCNN_FUSED_SET(4), QCNN_FUSED_SET(8)};
+// bfloat16 tables: slots of 64 positions, so half the slots of the fp32
+// tiles cover the same band.  Measured (same shapes): the pair-table build
+// costs about 1.3x the fp32 build, the 32-warp and pipelined tiles never win.
+#define QCNN_FUSED_BF_SET(C4)                                                      \
+    QCNN_FUSED_BF(2, 8, 2, C4, 8, 2, false, 0.45, 1.3),                            \
+    QCNN_FUSED_BF(4, 8, 1, C4, 16, 1, false, 1.0, 1.3),                            \
+    QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, false, 0.97, 1.3),                          \
+    QCNN_FUSED_BF(2, 8, 1, C4, 32, 1, false, 0.75, 1.3),                           \
+    QCNN_FUSED_BF(4, 4, 1, C4, 32, 1, false, 0.7, 1.3),                            \
+    QCNN_FUSED_BF(4, 8, 1, C4, 16, 1, true, 0.6, 0.4),                             \
+    QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, true, 0.6, 0.4)
+static const FusedVariant kFused[] = {QCNN_FUSED_SET(4), QCNN_FUSED_SET(8),
+                                      QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8)};
+#undef QCNN_FUSED_BF_SET
 #undef QCNN_FUSED_SET
+#undef QCNN_FUSED_BF
 #undef QCNN_FUSED
 constexpr int kNumFused = sizeof(kFused) / sizeof(kFused[0]);
 
@@ -415,14 +512,25 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         if (force >= 0 && v != force) continue;
 #endif
         const FusedVariant &fv = kFused[v];
-        if (fv.CSP4 != csp4) continue;
+        if (fv.CSP4 != csp4 || fv.BF != s.bf16) continue;
         const int slots = fv.WP * fv.P;
-        int TH = std::min(slots * 32 / pitch, s.Ho);
+        const int E = fv.BF ? 2 : 1;  // positions per lane and slot
+        int TH = std::min(slots * 32 * E / pitch, s.Ho);
         if (TH < 1) continue;
         const int row_tiles = cdiv(s.Ho, TH);
         TH = cdiv(s.Ho, row_tiles);  // balance the bands
         const int HP = (TH + s.kh - 1) * pitch;
-        const int KS = ks_for(slots * 32 + (s.kh - 1) * pitch + (s.kw - 1));
+        const int reach = (s.kh - 1) * pitch + (s.kw - 1);  // largest kernel offset
+        // fp32: KS floats per row, >= every position read; bf16: two copies
+        // of RW words per row, RW > every pair word read or written
+        int KS;
+        if (fv.BF) {
+            const int RW = ks_for(slots * 32 + (reach >> 1) + 1);
+            if ((HP - 1) / 2 >= RW) continue;
+            KS = 2 * RW;
+        } else {
+            KS = ks_for(slots * 32 + reach);
+        }
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
         const size_t smem =

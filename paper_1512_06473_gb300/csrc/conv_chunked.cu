@@ -20,6 +20,12 @@
 // (l = r*PW + c, columns c >= Wo are discarded) and CTW channels; its input
 // sub-vectors (QPT positions x CSPT channels) stay in registers across the
 // chunks of a sub-space.
+// bfloat16 tables (BF): a row holds 2-byte entries twice, copy 0 as built
+// and copy 1 shifted left by one entry, both SKW words long.  A lane takes
+// two neighbouring output columns (2 P positions) and reads one 32-bit word
+// per look-up pair: for an entry whose row offset e is even the word
+// (e/2 + lane) of copy 0, for an odd e the same word of copy 1.  The prep
+// kernel folds the copy choice into the entry's byte offset.
 #include "qcnn_internal.cuh"
 
 #include <algorithm>
@@ -31,7 +37,15 @@ constexpr int kChunkThreads = 512;
 
 struct ChunkGeom {
     int s, pad, kh, kw, TH, PR, PW, PS, SK, NQ, dymin, dymax, dxmin, dxmax, KC, NCH;
+    int bf;   // bfloat16 tables
+    int SKW;  // bf16: words of one row copy (entries SK <= 2 SKW)
 };
+
+// Byte offset of entry e of row kl inside a chunk table.
+__host__ __device__ inline unsigned chunk_entry_bytes(const ChunkGeom &g, int kl, int e) {
+    if (!g.bf) return 4u * (unsigned)(kl * g.SK + e);
+    return 4u * (unsigned)(((e & 1) * g.KC + kl) * g.SKW + (e >> 1));
+}
 
 __host__ __device__ inline int floor_div(int a, int b) {
     return (a >= 0) ? a / b : -((-a + b - 1) / b);
@@ -90,7 +104,7 @@ __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed,
         const int pos = wcount[warp * g.NCH + b] + rank;
         const int ky = pk / g.kw, kx = pk % g.kw;
         entries[(size_t)i * kk + pos] =
-            (uint32_t)(4 * ((code - b * g.KC) * g.SK + chunk_phase_off(g, ky, kx)));
+            chunk_entry_bytes(g, code - b * g.KC, chunk_phase_off(g, ky, kx));
     }
     for (int c = threadIdx.x; c <= g.NCH; c += blockDim.x)
         starts[(size_t)i * (g.NCH + 1) + c] = bstart[c];
@@ -108,23 +122,24 @@ struct ChunkArgs {
     ChunkGeom g;
 };
 
-template <int P, int CTW, int QPT, int CSPT>
+template <int P, int CTW, int QPT, int CSPT, bool BF>
 __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const ChunkArgs a) {
+    constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     extern __shared__ __align__(16) float csm[];
     const ChunkGeom &g = a.g;
-    float *lut = csm;                             // [KC][SK]
-    float *ds = csm + (size_t)g.KC * g.SK;        // [K][CSPT]
+    float *lut = csm;  // fp32 [KC][SK]; bf16 [2][KC][SKW] words
+    float *ds = csm + (BF ? (size_t)2 * g.KC * g.SKW : (size_t)g.KC * g.SK);  // [K][CSPT]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int oy0 = blockIdx.x * g.TH;
     const int ct0 = blockIdx.y * a.ct_cta;
     const int n = blockIdx.z;
     const int ctw0 = ct0 + warp * CTW;
 
-    float acc[CTW][P];
+    float acc[CTW][P * E];
 #pragma unroll
     for (int c = 0; c < CTW; ++c)
 #pragma unroll
-        for (int p = 0; p < P; ++p) acc[c][p] = 0.f;
+        for (int p = 0; p < P * E; ++p) acc[c][p] = 0.f;
 
     float xr[QPT][CSPT];  // input sub-vectors of positions tid + qi * 512
 
@@ -132,6 +147,41 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
     // writes its QPT positions (SK >= QPT * 512, positions past NQ hold 0)
     auto build = [&](int ch, float *L) {
         const int k0 = ch * g.KC, kc = min(g.KC, a.K - k0);
+        if constexpr (BF) {
+            // entry q of row kl -> copy 0 at q, copy 1 at q - 1 (2-byte slots)
+            unsigned short *h0 = reinterpret_cast<unsigned short *>(L);
+            unsigned short *h1 = h0 + (size_t)2 * g.KC * g.SKW;
+            for (int kl = 0; kl < kc; ++kl) {
+                float dk[CSPT];
+#pragma unroll
+                for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
+                const int rb = 2 * kl * g.SKW + tid;
+#pragma unroll
+                for (int qi = 0; qi + 1 < QPT; qi += 2) {
+                    float2 v = make_float2(0.f, 0.f);
+#pragma unroll
+                    for (int j = 0; j < CSPT; ++j)
+                        v = __ffma2_rn(make_float2(xr[qi][j], xr[qi + 1][j]),
+                                       make_float2(dk[j], dk[j]), v);
+                    const unsigned w = pack_bf16x2(v.x, v.y);
+                    const int q0 = rb + qi * kChunkThreads, q1 = q0 + kChunkThreads;
+                    h0[q0] = (unsigned short)(w & 0xffffu);
+                    h0[q1] = (unsigned short)(w >> 16);
+                    if (qi > 0 || tid > 0) h1[q0 - 1] = (unsigned short)(w & 0xffffu);
+                    h1[q1 - 1] = (unsigned short)(w >> 16);
+                }
+                if constexpr (QPT % 2 == 1) {
+                    float v = 0.f;
+#pragma unroll
+                    for (int j = 0; j < CSPT; ++j) v = fmaf(xr[QPT - 1][j], dk[j], v);
+                    const unsigned short hv = (unsigned short)(pack_bf16x2(v, 0.f) & 0xffffu);
+                    const int q = rb + (QPT - 1) * kChunkThreads;
+                    h0[q] = hv;
+                    if (QPT > 1 || tid > 0) h1[q - 1] = hv;
+                }
+            }
+            return;
+        }
         for (int kl = 0; kl < kc; ++kl) {
             float dk[CSPT];
 #pragma unroll
@@ -166,23 +216,25 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
                 const int e0 = __ldg(a.starts + row * (g.NCH + 1) + ch);
                 const int e1 = __ldg(a.starts + row * (g.NCH + 1) + ch + 1);
                 const uint32_t *ep = a.entries + row * a.kk;
+                auto look = [&](const unsigned char *b) {
+                    if constexpr (BF) {
+#pragma unroll
+                        for (int p = 0; p < P; ++p)
+                            add_bf16x2(acc[c][2 * p], acc[c][2 * p + 1],
+                                       *reinterpret_cast<const unsigned *>(b + p * 128));
+                    } else {
+                        accumulate<P>(acc[c], [&](int p) {
+                            return *reinterpret_cast<const float *>(b + p * 128);
+                        });
+                    }
+                };
                 int e = e0;
                 for (; e + 1 < e1; e += 2) {
                     const unsigned o0 = __ldg(ep + e), o1 = __ldg(ep + e + 1);
-                    const unsigned char *b0 = lb + o0, *b1 = lb + o1;
-                    accumulate<P>(acc[c], [&](int p) {
-                        return *reinterpret_cast<const float *>(b0 + p * 128);
-                    });
-                    accumulate<P>(acc[c], [&](int p) {
-                        return *reinterpret_cast<const float *>(b1 + p * 128);
-                    });
+                    look(lb + o0);
+                    look(lb + o1);
                 }
-                if (e < e1) {
-                    const unsigned char *b0 = lb + __ldg(ep + e);
-                    accumulate<P>(acc[c], [&](int p) {
-                        return *reinterpret_cast<const float *>(b0 + p * 128);
-                    });
-                }
+                if (e < e1) look(lb + __ldg(ep + e));
             }
         }
     };
@@ -226,8 +278,8 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
         if (ct >= a.Ct) continue;
         const float bv = a.bias ? a.bias[ct] : 0.f;
 #pragma unroll
-        for (int p = 0; p < P; ++p) {
-            const int l = p * 32 + lane;
+        for (int p = 0; p < P * E; ++p) {
+            const int l = BF ? (p >> 1) * 64 + 2 * lane + (p & 1) : p * 32 + lane;
             const int r = l / g.PW, col = l - r * g.PW;
             const int oy = oy0 + r;
             if (r < g.TH && col < a.Wo && oy < a.Ho) {
@@ -240,21 +292,29 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
 }
 
 struct ChunkVariant {
-    int P, CTW, QPT, CSPT;
+    int P, CTW, QPT, CSPT, BF;
     void (*fn)(ChunkArgs);
 };
-#define QCNN_CHUNK(P, CTW, QPT, C) {P, CTW, QPT, C, conv_chunked_kernel<P, CTW, QPT, C>}
+#define QCNN_CHUNK(P, CTW, QPT, C) {P, CTW, QPT, C, 0, conv_chunked_kernel<P, CTW, QPT, C, false>}
+#define QCNN_CHUNK_BF(P, CTW, QPT, C) {P, CTW, QPT, C, 1, conv_chunked_kernel<P, CTW, QPT, C, true>}
 static const ChunkVariant kChunk[] = {
     QCNN_CHUNK(8, 6, 11, 3),  // AlexNet conv1: 4 rows of 57, 96 channels per CTA
     QCNN_CHUNK(8, 1, 11, 3),  // same band, 16 channels per CTA: small batches
     QCNN_CHUNK(8, 8, 6, 4),
     QCNN_CHUNK(4, 8, 4, 8),
+    // bfloat16 tables: slots of 64 positions
+    QCNN_CHUNK_BF(4, 6, 11, 3),
+    QCNN_CHUNK_BF(4, 1, 11, 3),
+    QCNN_CHUNK_BF(4, 8, 6, 4),
+    QCNN_CHUNK_BF(2, 8, 4, 8),
 };
+#undef QCNN_CHUNK_BF
 #undef QCNN_CHUNK
 constexpr int kNumChunk = sizeof(kChunk) / sizeof(kChunk[0]);
 
-static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P, int QPT) {
+static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P, int QPT, int bf) {
     ChunkGeom g;
+    g.bf = bf;
     g.s = s.stride;
     g.pad = s.pad;
     g.kh = s.kh;
@@ -268,11 +328,18 @@ static ChunkGeom chunk_geom(const ConvShape &s, int TH, int KC, int P, int QPT) 
     g.PW = s.Wo + g.dxmax - g.dxmin;
     g.PS = g.PR * g.PW;
     g.NQ = s.stride * s.stride * g.PS;
+    // entries of a row: the largest entry offset plus the lanes' reach
     int sk = (s.stride * s.stride - 1) * g.PS + (g.dymax - g.dymin) * g.PW + (g.dxmax - g.dxmin) +
-             P * 32;
+             P * 32 * (bf ? 2 : 1) + (bf ? 1 : 0);
     sk = std::max(sk, QPT * kChunkThreads);  // every thread's positions fit a row
-    while (sk % 32 != 1) ++sk;
-    g.SK = sk;
+    if (bf) {
+        g.SKW = (sk + 1) / 2;
+        g.SK = 2 * g.SKW;
+    } else {
+        while (sk % 32 != 1) ++sk;
+        g.SK = sk;
+        g.SKW = 0;
+    }
     g.KC = KC;
     g.NCH = cdiv(s.K, KC);
     return g;
@@ -297,18 +364,20 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
         if (force >= 0 && v != force) continue;
 #endif
         const ChunkVariant &cv = kChunk[v];
-        if (s.Csp > cv.CSPT || s.kh * s.kw > kMaxPrepKK) continue;
+        if (cv.BF != s.bf16 || s.Csp > cv.CSPT || s.kh * s.kw > kMaxPrepKK) continue;
         const int ct_cta = 16 * cv.CTW;
+        const int E = cv.BF ? 2 : 1;
         // largest band that the variant's lanes and registers cover
         for (int TH = std::min(s.Ho, 64); TH >= 1; --TH) {
-            const ChunkGeom g0 = chunk_geom(s, TH, 1, cv.P, cv.QPT);
-            if (TH * g0.PW > cv.P * 32) continue;
+            const ChunkGeom g0 = chunk_geom(s, TH, 1, cv.P, cv.QPT, cv.BF);
+            if (TH * g0.PW > cv.P * 32 * E) continue;
             if (g0.NQ > cv.QPT * kChunkThreads) continue;
             const int row_tiles = cdiv(s.Ho, TH);
             const int th = cdiv(s.Ho, row_tiles);  // balance the bands
             for (int KC : {16, 8, 4, 2, 1}) {
                 if (KC > s.K) continue;
-                const ChunkGeom g = chunk_geom(s, th, KC, cv.P, cv.QPT);
+                const ChunkGeom g = chunk_geom(s, th, KC, cv.P, cv.QPT, cv.BF);
+                // fp32: KC rows of SK floats; bf16: two copies of KC x SKW words
                 const size_t smem = ((size_t)KC * g.SK + (size_t)s.K * cv.CSPT) * sizeof(float);
                 if (smem > (size_t)smem_optin) continue;
                 const int ct_tiles = cdiv(s.Ct, ct_cta);
@@ -317,7 +386,7 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
                 // per CTA and sub-space: gather wavefronts + table stores + a
                 // barrier cost per chunk
                 const double gather = (double)cv.P * ct_cta * s.kh * s.kw;
-                const double build = (double)g.NQ * s.K / 32.0;
+                const double build = (double)g.NQ * s.K / 32.0 * (cv.BF ? 2.0 : 1.0);
                 const double sync = (double)g.NCH * 1200.0;
                 const double score = waves * (gather + build + sync) * s.M;
                 if (!best.ok || score < best.score) {
@@ -338,7 +407,7 @@ ConvChunkPlan plan_conv_chunked(const ConvShape &s) {
     }
     if (best.ok) {
         const ChunkVariant &cv = kChunk[best.variant];
-        const ChunkGeom g = chunk_geom(s, best.g_TH, best.KC, cv.P, cv.QPT);
+        const ChunkGeom g = chunk_geom(s, best.g_TH, best.KC, cv.P, cv.QPT, cv.BF);
         best.NCH = g.NCH;
         best.entries_bytes = align_up((size_t)s.M * s.Ct * s.kh * s.kw * 4, kWsAlign);
         best.starts_bytes = align_up((size_t)s.M * s.Ct * (g.NCH + 1) * 4, kWsAlign);
@@ -351,7 +420,7 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
                                 const float *bias, float *y, int relu, void *ws,
                                 cudaStream_t st) {
     const ChunkVariant &cv = kChunk[p.variant];
-    const ChunkGeom g = chunk_geom(s, p.g_TH, p.KC, cv.P, cv.QPT);
+    const ChunkGeom g = chunk_geom(s, p.g_TH, p.KC, cv.P, cv.QPT, cv.BF);
     uint32_t *entries = static_cast<uint32_t *>(ws);
     int *starts = reinterpret_cast<int *>(static_cast<uint8_t *>(ws) + p.entries_bytes);
     const int kk = s.kh * s.kw;

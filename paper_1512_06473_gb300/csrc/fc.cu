@@ -12,6 +12,10 @@
 // copied to shared memory with cp.async one chunk ahead (double buffered), so
 // their device-memory latency overlaps the previous chunk's gather; each
 // code then serves NW images.
+// bfloat16 tables (BF): a 32-bit table word holds the entries of two images
+// (2i, 2i+1) for the same (mm, k) -- both use the same code -- so one load
+// serves two look-ups; the word pitch of a row is odd as above.  Tiles of a
+// single image per lane keep 2-byte entries (pitch NT | 1 halves).
 // When the sub-space range is split over several CTAs (to fill the GPU),
 // the partial sums go to the workspace and a second kernel adds them in a
 // fixed order (deterministic), then applies bias and ReLU.
@@ -32,7 +36,8 @@ struct FcArgs {
     float *__restrict__ partial;  // [splits][N][Ct] when splits > 1
     int N, Cs, Ct, Csp, K, M;
     int NT, CT_CTA, MCH, n_chunks, chunks_per_split, splits, relu;
-    int NTP;     // odd pitch of a table row (>= NT)
+    int NTP;     // odd pitch of a table row (fp32: floats >= NT; bf16 pairs:
+                 // words >= NT/2; bf16 singles: halves >= NT)
     int NTX;     // odd pitch of a staged x row (>= NT)
     int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
     int cvec_log2;
@@ -46,27 +51,42 @@ constexpr int kMchMax = 16;   // sub-spaces per chunk, at most
 struct FcSmem {
     size_t lut, xs, ds, cs, total;
 };
-__host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int NTP, int NTX, int Csp,
-                                                 int CT_CTA) {
+// row_bytes: bytes of one table row (NTP entries or words)
+__host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int row_bytes, int NTX,
+                                                 int Csp, int CT_CTA) {
     FcSmem s;
     s.lut = 0;
-    s.xs = ((size_t)MCH * K * NTP * 4 + 15) / 16 * 16;
+    s.xs = ((size_t)MCH * K * row_bytes + 15) / 16 * 16;
     s.ds = s.xs + ((size_t)2 * MCH * Csp * NTX * 4 + 15) / 16 * 16;
     s.cs = s.ds + ((size_t)2 * MCH * K * Csp * 4 + 15) / 16 * 16;
     s.total = s.cs + (size_t)2 * MCH * CT_CTA;
     return s;
 }
 
+// bytes of one table row
+__host__ __device__ inline int fc_row_bytes(int NT, int NTP, bool bf16) {
+    return bf16 && NT % 2 != 0 ? (NTP * 2 + 3) / 4 * 4 : NTP * 4;
+}
+
+// a += the bfloat16 value h, widened to fp32 (exact), one fp32 rounding
+__device__ __forceinline__ void add_bf16(float &a, unsigned short h) {
+    asm("add.rn.f32.bf16 %0, %1, %0;" : "+f"(a) : "h"(h));
+}
+
 // NW : images per lane;  WN : warps along images (8 / WN along outputs)
 // MINB : CTAs per SM the register budget is sized for
-template <int NW, int WN, int MINB>
+// BF : bfloat16 tables
+template <int NW, int WN, int MINB, bool BF>
 __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs a) {
     constexpr int CT_CTA = (8 / WN) * 32 * kCPL;
     constexpr int kCtCtaLog2 = CT_CTA == 1024 ? 10 : (CT_CTA == 512 ? 9 : 8);
     static_assert((1 << kCtCtaLog2) == CT_CTA, "output tile must be 256, 512 or 1024");
     constexpr int NT = NW * WN;  // images per CTA (== a.NT)
+    constexpr bool PAIRS = BF && NW % 2 == 0;  // bf16 words of two images
+    static_assert(!BF || NW % 2 == 0 || NW == 1, "bf16 tiles: even NW or NW == 1");
     extern __shared__ __align__(16) unsigned char smem[];
-    const FcSmem L = fc_smem_layout(a.MCH, a.K, a.NTP, a.NTX, a.Csp, CT_CTA);
+    const FcSmem L = fc_smem_layout(a.MCH, a.K, fc_row_bytes(NT, a.NTP, BF), a.NTX, a.Csp,
+                                    CT_CTA);
     float *lut = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
@@ -151,15 +171,38 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
             const float *xb = xs + (size_t)b * CCH * a.NTX;
             const float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
             for (int mm = 0; mm < mch; ++mm) {
-                for (int e = tid; e < a.K * NT; e += kFcThreads) {
-                    const int nn = e % NT, k = e / NT;
-                    const float *xp = xb + mm * a.Csp * a.NTX + nn;
-                    const float *dp = db + (mm * a.K + k) * a.Csp;
-                    float v = 0.f;
+                if constexpr (PAIRS) {
+                    constexpr int NP = NT / 2;  // image pairs
+                    unsigned *lw = reinterpret_cast<unsigned *>(lut);
+                    for (int e = tid; e < a.K * NP; e += kFcThreads) {
+                        const int np = e % NP, k = e / NP;
+                        const float *xp = xb + mm * a.Csp * a.NTX + 2 * np;
+                        const float *dp = db + (mm * a.K + k) * a.Csp;
+                        float v0 = 0.f, v1 = 0.f;
 #pragma unroll
-                    for (int j = 0; j < kMaxCsp; ++j)
-                        if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
-                    lut[(mm * a.K + k) * a.NTP + nn] = v;
+                        for (int j = 0; j < kMaxCsp; ++j) {
+                            if (j < a.Csp) {
+                                v0 = fmaf(xp[j * a.NTX], dp[j], v0);
+                                v1 = fmaf(xp[j * a.NTX + 1], dp[j], v1);
+                            }
+                        }
+                        lw[(mm * a.K + k) * a.NTP + np] = pack_bf16x2(v0, v1);
+                    }
+                } else {
+                    for (int e = tid; e < a.K * NT; e += kFcThreads) {
+                        const int nn = e % NT, k = e / NT;
+                        const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                        const float *dp = db + (mm * a.K + k) * a.Csp;
+                        float v = 0.f;
+#pragma unroll
+                        for (int j = 0; j < kMaxCsp; ++j)
+                            if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
+                        if constexpr (BF)
+                            reinterpret_cast<unsigned short *>(lut)[(mm * a.K + k) * a.NTP + nn] =
+                                (unsigned short)(pack_bf16x2(v, 0.f) & 0xffffu);
+                        else
+                            lut[(mm * a.K + k) * a.NTP + nn] = v;
+                    }
                 }
             }
         }
@@ -175,8 +218,21 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
 #pragma unroll
                 for (int q = 0; q < kCPL; ++q) {
                     const int code = (int)byte_of(w, q);
-                    const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
-                    accumulate<NW>(acc[q], [&](int i) { return row[i]; });
+                    if constexpr (PAIRS) {
+                        const unsigned *row = reinterpret_cast<const unsigned *>(lut) +
+                                              (mm * a.K + code) * a.NTP + nbase / 2;
+#pragma unroll
+                        for (int i = 0; i < NW / 2; ++i)
+                            add_bf16x2(acc[q][2 * i], acc[q][2 * i + 1], row[i]);
+                    } else if constexpr (BF) {
+                        const unsigned short *row = reinterpret_cast<const unsigned short *>(lut) +
+                                                    (mm * a.K + code) * a.NTP + nbase;
+#pragma unroll
+                        for (int i = 0; i < NW; ++i) add_bf16(acc[q][i], row[i]);
+                    } else {
+                        const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
+                        accumulate<NW>(acc[q], [&](int i) { return row[i]; });
+                    }
                 }
             }
         }
@@ -219,16 +275,23 @@ __global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, 
 // eff: measured gather throughput relative to the best variant (GB300,
 // AlexNet fc6-fc8 at batch 128).
 struct FcVariant {
-    int NW, WN, MINB;
+    int NW, WN, MINB, BF;
     double eff;
     void (*fn)(FcArgs);
 };
-#define QCNN_FC(NW, WN, MB, EFF) {NW, WN, MB, EFF, fc_fused_kernel<NW, WN, MB>}
-static const FcVariant kFcVariants[] = {QCNN_FC(16, 2, 2, 0.8), QCNN_FC(8, 2, 3, 0.84),
-                                        QCNN_FC(8, 4, 3, 0.6), QCNN_FC(4, 1, 3, 1.0),
-                                        QCNN_FC(1, 1, 3, 0.5)};
+#define QCNN_FC(NW, WN, MB, EFF) {NW, WN, MB, 0, EFF, fc_fused_kernel<NW, WN, MB, false>}
+#define QCNN_FC_BF(NW, WN, MB, EFF) {NW, WN, MB, 1, EFF, fc_fused_kernel<NW, WN, MB, true>}
+static const FcVariant kFcVariants[] = {
+    QCNN_FC(16, 2, 2, 0.8),   QCNN_FC(8, 2, 3, 0.84),   QCNN_FC(8, 4, 3, 0.6),
+    QCNN_FC(4, 1, 3, 1.0),    QCNN_FC(1, 1, 3, 0.5),    QCNN_FC_BF(16, 2, 2, 0.8),
+    QCNN_FC_BF(8, 2, 3, 0.84), QCNN_FC_BF(8, 4, 3, 0.6), QCNN_FC_BF(4, 1, 3, 1.0),
+    QCNN_FC_BF(1, 1, 3, 0.5)};
+#undef QCNN_FC_BF
 #undef QCNN_FC
 constexpr int kNumFc = sizeof(kFcVariants) / sizeof(kFcVariants[0]);
+
+// odd table-row pitch in the unit the kernel indexes (see FcArgs::NTP)
+static int fc_ntp(int NT, int bf16) { return (bf16 && NT % 2 == 0 ? NT / 2 : NT) | 1; }
 
 FcPlan plan_fc(const FcShape &s) {
     FcPlan best{};
@@ -244,15 +307,18 @@ FcPlan plan_fc(const FcShape &s) {
         if (force >= 0 && v != force) continue;
 #endif
         const FcVariant &fv = kFcVariants[v];
+        if (fv.BF != s.bf16) continue;
         const int NT = fv.NW * fv.WN;
         const int CT_CTA = (8 / fv.WN) * 32 * kCPL;
-        const int NTP = NT | 1, NTX = NT | 1;
+        const int NTP = fc_ntp(NT, fv.BF), NTX = NT | 1;
+        const int row_bytes = fc_row_bytes(NT, NTP, fv.BF);
         // largest chunk that lets MINB CTAs share an SM
         int MCH = std::min(kMchMax, std::max(1, 512 / s.K));
         while (MCH > 1 &&
-               (fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp, CT_CTA).total + 1024) * fv.MINB > sm_bytes)
+               (fc_smem_layout(MCH, s.K, row_bytes, NTX, s.Csp, CT_CTA).total + 1024) *
+                       fv.MINB > sm_bytes)
             --MCH;
-        const size_t smem = fc_smem_layout(MCH, s.K, NTP, NTX, s.Csp, CT_CTA).total;
+        const size_t smem = fc_smem_layout(MCH, s.K, row_bytes, NTX, s.Csp, CT_CTA).total;
         if (smem > 200 * 1024) continue;
         const int cps_sm = std::max(1, std::min(fv.MINB, (int)(sm_bytes / (smem + 1024))));
         const int n_chunks = cdiv(s.M, MCH);
@@ -266,7 +332,8 @@ FcPlan plan_fc(const FcShape &s) {
         const double waves = std::ceil(ctas / ((double)cps_sm * sms));
         // one CTA: shared-memory wavefronts (gather + build) per chunk; a wave
         // of cps_sm co-resident CTAs shares one SM
-        const double per_chunk = (double)MCH * NT * CT_CTA / 32.0 + (double)MCH * s.K * NT / 32.0 * 2;
+        const double per_chunk = (double)MCH * NT * CT_CTA / (fv.BF && fv.NW % 2 == 0 ? 64.0 : 32.0) +
+                                 (double)MCH * s.K * NT / 32.0 * 2;
         const double t_smem = waves * cpsplit * per_chunk * cps_sm / 1.2e9 / fv.eff;
         const double bytes = (double)s.M * s.Ct * n_tiles + 4.0 * s.N * s.Cs * ct_tiles +
                              (splits > 1 ? 8.0 * splits * s.N * s.Ct : 0.0);
@@ -313,7 +380,7 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.chunks_per_split = p.chunks_per_split;
     a.splits = p.splits;
     a.relu = relu;
-    a.NTP = p.NT | 1;
+    a.NTP = fc_ntp(p.NT, fv.BF);
     a.NTX = p.NT | 1;
     const uintptr_t base = reinterpret_cast<uintptr_t>(codes);
     a.cvec = (s.Ct % 16 == 0 && base % 16 == 0) ? 16

@@ -55,7 +55,7 @@ extern "C" qcnn_status qcnn_fc_forward_noalloc(const float *x, int N, int Cs, in
                                                const uint8_t *codes, const float *bias,
                                                float *y, int relu, void *stream) {
     size_t need = 0;
-    qcnn_status rc = qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, &need);
+    qcnn_status rc = qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, QCNN_LUT_FP32, &need);
     if (rc != QCNN_OK) return rc;
     if (!x || !D || !codes || !y) return QCNN_ERR_INVALID_ARG;
     if (need > kScratchBytes) return QCNN_ERR_WORKSPACE;  // larger than the fixed scratch
@@ -64,5 +64,6 @@ extern "C" qcnn_status qcnn_fc_forward_noalloc(const float *x, int N, int Cs, in
         rc = scratch_address(&scratch);
         if (rc != QCNN_OK) return rc;
     }
-    return qcnn_fc_forward(x, N, Cs, Ct, D, Csp, K, codes, bias, y, relu, scratch, need, stream);
+    return qcnn_fc_forward(x, N, Cs, Ct, D, Csp, K, codes, bias, y, relu, QCNN_LUT_FP32, scratch,
+                           need, stream);
 }

@@ -3,6 +3,8 @@
 // max-pool used between the layers of the whole-network stack.
 #include "qcnn_internal.cuh"
 
+#include <cuda_bf16.h>
+
 #include <algorithm>
 
 namespace qcnn {
@@ -10,13 +12,15 @@ namespace qcnn {
 // lut[n][m][p][k] = sum_j x[n][m*Csp + j][p] * D[m][k][j].
 // A CTA owns 32 consecutive (m, p) units of one image; its 32*K outputs are
 // one contiguous, coalesced stretch of `lut`.  The kernel is bound by the
-// table writes (K/Csp floats written per float read).
+// table writes (K/Csp entries written per float read).  T = float, or
+// __nv_bfloat16 for entries rounded to bfloat16 (nearest, ties to even).
 constexpr int kLutUnits = 32;
 
+template <typename T>
 __global__ void __launch_bounds__(256) lut_build_kernel(const float *__restrict__ x, int Cs,
                                                         int P, const float *__restrict__ D,
                                                         int Csp, int K, int M,
-                                                        float *__restrict__ lut) {
+                                                        T *__restrict__ lut) {
     __shared__ float xs[kLutUnits][kMaxCsp];
     const int n = blockIdx.y;
     const long long units = (long long)M * P;
@@ -33,23 +37,28 @@ __global__ void __launch_bounds__(256) lut_build_kernel(const float *__restrict_
     }
     __syncthreads();
     const int nu = (int)std::min<long long>(kLutUnits, units - u0);
-    float *out = lut + ((size_t)n * units + u0) * K;
+    T *out = lut + ((size_t)n * units + u0) * K;
     for (int e = threadIdx.x; e < nu * K; e += blockDim.x) {
         const int ul = e / K, k = e % K;
         const int m = (int)((u0 + ul) / P);
         const float *dk = D + ((size_t)m * K + k) * Csp;
         float v = 0.f;
         for (int j = 0; j < Csp; ++j) v = fmaf(xs[ul][j], __ldg(dk + j), v);
-        out[e] = v;
+        if constexpr (sizeof(T) == 2) out[e] = __float2bfloat16_rn(v);
+        else out[e] = v;
     }
 }
 
 qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *D, int Csp,
-                             int K, float *lut, cudaStream_t st) {
+                             int K, void *lut, int bf16, cudaStream_t st) {
     const int M = Cs / Csp;
     const long long units = (long long)M * P;
     dim3 grid((unsigned)((units + kLutUnits - 1) / kLutUnits), N);
-    lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M, lut);
+    if (bf16)
+        lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M,
+                                               static_cast<__nv_bfloat16 *>(lut));
+    else
+        lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M, static_cast<float *>(lut));
     return after_launch();
 }
 

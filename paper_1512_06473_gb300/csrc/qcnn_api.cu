@@ -57,8 +57,11 @@ bool pq_ok(int Cs, int Csp, int K) {
     return Cs > 0 && Csp >= 1 && Csp <= kMaxCsp && K >= 1 && K <= kMaxK && Cs % Csp == 0;
 }
 
+bool lut_type_ok(int t) { return t == QCNN_LUT_FP32 || t == QCNN_LUT_BF16; }
+
 bool conv_shape(int N, int Cs, int H, int W, int Ct, int kh, int kw, int stride, int pad,
-                int Csp, int K, ConvShape *s) {
+                int Csp, int K, int lut_type, ConvShape *s) {
+    if (!lut_type_ok(lut_type)) return false;
     if (N <= 0 || H <= 0 || W <= 0 || Ct <= 0 || kh <= 0 || kw <= 0 || stride <= 0 || pad < 0)
         return false;
     if (!pq_ok(Cs, Csp, K)) return false;
@@ -68,16 +71,17 @@ bool conv_shape(int N, int Cs, int H, int W, int Ct, int kh, int kw, int stride,
     if (!fits_int((long long)N * Cs * H * W) || !fits_int((long long)N * Ct * Ho * Wo) ||
         !fits_int((long long)Ct * kh * kw * (Cs / Csp)))
         return false;
-    *s = ConvShape{N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, Cs / Csp, Ho, Wo};
+    *s = ConvShape{N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, Cs / Csp, Ho, Wo,
+                   lut_type == QCNN_LUT_BF16};
     return true;
 }
 
-bool fc_shape(int N, int Cs, int Ct, int Csp, int K, FcShape *s) {
-    if (N <= 0 || Ct <= 0 || !pq_ok(Cs, Csp, K)) return false;
+bool fc_shape(int N, int Cs, int Ct, int Csp, int K, int lut_type, FcShape *s) {
+    if (N <= 0 || Ct <= 0 || !pq_ok(Cs, Csp, K) || !lut_type_ok(lut_type)) return false;
     if (!fits_int((long long)N * Cs) || !fits_int((long long)N * Ct) ||
         !fits_int((long long)(Cs / Csp) * Ct))
         return false;
-    *s = FcShape{N, Cs, Ct, Csp, K, Cs / Csp};
+    *s = FcShape{N, Cs, Ct, Csp, K, Cs / Csp, lut_type == QCNN_LUT_BF16};
     return true;
 }
 
@@ -109,6 +113,8 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         if (c->cp.ok) c->algo = QCNN_ALGO_CHUNKED;
         else if (algo == QCNN_ALGO_CHUNKED) return QCNN_ERR_UNSUPPORTED;
     }
+    // the unfused path has fp32 tables only
+    if (c->algo == QCNN_ALGO_UNFUSED && s.bf16) return QCNN_ERR_UNSUPPORTED;
     size_t off = 0;
     c->packed_off = off;
     // the chunked path reads either code layout directly
@@ -193,7 +199,8 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
         if (L.kind == QCNN_LAYER_CONV) {
             if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
             ConvShape s;
-            if (!conv_shape(N, c, h, w, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K, &s))
+            if (!conv_shape(N, c, h, w, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K,
+                            L.lut_type, &s))
                 return QCNN_ERR_INVALID_ARG;
             qcnn_status rc = plan_conv_call(s, L.codes_layout, L.algo, &st.conv);
             if (rc != QCNN_OK) return rc;
@@ -205,7 +212,8 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
             if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
             const long long cs = (long long)c * h * w;
             if (cs >= INT_MAX) return QCNN_ERR_INVALID_ARG;
-            if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, &st.fc)) return QCNN_ERR_INVALID_ARG;
+            if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, L.lut_type, &st.fc))
+                return QCNN_ERR_INVALID_ARG;
             st.fcp = plan_fc(st.fc);
             st.scratch = align_up(st.fcp.partial_bytes, kWsAlign);
             st.oC = L.Ct;
@@ -293,27 +301,31 @@ int qcnn_last_cuda_error(void) { return g_last_cuda_error.load(); }
 uint64_t qcnn_launch_count(void) { return g_launches.load(); }
 
 qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W, const float *D, int Csp,
-                           int K, float *lut, void *stream) {
-    if (!x || !D || !lut || N <= 0 || H <= 0 || W <= 0 || !pq_ok(Cs, Csp, K))
+                           int K, void *lut, int lut_type, void *stream) {
+    if (!x || !D || !lut || N <= 0 || H <= 0 || W <= 0 || !pq_ok(Cs, Csp, K) ||
+        !lut_type_ok(lut_type))
         return QCNN_ERR_INVALID_ARG;
     const long long P = (long long)H * W;
     if (!fits_int((long long)N * Cs * P) || !fits_int((long long)N * (Cs / Csp) * P * K))
         return QCNN_ERR_INVALID_ARG;
-    return launch_lut_build(x, N, Cs, (int)P, D, Csp, K, lut, as_stream(stream));
+    return launch_lut_build(x, N, Cs, (int)P, D, Csp, K, lut, lut_type == QCNN_LUT_BF16,
+                            as_stream(stream));
 }
 
-qcnn_status qcnn_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K, size_t *bytes) {
+qcnn_status qcnn_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K, int lut_type,
+                                   size_t *bytes) {
     FcShape s;
-    if (!bytes || !fc_shape(N, Cs, Ct, Csp, K, &s)) return QCNN_ERR_INVALID_ARG;
+    if (!bytes || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s)) return QCNN_ERR_INVALID_ARG;
     *bytes = align_up(plan_fc(s).partial_bytes, kWsAlign);
     return QCNN_OK;
 }
 
 qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct, const float *D, int Csp,
                             int K, const uint8_t *codes, const float *bias, float *y, int relu,
-                            void *workspace, size_t workspace_bytes, void *stream) {
+                            int lut_type, void *workspace, size_t workspace_bytes,
+                            void *stream) {
     FcShape s;
-    if (!x || !D || !codes || !y || !fc_shape(N, Cs, Ct, Csp, K, &s))
+    if (!x || !D || !codes || !y || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
@@ -336,9 +348,9 @@ qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw, i
 
 qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh, int kw,
                                      int stride, int pad, int Csp, int K, int codes_layout,
-                                     int algo, size_t *bytes) {
+                                     int algo, int lut_type, size_t *bytes) {
     ConvShape s;
-    if (!bytes || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, &s))
+    if (!bytes || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
     qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
@@ -350,11 +362,11 @@ qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh
 qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int Ct, int kh,
                               int kw, int stride, int pad, const float *D, int Csp, int K,
                               const uint8_t *codes, int codes_layout, const float *bias,
-                              float *y, int relu, int algo, void *workspace,
+                              float *y, int relu, int algo, int lut_type, void *workspace,
                               size_t workspace_bytes, void *stream) {
     ConvShape s;
     if (!x || !D || !codes || !y ||
-        !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, &s))
+        !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
     qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);

@@ -29,6 +29,7 @@ qcnn_status after_launch();
 // ---------------------------------------------------------------- conv ----
 struct ConvShape {
     int N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, M, Ho, Wo;
+    int bf16;  // 1: table entries rounded to bfloat16 (QCNN_LUT_BF16)
 };
 
 // Fused plan: one CTA = (image, band of TH output rows, CT_CTA channels).
@@ -38,7 +39,8 @@ struct ConvFusedPlan {
     int P, CTW, WP;     // slots per warp, channels per warp, warps on positions
     int TH;             // output rows per CTA
     int pitch;          // W + 2 pad
-    int KS;             // floats per table row (per sub-codeword)
+    int KS;             // 32-bit words per table row (per sub-codeword; bf16:
+                        // both copies, 2 x an odd word count)
     int HP;             // halo positions with data: (TH + kh - 1) * pitch
     int ct_cta;         // channels per CTA
     int row_tiles, ct_tiles;
@@ -91,6 +93,7 @@ qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
 // ------------------------------------------------------------------ fc ----
 struct FcShape {
     int N, Cs, Ct, Csp, K, M;
+    int bf16;  // 1: table entries rounded to bfloat16 (QCNN_LUT_BF16)
 };
 struct FcPlan {
     int variant;        // kernel table index
@@ -109,8 +112,9 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x,
                       float *y, int relu, float *partial_ws, cudaStream_t st);
 
 // ------------------------------------------------------------ lut, pool ----
+// lut: fp32 entries, or bfloat16 bit patterns when bf16 != 0
 qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *D,
-                             int Csp, int K, float *lut, cudaStream_t st);
+                             int Csp, int K, void *lut, int bf16, cudaStream_t st);
 qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k,
                            int s, float *y, cudaStream_t st);
 
@@ -158,6 +162,24 @@ __device__ __forceinline__ void add2(float &a, float &b, float x, float y) {
     const float2 r = __fadd2_rn(make_float2(a, b), make_float2(x, y));
     a = r.x;
     b = r.y;
+}
+
+// a += low bfloat16 half of w, b += high half: each half widened to fp32
+// (exact) and added with one round-to-nearest fp32 addition, bit-identical
+// to converting first and adding in fp32.
+__device__ __forceinline__ void add_bf16x2(float &a, float &b, unsigned w) {
+    unsigned short lo, hi;
+    asm("mov.b32 {%0, %1}, %2;" : "=h"(lo), "=h"(hi) : "r"(w));
+    asm("add.rn.f32.bf16 %0, %1, %0;" : "+f"(a) : "h"(lo));
+    asm("add.rn.f32.bf16 %0, %1, %0;" : "+f"(b) : "h"(hi));
+}
+
+// Two fp32 values rounded to bfloat16 (nearest, ties to even) and packed:
+// lo in bits 0-15, hi in bits 16-31.
+__device__ __forceinline__ unsigned pack_bf16x2(float lo, float hi) {
+    unsigned r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
 }
 
 // acc[p] += v(p) for p < P, pairing the adds where possible.

@@ -40,19 +40,20 @@ N0 = None  # null device pointer
 def test_fc_rejects_bad_sizes(args):
     N, Cs, Ct, Csp, K = args
     nb = ctypes.c_size_t()
-    assert lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
-    assert lib.qcnn_fc_forward(8, N, Cs, Ct, 8, Csp, K, 8, None, 8, 0, None, 0, None) \
+    assert lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, 0, ctypes.byref(nb)) \
+        == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_forward(8, N, Cs, Ct, 8, Csp, K, 8, None, 8, 0, 0, None, 0, None) \
         == _lib.ERR_INVALID_ARG
 
 
 def test_fc_rejects_null_pointers():
-    assert lib.qcnn_fc_forward(None, 2, 8, 4, 8, 4, 16, 8, None, 8, 0, None, 0, None) \
+    assert lib.qcnn_fc_forward(None, 2, 8, 4, 8, 4, 16, 8, None, 8, 0, 0, None, 0, None) \
         == _lib.ERR_INVALID_ARG
-    assert lib.qcnn_fc_forward(8, 2, 8, 4, None, 4, 16, 8, None, 8, 0, None, 0, None) \
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, None, 4, 16, 8, None, 8, 0, 0, None, 0, None) \
         == _lib.ERR_INVALID_ARG
-    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, None, None, 8, 0, None, 0, None) \
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, None, None, 8, 0, 0, None, 0, None) \
         == _lib.ERR_INVALID_ARG
-    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, 8, None, None, 0, None, 0, None) \
+    assert lib.qcnn_fc_forward(8, 2, 8, 4, 8, 4, 16, 8, None, None, 0, 0, None, 0, None) \
         == _lib.ERR_INVALID_ARG
 
 
@@ -66,35 +67,48 @@ def test_fc_rejects_null_pointers():
 def test_conv_rejects_bad_sizes(args):
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = args
     nb = ctypes.c_size_t()
-    assert lib.qcnn_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, 0, 0,
+    assert lib.qcnn_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, 0, 0, 0,
                                         ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
     assert lib.qcnn_conv_forward(8, N, Cs, H, W, Ct, kh, kw, s, p, 8, Csp, K, 8, 0, None, 8, 0, 0,
-                                 None, 0, None) == _lib.ERR_INVALID_ARG
+                                 0, None, 0, None) == _lib.ERR_INVALID_ARG
 
 
 def test_conv_bad_enums_and_fused_stride():
     nb = ctypes.c_size_t()
-    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 7, 0,
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 7, 0, 0,
                                         ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
-    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 9,
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 9, 0,
                                         ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    # lut type outside the enum
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 0, 2,
+                                        ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_workspace_size(2, 8, 4, 4, 16, -1, ctypes.byref(nb)) \
+        == _lib.ERR_INVALID_ARG
     # the fused kernel serves stride 1 only
-    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 1,
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 1, 0,
                                         ctypes.byref(nb)) == _lib.ERR_UNSUPPORTED
-    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 0,
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 0, 0,
                                         ctypes.byref(nb)) == _lib.OK
+    # bf16 tables: fused and chunked serve them, the unfused path does not
+    for algo in (0, 1, 3):
+        assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, algo, 1,
+                                            ctypes.byref(nb)) == _lib.OK, algo
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 0, 0, 1,
+                                        ctypes.byref(nb)) == _lib.OK
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 2, 1,
+                                        ctypes.byref(nb)) == _lib.ERR_UNSUPPORTED
 
 
 def test_conv_workspace_too_small_is_reported_before_launch():
     nb = ctypes.c_size_t()
-    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 0,
+    assert lib.qcnn_conv_workspace_size(1, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 0, 0, 0,
                                         ctypes.byref(nb)) == _lib.OK
     assert nb.value > 0  # canonical codes are re-laid out in the workspace
     assert lib.qcnn_conv_forward(8, 1, 8, 9, 9, 4, 3, 3, 1, 1, 8, 4, 16, 8, 0, None, 8, 0, 0,
-                                 None, 0, None) == _lib.ERR_WORKSPACE
+                                 0, None, 0, None) == _lib.ERR_WORKSPACE
     # misaligned workspace
     assert lib.qcnn_conv_forward(8, 1, 8, 9, 9, 4, 3, 3, 1, 1, 8, 4, 16, 8, 0, None, 8, 0, 0,
-                                 4096 + 8, nb.value, None) == _lib.ERR_WORKSPACE
+                                 0, 4096 + 8, nb.value, None) == _lib.ERR_WORKSPACE
 
 
 def _layers(workload, N=1):

@@ -22,7 +22,7 @@ LIMIT = 16 << 20  # QCNN_FC_NOALLOC_SCRATCH_BYTES
 
 def _ws_bytes(lib, N, Cs, Ct, Csp, K):
     nb = ctypes.c_size_t()
-    assert lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)) == 0
+    assert lib.qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, 0, ctypes.byref(nb)) == 0
     return nb.value
 
 
@@ -43,7 +43,7 @@ def _with_workspace(lib, x, D, codes, bias, Ct, relu, stream):
     off = (-raw.data_ptr()) % 256
     y = torch.empty((N, Ct), dtype=torch.float32, device="cuda")
     rc = lib.qcnn_fc_forward(x.data_ptr(), N, Cs, Ct, D.data_ptr(), Csp, K, codes.data_ptr(),
-                             bias.data_ptr(), y.data_ptr(), int(relu), raw.data_ptr() + off,
+                             bias.data_ptr(), y.data_ptr(), int(relu), 0, raw.data_ptr() + off,
                              nbytes, stream)
     assert rc == 0
     return y
