@@ -17,6 +17,9 @@ Paper: Wu et al., "Quantized Convolutional Neural Networks for Mobile Devices"
   - ``lut_bf16=True``: every table entry rounded to bfloat16 (nearest, ties to
     even) before the sums, the rounding model of the library's reduced-precision
     table variant; ``round_bf16`` exposes that rounding.
+  - Quantizer: k-means in every sub-space (Eq. 4 for FC, Eq. 6 for conv),
+    ``kmeans``, ``pq_quantize_fc``, ``pq_quantize_conv`` (float32 in and out;
+    distances in binary32, centroid sums in double, see the C file).
 
 Array conventions (all numpy):
   fc:   x [N, Cs], codebooks D [M, K, Csp], codes [M, Ct] uint8, bias [Ct]
@@ -38,6 +41,7 @@ _SO = os.path.join(_HERE, "_build", "libqcnn_oracle.so")
 _lock = threading.Lock()
 
 _D = ctypes.POINTER(ctypes.c_double)
+_F = ctypes.POINTER(ctypes.c_float)
 _U8 = ctypes.POINTER(ctypes.c_uint8)
 GCC_FLAGS = ["-O2", "-std=c99", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
 
@@ -67,6 +71,10 @@ class OracleError(RuntimeError):
 
 def _f64(a):
     return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def _f32(a):
+    return np.ascontiguousarray(a, dtype=np.float32)
 
 
 def _u8(a):
@@ -99,8 +107,13 @@ class Oracle:
         lib.qo_round_bf16.argtypes = [ctypes.c_double]
         lib.qo_round_bf16.restype = ctypes.c_double
         lib.qo_maxpool.argtypes = [_D, i, i, i, i, i, i, _D]
+        i64 = ctypes.c_longlong
+        lib.qo_kmeans.argtypes = [_F, i64, i, i, _F, i, _F, _U8]
+        lib.qo_pq_quantize_fc.argtypes = [_F, i, i, i, i, _F, i, _F, _U8]
+        lib.qo_pq_quantize_conv.argtypes = [_F, i, i, i, i, i, i, _F, i, _F, _U8]
         for f in (lib.qo_fc_lut, lib.qo_fc_forward, lib.qo_conv_lut,
-                  lib.qo_conv_forward, lib.qo_maxpool):
+                  lib.qo_conv_forward, lib.qo_maxpool, lib.qo_kmeans,
+                  lib.qo_pq_quantize_fc, lib.qo_pq_quantize_conv):
             f.restype = ctypes.c_int
         self.lib = lib
 
@@ -177,6 +190,48 @@ class Oracle:
                "maxpool")
         return y
 
+    def kmeans(self, points, init, iters):
+        """Lloyd's k-means of points [P, d] from centroids init [K, d]:
+        returns (centroids [K, d] float32, assignment [P] uint8)."""
+        pts, ini = _f32(points), _f32(init)
+        P, d = pts.shape
+        K = ini.shape[0]
+        if ini.shape[1] != d:
+            raise OracleError("kmeans: dimension mismatch")
+        cen = np.empty((K, d), np.float32)
+        a = np.empty(P, np.uint8)
+        _check(self.lib.qo_kmeans(_p(pts, _F), P, d, K, _p(ini, _F), int(iters),
+                                  _p(cen, _F), _p(a, _U8)), "kmeans")
+        return cen, a
+
+    def pq_quantize_fc(self, W, Csp, K, init, iters):
+        """Eq. 4 for W [Ct, Cs]: returns D [M, K, Csp] and codes [M, Ct]."""
+        W, ini = _f32(W), _f32(init)
+        Ct, Cs = W.shape
+        M = Cs // Csp
+        if ini.shape != (M, K, Csp):
+            raise OracleError("pq_quantize_fc: init must be [M, K, Csp]")
+        D = np.empty((M, K, Csp), np.float32)
+        codes = np.empty((M, Ct), np.uint8)
+        _check(self.lib.qo_pq_quantize_fc(_p(W, _F), Ct, Cs, Csp, K, _p(ini, _F), int(iters),
+                                          _p(D, _F), _p(codes, _U8)), "pq_quantize_fc")
+        return D, codes
+
+    def pq_quantize_conv(self, W, Csp, K, init, iters):
+        """Eq. 6 for W [Ct, Cs, kh, kw]: returns D [M, K, Csp] and codes
+        [Ct, kh*kw, M]."""
+        W, ini = _f32(W), _f32(init)
+        Ct, Cs, kh, kw = W.shape
+        M = Cs // Csp
+        if ini.shape != (M, K, Csp):
+            raise OracleError("pq_quantize_conv: init must be [M, K, Csp]")
+        D = np.empty((M, K, Csp), np.float32)
+        codes = np.empty((Ct, kh * kw, M), np.uint8)
+        _check(self.lib.qo_pq_quantize_conv(_p(W, _F), Ct, Cs, kh, kw, Csp, K, _p(ini, _F),
+                                            int(iters), _p(D, _F), _p(codes, _U8)),
+               "pq_quantize_conv")
+        return D, codes
+
     def net_forward(self, x, layers, return_all=False):
         """Compose the oracle layers into a network (Sec. 4.2.3).
 
@@ -250,6 +305,18 @@ def maxpool(x, k, s):
 
 def net_forward(x, layers, return_all=False):
     return default().net_forward(x, layers, return_all)
+
+
+def kmeans(points, init, iters):
+    return default().kmeans(points, init, iters)
+
+
+def pq_quantize_fc(W, Csp, K, init, iters):
+    return default().pq_quantize_fc(W, Csp, K, init, iters)
+
+
+def pq_quantize_conv(W, Csp, K, init, iters):
+    return default().pq_quantize_conv(W, Csp, K, init, iters)
 
 
 def conv_out_size(H, W, kh, kw, stride, pad):

@@ -268,3 +268,142 @@ int qo_maxpool(const double *x, int N, int C, int H, int W, int k, int s,
     }
     return QO_OK;
 }
+
+/* ------------------------------------------------------------------ */
+/* Quantizer: k-means in every sub-space (Sec. 3.1, Eq. 4; Sec. 3.2,   */
+/* Eq. 6).  For sub-space m, the points are the m-th sub-vectors of    */
+/* all weight vectors (FC: one per c_t; conv: one per (c_t, p_k)); the */
+/* K centroids become D^(m) and the index of each point's centroid its */
+/* code, minimising sum ||D^(m) B^(m) - W^(m)||_F^2 (Lloyd's           */
+/* algorithm: alternate the assignment and the centroid update).       */
+/*                                                                     */
+/* Readings (the paper only says "k-means clustering"):                */
+/*   - the initial centroids are an input (the caller's seeded draw);  */
+/*   - `iters` rounds of (assign, update), then a final assignment     */
+/*     against the final centroids gives the codes;                    */
+/*   - squared distances are evaluated in binary32, term by term in    */
+/*     j order: d = sum_j (x_j - c_j)^2 with each subtraction,         */
+/*     product and sum rounded to binary32, because the assignment is  */
+/*     an integer decided by floating point and the GPU kernels decide */
+/*     it in that precision; ties go to the smallest index;            */
+/*   - a centroid is the mean of its points: the sum in double over    */
+/*     the points in index order, divided by the count, rounded to     */
+/*     binary32; a centroid with no points keeps its value.            */
+/* ------------------------------------------------------------------ */
+static int kmeans_assign(const float *pts, i64 P, int d, int K, const float *cen,
+                         uint8_t *assign)
+{
+    for (i64 p = 0; p < P; ++p) {
+        const float *x = pts + p * d;
+        int best = 0;
+        float best_d = 0.0f;
+        for (int k = 0; k < K; ++k) {
+            const float *c = cen + (i64)k * d;
+            float dist = 0.0f;
+            for (int j = 0; j < d; ++j) {
+                const float diff = x[j] - c[j];
+                const float sq = diff * diff;
+                dist = dist + sq;
+            }
+            if (k == 0 || dist < best_d) {
+                best = k;
+                best_d = dist;
+            }
+        }
+        assign[p] = (uint8_t)best;
+    }
+    return QO_OK;
+}
+
+static int kmeans_update(const float *pts, i64 P, int d, int K, const uint8_t *assign,
+                         float *cen)
+{
+    double *sum = (double *)calloc((size_t)K * d, sizeof(double));
+    i64 *cnt = (i64 *)calloc((size_t)K, sizeof(i64));
+    if (!sum || !cnt) { free(sum); free(cnt); return QO_ENOMEM; }
+    for (i64 p = 0; p < P; ++p) {
+        const int k = assign[p];
+        cnt[k] += 1;
+        for (int j = 0; j < d; ++j) sum[(i64)k * d + j] += (double)pts[p * d + j];
+    }
+    for (int k = 0; k < K; ++k)
+        if (cnt[k] > 0)
+            for (int j = 0; j < d; ++j)
+                cen[(i64)k * d + j] = (float)(sum[(i64)k * d + j] / (double)cnt[k]);
+    free(sum);
+    free(cnt);
+    return QO_OK;
+}
+
+/*
+ * k-means on the points of one sub-space.
+ * pts: [P][d] binary32; init: [K][d]; cen (out): [K][d]; assign (out): [P].
+ */
+int qo_kmeans(const float *pts, i64 P, int d, int K, const float *init, int iters,
+              float *cen, uint8_t *assign)
+{
+    if (P <= 0 || d <= 0 || K < 1 || K > 256 || iters < 0) return QO_EINVAL;
+    for (i64 e = 0; e < (i64)K * d; ++e) cen[e] = init[e];
+    for (int it = 0; it < iters; ++it) {
+        kmeans_assign(pts, P, d, K, cen, assign);
+        int rc = kmeans_update(pts, P, d, K, assign, cen);
+        if (rc) return rc;
+    }
+    return kmeans_assign(pts, P, d, K, cen, assign);
+}
+
+/*
+ * PQ quantization of an FC weight matrix (Eq. 4).  The paper's W is
+ * C_s x C_t with weight vectors as columns; here W is stored [Ct][Cs]
+ * (one weight vector per row).  init: [M][K][Csp].
+ * D (out): [M][K][Csp]; codes (out): [M][Ct].
+ */
+int qo_pq_quantize_fc(const float *W, int Ct, int Cs, int Csp, int K, const float *init,
+                      int iters, float *D, uint8_t *codes)
+{
+    if (check_pq(Cs, Csp, K) || Ct <= 0) return QO_EINVAL;
+    const int M = Cs / Csp;
+    float *pts = (float *)malloc(sizeof(float) * (size_t)Ct * Csp);
+    if (!pts) return QO_ENOMEM;
+    int rc = QO_OK;
+    for (int m = 0; m < M && rc == QO_OK; ++m) {
+        for (int ct = 0; ct < Ct; ++ct)
+            for (int j = 0; j < Csp; ++j)
+                pts[(i64)ct * Csp + j] = W[(i64)ct * Cs + m * Csp + j];
+        rc = qo_kmeans(pts, Ct, Csp, K, init + (i64)m * K * Csp, iters,
+                       D + (i64)m * K * Csp, codes + (i64)m * Ct);
+    }
+    free(pts);
+    return rc;
+}
+
+/*
+ * PQ quantization of conv kernels (Eq. 6): sub-space m pools the m-th
+ * sub-vectors of every kernel at every offset, point index
+ * p = c_t * (kh*kw) + p_k.  W: [Ct][Cs][kh][kw]; init: [M][K][Csp].
+ * D (out): [M][K][Csp]; codes (out): [Ct][kh*kw][M].
+ */
+int qo_pq_quantize_conv(const float *W, int Ct, int Cs, int kh, int kw, int Csp, int K,
+                        const float *init, int iters, float *D, uint8_t *codes)
+{
+    if (check_pq(Cs, Csp, K) || Ct <= 0 || kh <= 0 || kw <= 0) return QO_EINVAL;
+    const int M = Cs / Csp, KK = kh * kw;
+    const i64 P = (i64)Ct * KK;
+    float *pts = (float *)malloc(sizeof(float) * (size_t)P * Csp);
+    uint8_t *a = (uint8_t *)malloc((size_t)P);
+    if (!pts || !a) { free(pts); free(a); return QO_ENOMEM; }
+    int rc = QO_OK;
+    for (int m = 0; m < M && rc == QO_OK; ++m) {
+        for (int ct = 0; ct < Ct; ++ct)
+            for (int pk = 0; pk < KK; ++pk)
+                for (int j = 0; j < Csp; ++j)
+                    pts[((i64)ct * KK + pk) * Csp + j] =
+                        W[((i64)ct * Cs + m * Csp + j) * KK + pk];
+        rc = qo_kmeans(pts, P, Csp, K, init + (i64)m * K * Csp, iters,
+                       D + (i64)m * K * Csp, a);
+        for (i64 p = 0; p < P; ++p) codes[p * M + m] = a[p];
+    }
+    free(pts);
+    free(a);
+    return rc;
+}

@@ -463,9 +463,150 @@ def pin_bf16_tables(o):
     return fails
 
 
+# ----------------------------------------------------------- quantizer
+def _clustered(seed, K, d, per, spread=10.0, noise=0.3):
+    """K well-separated centres on a grid, `per` points each (shuffled)."""
+    r = _rng(seed)
+    grid = np.stack(np.meshgrid(*[np.arange(3)] * d, indexing="ij"), -1).reshape(-1, d)
+    centres = grid[r.choice(len(grid), K, replace=False)] * spread
+    labels = np.repeat(np.arange(K), per)
+    pts = centres[labels] + r.uniform(-noise, noise, (K * per, d))
+    order = r.permutation(K * per)
+    return pts[order].astype(np.float32), labels[order]
+
+
+def pin_kmeans_separated(o):
+    """Well-separated clusters: from one point of each cluster, Lloyd's
+    iterations find the true labels and each centroid is its cluster's mean."""
+    fails = []
+    for d, K in [(4, 16), (3, 9), (8, 5)]:
+        pts, labels = _clustered(41 + d, K, d, 37)
+        first = np.array([np.flatnonzero(labels == k)[0] for k in range(K)])
+        for iters in (1, 3):
+            cen, a = o.kmeans(pts, pts[first], iters)
+            if not np.array_equal(a, labels.astype(np.uint8)):
+                fails.append(f"d={d} K={K} iters={iters}: labels not recovered")
+                continue
+            want = np.stack([pts[labels == k].astype(np.float64).mean(0) for k in range(K)])
+            if np.max(np.abs(cen - want)) > 1e-6 * np.max(np.abs(want)):
+                fails.append(f"d={d} K={K} iters={iters}: centroids are not the cluster means")
+        # a duplicated initial centroid: exact distance ties go to the first
+        # index, and the copy, left without points, keeps its value
+        init = np.concatenate([pts[first], pts[first[:1]]])
+        _, a0 = o.kmeans(pts, init, 0)          # assignment to the initial centroids
+        cen1, _ = o.kmeans(pts, init, 1)        # one round: the copy had no points
+        if not np.array_equal(a0, labels.astype(np.uint8)):
+            fails.append(f"d={d} K={K}: an exact distance tie did not go to the first index")
+        if not np.array_equal(cen1[K], init[K]):
+            fails.append(f"d={d} K={K}: a centroid without points did not keep its value")
+    return fails
+
+
+def pin_kmeans_scipy(o):
+    """Lloyd's algorithm as scipy runs it (kmeans2 with a given initial
+    codebook, float64): same centroids after T rounds, and the same final
+    assignment as scipy's vq against them, on points whose nearest and
+    second-nearest centroids are not near-tied."""
+    import warnings
+
+    from scipy.cluster import vq as spvq
+    fails = []
+    r = _rng(43)
+    for (P, d, K, T) in [(600, 4, 8, 3), (400, 3, 16, 4), (300, 8, 4, 2), (64, 2, 256, 1)]:
+        pts = r.standard_normal((P, d)).astype(np.float32)
+        init = pts[r.choice(P, K, replace=K > P)] if K <= P else \
+            r.standard_normal((K, d)).astype(np.float32)
+        with warnings.catch_warnings():
+            warnings.simplefilter("ignore")  # empty clusters keep their centroid
+            ref_cb, _ = spvq.kmeans2(pts.astype(np.float64), init.astype(np.float64), iter=T,
+                                     minit="matrix", missing="warn")
+        ref_a, _ = spvq.vq(pts.astype(np.float64), ref_cb)
+        cen, a = o.kmeans(pts, init, T)
+        if np.max(np.abs(cen - ref_cb)) > 1e-6 * max(1.0, np.max(np.abs(ref_cb))):
+            fails.append(f"P={P} d={d} K={K} T={T}: centroids differ from scipy")
+            continue
+        dist = ((pts[:, None, :].astype(np.float64) - ref_cb[None]) ** 2).sum(-1)
+        two = np.sort(dist, axis=1)[:, :2]
+        clear = two[:, 1] - two[:, 0] > 1e-4 * (1 + two[:, 1])
+        if np.mean(clear) < 0.95 or not np.array_equal(a[clear], ref_a[clear]):
+            fails.append(f"P={P} d={d} K={K} T={T}: assignment differs from scipy")
+    return fails
+
+
+def pin_kmeans_distortion_monotone(o):
+    """Each Lloyd round can only lower sum ||x - c(x)||^2."""
+    r = _rng(47)
+    pts = r.standard_normal((500, 4)).astype(np.float32)
+    init = pts[:32]
+    prev, fails = np.inf, []
+    for T in range(6):
+        cen, a = o.kmeans(pts, init, T)
+        dist = float(((pts.astype(np.float64) - cen[a].astype(np.float64)) ** 2).sum())
+        if dist > prev * (1 + 1e-9):
+            fails.append(f"distortion rose at T={T}: {dist} > {prev}")
+        prev = dist
+    return fails
+
+
+def pin_pq_quantize_exact(o):
+    """Eq. 4 / Eq. 6 solved with zero error: a dense W whose sub-vectors are
+    drawn from K prototypes per sub-space.  Started from the prototypes, the
+    quantizer returns them and the codes W was built from; the PQ response
+    then equals the dense conv / FC of W (torch)."""
+    fails = []
+    r = _rng(53)
+    for (Ct, Cs, kh, kw, Csp, K) in [(12, 8, 3, 3, 4, 16), (7, 6, 1, 2, 3, 5), (5, 16, 2, 2, 8, 8)]:
+        M = Cs // Csp
+        D0 = r.standard_normal((M, K, Csp)).astype(np.float32)
+        c0 = r.integers(0, K, (Ct, kh * kw, M), dtype=np.uint8)
+        c0[:K, 0, :] = np.arange(K)[:, None] % K if Ct >= K else c0[:K, 0, :]
+        W = w_hat_conv(D0, c0, kh, kw).astype(np.float32)
+        D, codes = o.pq_quantize_conv(W, Csp, K, D0, 2)
+        used = np.zeros((M, K), bool)
+        used[np.arange(M)[None, None, :], c0.astype(np.int64)] = True
+        if not np.array_equal(codes, c0) or not np.array_equal(D[used], D0[used]):
+            fails.append(f"conv {Ct}x{Cs}x{kh}x{kw}: prototypes/codes not recovered")
+            continue
+        x = r.standard_normal((1, Cs, 6, 7))
+        got = o.conv_forward(x, D, codes, kh, kw, 1, 1)
+        ref = torch_conv(x, W.astype(np.float64), None, 1, 1, False)
+        if relerr(got, ref) > 1e-12:
+            fails.append(f"conv {Ct}x{Cs}: response differs from the dense conv")
+    for (Ct, Cs, Csp, K) in [(40, 12, 4, 8), (33, 16, 2, 32)]:
+        M = Cs // Csp
+        D0 = r.standard_normal((M, K, Csp)).astype(np.float32)
+        c0 = r.integers(0, K, (M, Ct), dtype=np.uint8)
+        W = w_hat_fc(D0, c0).astype(np.float32)
+        D, codes = o.pq_quantize_fc(W, Csp, K, D0, 2)
+        used = np.zeros((M, K), bool)
+        used[np.arange(M)[:, None], c0.astype(np.int64)] = True
+        if not np.array_equal(codes, c0) or not np.array_equal(D[used], D0[used]):
+            fails.append(f"fc {Ct}x{Cs}: prototypes/codes not recovered")
+            continue
+        x = r.standard_normal((3, Cs))
+        if relerr(o.fc_forward(x, D, codes), torch_fc(x, W.astype(np.float64), None, False)) > 1e-12:
+            fails.append(f"fc {Ct}x{Cs}: response differs from the dense FC")
+    return fails
+
+
+def pin_pq_quantize_conv_1x1_is_fc(o):
+    """A 1x1 conv kernel set quantizes like the FC matrix it equals."""
+    r = _rng(59)
+    Ct, Cs, Csp, K = 50, 12, 3, 8
+    W = r.standard_normal((Ct, Cs)).astype(np.float32)
+    init = r.standard_normal((Cs // Csp, K, Csp)).astype(np.float32)
+    Dc, cc = o.pq_quantize_conv(W[:, :, None, None], Csp, K, init, 3)
+    Df, cf = o.pq_quantize_fc(W, Csp, K, init, 3)
+    if not (np.array_equal(Dc, Df) and np.array_equal(cc[:, 0, :].T, cf)):
+        return ["1x1 conv quantization differs from the FC quantization"]
+    return []
+
+
 ALL_PINS = [pin_conv_vs_dense, pin_fc_vs_dense, pin_integer_exact, pin_exactness,
             pin_linearity, pin_permutation, pin_k1_closed_form, pin_conv_fc_equivalence,
-            pin_lut_one_hot, pin_maxpool, pin_tiny_net, pin_bf16_rounding, pin_bf16_tables]
+            pin_lut_one_hot, pin_maxpool, pin_tiny_net, pin_bf16_rounding, pin_bf16_tables,
+            pin_kmeans_separated, pin_kmeans_scipy, pin_kmeans_distortion_monotone,
+            pin_pq_quantize_exact, pin_pq_quantize_conv_1x1_is_fc]
 
 
 def run_all(o):

@@ -53,6 +53,29 @@ MUTANTS = {
     "bf16_flag_ignored": (
         "lut[(i64)m * K + k] = lut_bf16 ? qo_round_bf16(acc) : acc;",
         "lut[(i64)m * K + k] = acc;"),
+    "kmeans_argmax": (
+        "if (k == 0 || dist < best_d) {", "if (k == 0 || dist > best_d) {"),
+    "kmeans_ties_to_last": (
+        "if (k == 0 || dist < best_d) {", "if (k == 0 || dist <= best_d) {"),
+    "kmeans_l1_distance": (
+        "const float sq = diff * diff;", "const float sq = diff < 0 ? -diff : diff;"),
+    "kmeans_mean_off_by_one": (
+        "(float)(sum[(i64)k * d + j] / (double)cnt[k]);",
+        "(float)(sum[(i64)k * d + j] / (double)(cnt[k] + 1));"),
+    "kmeans_empty_cluster_divided": (
+        "        if (cnt[k] > 0)\n", "        if (cnt[k] >= 0)\n"),
+    "kmeans_final_assignment_skipped": (
+        "    return kmeans_assign(pts, P, d, K, cen, assign);", "    return QO_OK;"),
+    "kmeans_one_round_short": (
+        "for (int it = 0; it < iters; ++it) {", "for (int it = 0; it < iters - 1; ++it) {"),
+    "pq_conv_offsets_reversed": (
+        "W[((i64)ct * Cs + m * Csp + j) * KK + pk];",
+        "W[((i64)ct * Cs + m * Csp + j) * KK + (KK - 1 - pk)];"),
+    "pq_conv_codes_layout": (
+        "codes[p * M + m] = a[p];", "codes[m * P + p] = a[p];"),
+    "pq_fc_subvectors_interleaved": (
+        "pts[(i64)ct * Csp + j] = W[(i64)ct * Cs + m * Csp + j];",
+        "pts[(i64)ct * Csp + j] = W[(i64)ct * Cs + j * M + m];"),
     "lut_dot_product_drops_last_dim": (
         "for (int j = 0; j < Csp; ++j)\n                acc +=",
         "for (int j = 0; j < Csp - 1; ++j)\n                acc +="),
