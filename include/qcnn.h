@@ -220,6 +220,47 @@ typedef struct {
     const float *bias;  /* [Ct] or NULL, device                              */
 } qcnn_layer;
 
+/*
+ * Quantizer: learning D and the codes from dense weights by k-means in
+ * every sub-space (Sec. 3.1, Eq. 4 for FC; Sec. 3.2, Eq. 6 for conv), all
+ * sub-spaces at once.  Lloyd's algorithm from caller-supplied initial
+ * centroids: `iters` rounds of (assign every point to its nearest centroid;
+ * move every centroid to the mean of its points), then a last assignment
+ * against the final centroids gives the codes.
+ *   - distances: sum_j (x_j - c_j)^2 in binary32, term by term (each
+ *     subtraction, square and sum rounded, no fused multiply-add); ties go
+ *     to the smallest index;
+ *   - means: coordinates summed in double in point-index order, divided by
+ *     the count, rounded to binary32; a centroid without points keeps its
+ *     value.
+ * Both rules are fixed, so the results are reproducible bit for bit.
+ *
+ * qcnn_kmeans: generic form.
+ *   points [M][P][Csp] fp32, init [M][K][Csp] fp32 (device)
+ *   D      [M][K][Csp] fp32, written;  assign [M][P] uint8, written
+ * qcnn_pq_quantize: a layer's weights.
+ *   kind QCNN_LAYER_FC:   W [Ct][Cs] (one weight vector per row; kh, kw
+ *                         ignored); codes [M][Ct] (qcnn_fc_forward layout)
+ *   kind QCNN_LAYER_CONV: W [Ct][Cs][kh][kw]; sub-space m pools the m-th
+ *                         sub-vectors of every kernel at every offset, point
+ *                         p = c_t * kh*kw + p_k; codes [Ct][kh*kw][M]
+ *                         (qcnn_conv_forward canonical layout)
+ *   init [M][K][Csp]; D [M][K][Csp] written.
+ * Limits as for the forward calls (1 <= Csp <= 8, 1 <= K <= 256,
+ * Cs % Csp == 0), iters >= 0.  Workspace from the matching query,
+ * 256-byte aligned.
+ */
+qcnn_status qcnn_kmeans_workspace_size(int M, int P, int Csp, int K, size_t *bytes);
+qcnn_status qcnn_kmeans(const float *points, int M, int P, int Csp, int K,
+                        const float *init, int iters, float *D, uint8_t *assign,
+                        void *workspace, size_t workspace_bytes, void *stream);
+qcnn_status qcnn_pq_quantize_workspace_size(int kind, int Ct, int Cs, int kh, int kw,
+                                            int Csp, int K, size_t *bytes);
+qcnn_status qcnn_pq_quantize(int kind, const float *W, int Ct, int Cs, int kh, int kw,
+                             int Csp, int K, const float *init, int iters, float *D,
+                             uint8_t *codes, void *workspace, size_t workspace_bytes,
+                             void *stream);
+
 /* Output shape of the stack for one image (C, H, W; H = W = 1 after an FC). */
 qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers,
                                   int C, int H, int W, int *out_C, int *out_H,

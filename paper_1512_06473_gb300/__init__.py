@@ -25,6 +25,7 @@ from . import _lib
 from ._lib import QcnnError, load  # noqa: F401
 
 __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
+           "kmeans", "pq_quantize_fc", "pq_quantize_conv",
            "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
 
 
@@ -172,6 +173,64 @@ def maxpool(x, k, s, out=None, stream=None):
     _lib.check(load().qcnn_maxpool(_ptr(x), N, C, H, W, k, s, _ptr(out), _stream(stream)),
                "qcnn_maxpool")
     return out
+
+
+# ---------------------------------------------------------------- quantizer
+def kmeans(points, init, iters, stream=None):
+    """k-means in each of M sub-spaces (Eq. 4 / Eq. 6): points [M, P, Csp],
+    init [M, K, Csp] -> (D [M, K, Csp] float32, assign [M, P] uint8)."""
+    _need(points, "points", torch.float32, 3)
+    _need(init, "init", torch.float32, 3)
+    M, P, Csp = points.shape
+    K = init.shape[1]
+    if init.shape != (M, K, Csp):
+        raise ValueError("init must be [M, K, Csp]")
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_kmeans_workspace_size(M, P, Csp, K, ctypes.byref(nb)),
+               "qcnn_kmeans_workspace_size")
+    ws, wsb = _workspace(nb.value, points.device, None)
+    D = torch.empty((M, K, Csp), dtype=torch.float32, device=points.device)
+    a = torch.empty((M, P), dtype=torch.uint8, device=points.device)
+    _lib.check(lib.qcnn_kmeans(_ptr(points), M, P, Csp, K, _ptr(init), int(iters), _ptr(D),
+                               _ptr(a), _ptr(ws), wsb, _stream(stream)), "qcnn_kmeans")
+    return D, a
+
+
+def _pq_quantize(kind, W, Csp, K, init, iters, stream):
+    _need(init, "init", torch.float32, 3)
+    if kind == _lib.LAYER_FC:
+        _need(W, "W", torch.float32, 2)
+        (Ct, Cs), kh, kw = W.shape, 1, 1
+    else:
+        _need(W, "W", torch.float32, 4)
+        Ct, Cs, kh, kw = W.shape
+    M = Cs // Csp
+    if init.shape != (M, K, Csp):
+        raise ValueError("init must be [M, K, Csp]")
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_pq_quantize_workspace_size(kind, Ct, Cs, kh, kw, Csp, K,
+                                                   ctypes.byref(nb)),
+               "qcnn_pq_quantize_workspace_size")
+    ws, wsb = _workspace(nb.value, W.device, None)
+    D = torch.empty((M, K, Csp), dtype=torch.float32, device=W.device)
+    shape = (M, Ct) if kind == _lib.LAYER_FC else (Ct, kh * kw, M)
+    codes = torch.empty(shape, dtype=torch.uint8, device=W.device)
+    _lib.check(lib.qcnn_pq_quantize(kind, _ptr(W), Ct, Cs, kh, kw, Csp, K, _ptr(init),
+                                    int(iters), _ptr(D), _ptr(codes), _ptr(ws), wsb,
+                                    _stream(stream)), "qcnn_pq_quantize")
+    return D, codes
+
+
+def pq_quantize_fc(W, Csp, K, init, iters, stream=None):
+    """Eq. 4: W [Ct, Cs] -> (D [M, K, Csp], codes [M, Ct])."""
+    return _pq_quantize(_lib.LAYER_FC, W, Csp, K, init, iters, stream)
+
+
+def pq_quantize_conv(W, Csp, K, init, iters, stream=None):
+    """Eq. 6: W [Ct, Cs, kh, kw] -> (D [M, K, Csp], codes [Ct, kh*kw, M])."""
+    return _pq_quantize(_lib.LAYER_CONV, W, Csp, K, init, iters, stream)
 
 
 # ------------------------------------------------------------------ network

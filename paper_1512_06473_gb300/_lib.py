@@ -63,6 +63,13 @@ _SIGS = {
                                  c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
     "qcnn_net_forward_host": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int,
                                       c_int, c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "qcnn_kmeans_workspace_size": (c_int, [c_int, c_int, c_int, c_int, ctypes.POINTER(c_size_t)]),
+    "qcnn_kmeans": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_void_p,
+                            c_void_p, c_void_p, c_size_t, c_void_p]),
+    "qcnn_pq_quantize_workspace_size": (c_int, [c_int] * 7 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_pq_quantize": (c_int, [c_int, c_void_p, c_int, c_int, c_int, c_int, c_int, c_int,
+                                 c_void_p, c_int, c_void_p, c_void_p, c_void_p, c_size_t,
+                                 c_void_p]),
 }
 
 _lock = threading.Lock()

@@ -53,6 +53,12 @@ def uniform_codes(shape, K: int, seed: int, *salt: int) -> np.ndarray:
     return rng(seed, *salt).integers(0, K, size=shape, dtype=np.uint8)
 
 
+def sample_indices(n: int, k: int, seed: int, *salt: int) -> np.ndarray:
+    """k indices drawn from range(n): distinct when k <= n, with repeats
+    otherwise (the initial-centroid draw of a k-means run)."""
+    return rng(seed, *salt).choice(n, size=k, replace=k > n).astype(np.int64)
+
+
 def small_integers(shape, lo: int, hi: int, seed: int, *salt: int) -> np.ndarray:
     """float32 holding integers uniform in [lo, hi] -- every sum of a few
     thousand products of such values is exact in fp32 and in fp64."""

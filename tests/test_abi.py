@@ -165,3 +165,21 @@ def test_net_rejects_mismatched_layer():
         == _lib.ERR_INVALID_ARG
     assert lib.qcnn_net_workspace_size(None, 3, 1, 3, 227, 227, 0, ctypes.byref(nb)) \
         == _lib.ERR_INVALID_ARG
+
+
+def test_quantizer_argument_checks():
+    nb = ctypes.c_size_t()
+    FC, CONV = _lib.LAYER_FC, _lib.LAYER_CONV
+    assert lib.qcnn_pq_quantize_workspace_size(FC, 10, 12, 0, 0, 4, 16, ctypes.byref(nb)) == _lib.OK
+    assert nb.value > 0
+    assert lib.qcnn_pq_quantize_workspace_size(CONV, 10, 12, 3, 3, 4, 16, ctypes.byref(nb)) == _lib.OK
+    for bad in [(FC, 10, 12, 0, 0, 5, 16), (FC, 10, 12, 0, 0, 4, 0), (FC, 10, 12, 0, 0, 4, 257),
+                (CONV, 10, 12, 0, 3, 4, 16), (7, 10, 12, 1, 1, 4, 16), (FC, 0, 12, 1, 1, 4, 16),
+                (FC, 10, 18, 1, 1, 9, 16)]:
+        assert lib.qcnn_pq_quantize_workspace_size(*bad, ctypes.byref(nb)) == _lib.ERR_INVALID_ARG, bad
+    assert lib.qcnn_kmeans_workspace_size(4, 100, 4, 16, ctypes.byref(nb)) == _lib.OK
+    assert lib.qcnn_kmeans(None, 4, 100, 4, 16, 8, 2, 8, 8, 8, nb.value, None) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_kmeans(8, 4, 100, 4, 16, 8, -1, 8, 8, 8, nb.value, None) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_kmeans(8, 4, 100, 4, 16, 8, 2, 8, 8, None, 0, None) == _lib.ERR_WORKSPACE
+    assert lib.qcnn_pq_quantize(FC, 8, 10, 12, 1, 1, 4, 16, 8, 2, 8, 8, 4096 + 8, 1 << 20,
+                                None) == _lib.ERR_WORKSPACE  # misaligned workspace
