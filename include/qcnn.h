@@ -51,7 +51,9 @@ typedef enum {
     QCNN_ERR_INVALID_ARG = 1, /* bad size, null pointer, limit exceeded     */
     QCNN_ERR_UNSUPPORTED = 2, /* valid request this build cannot serve      */
     QCNN_ERR_WORKSPACE = 3,   /* workspace smaller than the query asked for */
-    QCNN_ERR_CUDA = 4         /* a CUDA call or kernel launch failed        */
+    QCNN_ERR_CUDA = 4,        /* a CUDA call or kernel launch failed        */
+    QCNN_ERR_DATA = 5         /* input data unusable (rank-deficient
+                                 calibration set of qcnn_ec_quantize_fc)    */
 } qcnn_status;
 
 typedef enum {
@@ -260,6 +262,32 @@ qcnn_status qcnn_pq_quantize(int kind, const float *W, int Ct, int Cs, int kh, i
                              int Csp, int K, const float *init, int iters, float *D,
                              uint8_t *codes, void *workspace, size_t workspace_bytes,
                              void *stream);
+
+/*
+ * qcnn_ec_quantize_fc -- quantization with error correction of an FC layer
+ * (Sec. 3.3.1, Eq. 8-12): minimises
+ *     sum_n || T_n - sum_m (D^(m) B^(m))^T S_n^(m) ||^2
+ * over N calibration vectors (S_n: the layer input in the quantized
+ * network, T_n: the response of the original layer), by block coordinate
+ * descent over the sub-spaces m = 0..M-1, `outer` sweeps.  For each m the
+ * residual of Eq. 9 is held fixed and `inner` alternations run, each a
+ * codeword update (Eq. 11: per-codeword least squares, solved with the
+ * Cholesky factor of G = sum_n S_n^(m) S_n^(m)T; a codeword assigned to no
+ * output keeps its value) followed by an assignment update (Eq. 12, ties
+ * to the smallest index).  Arithmetic in double.
+ *   S [N][Cs] fp32, T [N][Ct] fp32 (device)
+ *   D [M][K][Csp] fp32, codes [M][Ct] uint8: the starting point on entry
+ *     (e.g. from qcnn_pq_quantize), the result on return
+ * Synchronizes `stream` before returning.  Returns QCNN_ERR_DATA when some
+ * G is not positive definite (fewer than Csp independent calibration
+ * sub-vectors); D and codes are then unspecified.
+ */
+qcnn_status qcnn_ec_quantize_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K,
+                                               size_t *bytes);
+qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, int Ct,
+                                int Csp, int K, float *D, uint8_t *codes, int outer,
+                                int inner, void *workspace, size_t workspace_bytes,
+                                void *stream);
 
 /* Output shape of the stack for one image (C, H, W; H = W = 1 after an FC). */
 qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers,

@@ -25,7 +25,7 @@ from . import _lib
 from ._lib import QcnnError, load  # noqa: F401
 
 __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
-           "kmeans", "pq_quantize_fc", "pq_quantize_conv",
+           "kmeans", "pq_quantize_fc", "pq_quantize_conv", "ec_quantize_fc",
            "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
 
 
@@ -231,6 +231,29 @@ def pq_quantize_fc(W, Csp, K, init, iters, stream=None):
 def pq_quantize_conv(W, Csp, K, init, iters, stream=None):
     """Eq. 6: W [Ct, Cs, kh, kw] -> (D [M, K, Csp], codes [Ct, kh*kw, M])."""
     return _pq_quantize(_lib.LAYER_CONV, W, Csp, K, init, iters, stream)
+
+
+def ec_quantize_fc(S, T, D, codes, outer, inner, stream=None):
+    """Error-corrected FC quantization (Eq. 8 - 12) from the starting point
+    (D [M, K, Csp], codes [M, Ct]) on calibration pairs S [N, Cs], T [N, Ct].
+    Returns new (D, codes); the inputs are not modified."""
+    _need(S, "S", torch.float32, 2)
+    _need(T, "T", torch.float32, 2)
+    _need(D, "D", torch.float32, 3)
+    _need(codes, "codes", torch.uint8, 2)
+    N, Cs = S.shape
+    Ct = T.shape[1]
+    M, K, Csp = D.shape
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_ec_quantize_fc_workspace_size(N, Cs, Ct, Csp, K, ctypes.byref(nb)),
+               "qcnn_ec_quantize_fc_workspace_size")
+    ws, wsb = _workspace(nb.value, S.device, None)
+    D2, c2 = D.clone(), codes.clone()
+    _lib.check(lib.qcnn_ec_quantize_fc(_ptr(S), _ptr(T), N, Cs, Ct, Csp, K, _ptr(D2), _ptr(c2),
+                                       int(outer), int(inner), _ptr(ws), wsb, _stream(stream)),
+               "qcnn_ec_quantize_fc")
+    return D2, c2
 
 
 # ------------------------------------------------------------------ network

@@ -11,7 +11,7 @@ from . import build as _build
 
 c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_uint64
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_DATA = 0, 1, 2, 3, 4, 5
 ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3}
 CODES_CANONICAL, CODES_PACKED = 0, 1
 LUT = {"fp32": 0, "bf16": 1}
@@ -67,6 +67,10 @@ _SIGS = {
     "qcnn_kmeans": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_void_p,
                             c_void_p, c_void_p, c_size_t, c_void_p]),
     "qcnn_pq_quantize_workspace_size": (c_int, [c_int] * 7 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_ec_quantize_fc_workspace_size": (c_int, [c_int] * 5 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_ec_quantize_fc": (c_int, [c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_int,
+                                    c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t,
+                                    c_void_p]),
     "qcnn_pq_quantize": (c_int, [c_int, c_void_p, c_int, c_int, c_int, c_int, c_int, c_int,
                                  c_void_p, c_int, c_void_p, c_void_p, c_void_p, c_size_t,
                                  c_void_p]),

@@ -292,6 +292,7 @@ const char *qcnn_status_string(qcnn_status s) {
         case QCNN_ERR_UNSUPPORTED: return "unsupported by this build";
         case QCNN_ERR_WORKSPACE: return "workspace too small or misaligned";
         case QCNN_ERR_CUDA: return "CUDA error";
+        case QCNN_ERR_DATA: return "input data unusable (rank-deficient calibration set)";
     }
     return "unknown status";
 }

@@ -124,6 +124,11 @@ qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k,
 #ifdef __CUDACC__
 namespace qcnn {
 
+// quantize.cu: one CTA of kSortThreads (1024) threads per label array of P
+// entries: order[*] = indices grouped by label, increasing inside a group;
+// starts[k] = first slot of label k, starts[K] = P.
+__global__ void kmeans_order_kernel(const uint8_t *assign, int P, int K, int *order, int *starts);
+
 __device__ __forceinline__ unsigned smem_addr(const void *p) {
     return static_cast<unsigned>(__cvta_generic_to_shared(p));
 }
