@@ -602,11 +602,43 @@ def pin_pq_quantize_conv_1x1_is_fc(o):
     return []
 
 
+# ---------------------------------------------------------------- bit codes
+def pin_bits(o):
+    """Bit packing (oracle/bits.py) against hand-worked streams, numpy's
+    little-endian packbits of the bit expansion, and the round trip."""
+    from oracle import bits
+    fails = []
+    worked = [
+        (([1, 2, 3], 2), bytes([0b00111001])),           # 01 | 10 | 11, LSB first
+        (([5, 31, 0, 17], 5), bytes([0xE5, 0x83, 0x08])),  # 17 -> stream bits 15 and 19
+        (([255, 1], 8), bytes([255, 1])),
+        (([1, 0, 1, 1, 0, 0, 0, 1, 1], 1), bytes([0b10001101, 0b1])),
+        (([7, 7, 7], 3), bytes([0xFF, 0x01])),
+    ]
+    for (codes, b), want in worked:
+        if bits.pack(codes, b) != want:
+            fails.append(f"pack({codes}, {b}) = {bits.pack(codes, b).hex()}, want {want.hex()}")
+    if [bits.bits_for(K) for K in (1, 2, 3, 4, 5, 16, 17, 32, 128, 129, 256)] != \
+            [1, 1, 2, 2, 3, 4, 5, 5, 7, 8, 8]:
+        fails.append("bits_for")
+    r = _rng(83)
+    for b in range(1, 9):
+        c = r.integers(0, 1 << b, 1000)
+        expand = ((c[:, None] >> np.arange(b)[None, :]) & 1).astype(np.uint8).ravel()
+        ref = np.packbits(expand, bitorder="little").tobytes()
+        got = bits.pack(c, b)
+        if got != ref:
+            fails.append(f"b={b}: differs from numpy packbits")
+        if not np.array_equal(bits.unpack(got, len(c), b), c.astype(np.uint8)):
+            fails.append(f"b={b}: round trip")
+    return fails
+
+
 ALL_PINS = [pin_conv_vs_dense, pin_fc_vs_dense, pin_integer_exact, pin_exactness,
             pin_linearity, pin_permutation, pin_k1_closed_form, pin_conv_fc_equivalence,
             pin_lut_one_hot, pin_maxpool, pin_tiny_net, pin_bf16_rounding, pin_bf16_tables,
             pin_kmeans_separated, pin_kmeans_scipy, pin_kmeans_distortion_monotone,
-            pin_pq_quantize_exact, pin_pq_quantize_conv_1x1_is_fc]
+            pin_pq_quantize_exact, pin_pq_quantize_conv_1x1_is_fc, pin_bits]
 
 
 def run_all(o):

@@ -91,3 +91,27 @@ def test_mutant_is_caught(name, tmp_path):
     so = oracle.compile_c(str(src), str(tmp_path / "libmutant.so"))
     fails = pins.run_all(oracle.Oracle(so))
     assert fails, f"no pin caught the planted mistake {name!r}"
+
+
+
+@pytest.mark.parametrize("name,old,new", [
+    ("bits_msb_first", "out[s // 8] |= 1 << (s % 8)", "out[s // 8] |= 1 << (7 - s % 8)"),
+    ("bits_code_bits_reversed", "if (c >> t) & 1:", "if (c >> (b - 1 - t)) & 1:"),
+    ("bits_rounded_down", "while (1 << b) < K:", "while (1 << b) <= K // 2 + 1:"),
+])
+def test_bits_mutant_is_caught(name, old, new, tmp_path, monkeypatch):
+    import importlib.util
+    import sys
+
+    from oracle import bits
+    src = open(bits.__file__).read()
+    assert src.count(old) == 1, name
+    path = tmp_path / "bits.py"
+    path.write_text(src.replace(old, new))
+    spec = importlib.util.spec_from_file_location("oracle.bits", path)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    monkeypatch.setitem(sys.modules, "oracle.bits", mod)
+    import oracle as pkg
+    monkeypatch.setattr(pkg, "bits", mod, raising=False)
+    assert pins.pin_bits(oracle.default()), f"no pin caught {name!r}"
