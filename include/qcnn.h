@@ -127,6 +127,34 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
                             size_t workspace_bytes, void *stream);
 
 /*
+ * Bit-packed codes: the storage model of Table 1 (Sec. 3.4), each code in
+ * b = qcnn_code_bits(K) = ceil(log2 K) bits (at least 1).  Stream layout:
+ * code i occupies stream bits [i*b, (i+1)*b), its bit t at stream bit
+ * i*b + t; stream bit s is bit (s mod 8) of byte s / 8.
+ *   qcnn_pack_bits / qcnn_unpack_bits: n codes <-> ceil(n*b/8) stream
+ *     bytes (device buffers; packing clamps codes to 2^b - 1).
+ *   qcnn_fc_pack_codes: FC codes [M][Ct] -> M rows, each packed on its own
+ *     and zero-padded to a 16-byte pitch (qcnn_fc_packed_codes_bytes in
+ *     all); codes >= K are clamped to K - 1.
+ *   qcnn_fc_forward_packed: qcnn_fc_forward reading those rows (16-byte
+ *     aligned), same result, 8/b times fewer code bytes; the workspace is
+ *     the one qcnn_fc_workspace_size gives.  In a qcnn_layer, an FC layer
+ *     with codes_layout QCNN_CODES_PACKED takes them too.
+ */
+int qcnn_code_bits(int K);
+qcnn_status qcnn_pack_bits(const uint8_t *codes, long long n, int bits, uint8_t *stream,
+                           void *cuda_stream);
+qcnn_status qcnn_unpack_bits(const uint8_t *stream, long long n, int bits, uint8_t *codes,
+                             void *cuda_stream);
+size_t qcnn_fc_packed_codes_bytes(int M, int Ct, int K);
+qcnn_status qcnn_fc_pack_codes(const uint8_t *codes, int M, int Ct, int K, uint8_t *packed,
+                               void *stream);
+qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const float *D,
+                                   int Csp, int K, const uint8_t *packed, const float *bias,
+                                   float *y, int relu, int lut_type, void *workspace,
+                                   size_t workspace_bytes, void *stream);
+
+/*
  * qcnn_fc_forward_noalloc -- the same result as qcnn_fc_forward, for callers
  * that cannot hand the library any device memory: code running inside
  * another runtime's execution step, where that runtime owns all device
@@ -215,7 +243,8 @@ typedef struct {
     int Csp, K;         /* CONV / FC: sub-space dimension, sub-codewords     */
     int relu;           /* CONV / FC: 1 = ReLU after the bias                */
     int algo;           /* CONV: qcnn_algo                                   */
-    int codes_layout;   /* CONV: qcnn_codes_layout of `codes`                */
+    int codes_layout;   /* CONV: qcnn_codes_layout of `codes`; FC: CANONICAL
+                           ([M][Ct] bytes) or PACKED (qcnn_fc_pack_codes)   */
     int lut_type;       /* CONV / FC: qcnn_lut_type of the table entries     */
     const float *D;     /* CONV / FC: [M][K][Csp], device                    */
     const uint8_t *codes; /* CONV: see qcnn_conv_forward; FC: [M][Ct]; device */
@@ -288,6 +317,39 @@ qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, i
                                 int Csp, int K, float *D, uint8_t *codes, int outer,
                                 int inner, void *workspace, size_t workspace_bytes,
                                 void *stream);
+
+/*
+ * Model blob: a whole stack in one byte string, codes stored in
+ * ceil(log2 K) bits (the storage model of Table 1) -- 4 Cs K bytes of
+ * sub-codebooks plus kh kw M Ct log2(K) / 8 bytes of codes per layer, and
+ * the biases.  Layout (little-endian, arrays 16-byte aligned):
+ *   header   32 B: "QCNNMDL1", u32 version 1, u32 n_layers, u32 C, H, W,
+ *                  u32 0
+ *   records  80 B per layer: u32 kind, Ct, kh, kw, stride, pad, Csp, K,
+ *                  relu, bits, has_bias, Cs; u64 off_D, off_codes,
+ *                  off_bias, 0 (offsets from the end of the records)
+ *   payload  D [M][K][Csp] fp32; codes, one bit stream (qcnn_pack_bits
+ *            layout) in the canonical order (FC [M][Ct], conv
+ *            [Ct][kh*kw][M]); bias [Ct] fp32
+ * qcnn_model_serialize: `layers` hold HOST pointers (D, canonical codes,
+ *   bias or NULL) for the input C x H x W; writes the blob to host memory
+ *   `out` (NULL: only sets *bytes_needed).  QCNN_ERR_WORKSPACE when
+ *   out_bytes is too small.
+ * qcnn_model_info: validates a blob in host memory (every size, offset and
+ *   the layer chain) and gives its layer count, input shape and the device
+ *   bytes qcnn_model_upload needs.
+ * qcnn_model_upload: copies the blob's arrays into `device_buffer` (256-byte
+ *   aligned, at least that size), lays the codes out for the kernels and
+ *   fills layers[n_layers] with device pointers into it (codes_layout
+ *   PACKED, algo AUTO, lut_type FP32), ready for qcnn_net_forward.
+ *   Synchronizes `stream` before returning.
+ */
+qcnn_status qcnn_model_serialize(const qcnn_layer *layers, int n_layers, int C, int H, int W,
+                                 void *out, size_t out_bytes, size_t *bytes_needed);
+qcnn_status qcnn_model_info(const void *blob, size_t bytes, int *n_layers, int *C, int *H,
+                            int *W, size_t *device_bytes);
+qcnn_status qcnn_model_upload(const void *blob, size_t bytes, void *device_buffer,
+                              size_t device_bytes, qcnn_layer *layers, void *stream);
 
 /* Output shape of the stack for one image (C, H, W; H = W = 1 after an FC). */
 qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers,

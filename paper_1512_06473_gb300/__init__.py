@@ -26,6 +26,8 @@ from ._lib import QcnnError, load  # noqa: F401
 
 __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
            "kmeans", "pq_quantize_fc", "pq_quantize_conv", "ec_quantize_fc",
+           "code_bits", "pack_bits", "unpack_bits", "fc_pack_codes", "serialize_model",
+           "model_info", "load_model",
            "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
 
 
@@ -88,14 +90,21 @@ def lut_build(x: torch.Tensor, D: torch.Tensor, out: Optional[torch.Tensor] = No
 
 
 def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, stream=None,
-               lut="fp32"):
-    """Eq. 5: y[n, ct] = bias[ct] + sum_m LUT_n[m, codes[m, ct]] (then ReLU)."""
+               lut="fp32", Ct=None):
+    """Eq. 5: y[n, ct] = bias[ct] + sum_m LUT_n[m, codes[m, ct]] (then ReLU).
+    ``codes`` is [M, Ct] uint8, or the 1-d output of fc_pack_codes (then
+    ``Ct`` is required)."""
     _need(x, "x", torch.float32, 2)
     _need(D, "D", torch.float32, 3)
-    _need(codes, "codes", torch.uint8, 2)
+    packed = codes.dim() == 1
+    _need(codes, "codes", torch.uint8, 1 if packed else 2)
     N, Cs = x.shape
     M, K, Csp = D.shape
-    Ct = codes.shape[1]
+    if packed:
+        if Ct is None:
+            raise ValueError("Ct is required with packed codes")
+    else:
+        Ct = codes.shape[1]
     if bias is not None:
         _need(bias, "bias", torch.float32, 1)
     lib = load()
@@ -106,9 +115,49 @@ def fc_forward(x, D, codes, bias=None, relu=False, out=None, workspace=None, str
     ws, wsb = _workspace(nb.value, x.device, workspace)
     if out is None:
         out = torch.empty((N, Ct), dtype=torch.float32, device=x.device)
-    _lib.check(lib.qcnn_fc_forward(_ptr(x), N, Cs, Ct, _ptr(D), Csp, K, _ptr(codes),
-                                   _ptr(bias), _ptr(out), int(bool(relu)), lt, _ptr(ws), wsb,
-                                   _stream(stream)), "qcnn_fc_forward")
+    fn = lib.qcnn_fc_forward_packed if packed else lib.qcnn_fc_forward
+    _lib.check(fn(_ptr(x), N, Cs, Ct, _ptr(D), Csp, K, _ptr(codes), _ptr(bias), _ptr(out),
+                  int(bool(relu)), lt, _ptr(ws), wsb, _stream(stream)), "qcnn_fc_forward")
+    return out
+
+
+def _aligned_bytes(nbytes, device, align=256):
+    raw = torch.empty(nbytes + align, dtype=torch.uint8, device=device)
+    off = (-raw.data_ptr()) % align
+    return raw[off:off + nbytes]
+
+
+def code_bits(K: int) -> int:
+    """Bits per stored code, ceil(log2 K) (at least 1)."""
+    return int(load().qcnn_code_bits(K))
+
+
+def pack_bits(codes: torch.Tensor, bits: int, stream=None) -> torch.Tensor:
+    """Codes (any shape, uint8) -> the packed stream, ceil(n*bits/8) bytes."""
+    _need(codes, "codes", torch.uint8, codes.dim())
+    n = codes.numel()
+    out = torch.empty((n * bits + 7) // 8, dtype=torch.uint8, device=codes.device)
+    _lib.check(load().qcnn_pack_bits(_ptr(codes), n, bits, _ptr(out), _stream(stream)),
+               "qcnn_pack_bits")
+    return out
+
+
+def unpack_bits(stream_bytes: torch.Tensor, n: int, bits: int, stream=None) -> torch.Tensor:
+    _need(stream_bytes, "stream_bytes", torch.uint8, 1)
+    out = torch.empty(n, dtype=torch.uint8, device=stream_bytes.device)
+    _lib.check(load().qcnn_unpack_bits(_ptr(stream_bytes), n, bits, _ptr(out), _stream(stream)),
+               "qcnn_unpack_bits")
+    return out
+
+
+def fc_pack_codes(codes: torch.Tensor, K: int, stream=None) -> torch.Tensor:
+    """FC codes [M, Ct] -> bit-packed rows (16-byte pitch) for fc_forward."""
+    _need(codes, "codes", torch.uint8, 2)
+    M, Ct = codes.shape
+    lib = load()
+    out = _aligned_bytes(lib.qcnn_fc_packed_codes_bytes(M, Ct, K), codes.device)
+    _lib.check(lib.qcnn_fc_pack_codes(_ptr(codes), M, Ct, K, _ptr(out), _stream(stream)),
+               "qcnn_fc_pack_codes")
     return out
 
 
@@ -276,10 +325,12 @@ class ConvLayer:
 @dataclass
 class FCLayer:
     D: torch.Tensor
-    codes: torch.Tensor         # [M, Ct]
+    codes: torch.Tensor         # [M, Ct], or fc_pack_codes rows (packed=True, Ct given)
     bias: Optional[torch.Tensor]
     relu: bool = True
     lut: str = "fp32"
+    packed: bool = False
+    Ct: Optional[int] = None
 
 
 @dataclass
@@ -306,7 +357,9 @@ class Net:
                 d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
             elif isinstance(L, FCLayer):
                 M, K, Csp = L.D.shape
-                d.kind, d.Ct, d.Csp, d.K, d.relu = _lib.LAYER_FC, L.codes.shape[1], Csp, K, int(L.relu)
+                ct = L.Ct if L.packed else L.codes.shape[1]
+                d.kind, d.Ct, d.Csp, d.K, d.relu = _lib.LAYER_FC, ct, Csp, K, int(L.relu)
+                d.codes_layout = _lib.CODES_PACKED if L.packed else _lib.CODES_CANONICAL
                 d.lut_type = _lib.LUT[L.lut]
                 d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)
             elif isinstance(L, PoolLayer):
@@ -368,3 +421,92 @@ class Net:
                                                 workspace.numel(), _stream(stream)),
                    "qcnn_net_forward_host")
         return out_host
+
+
+# ------------------------------------------------------------- model blob
+def _host_layers(layers):
+    """(qcnn_layer array with host pointers, arrays kept alive)."""
+    import numpy as np
+    arr = (_lib.Layer * len(layers))()
+    keep = []
+    for i, L in enumerate(layers):
+        d = arr[i]
+        kind = L["kind"]
+        if kind == "maxpool":
+            d.kind, d.kh, d.kw, d.stride = _lib.LAYER_MAXPOOL, L["k"], L["k"], L["s"]
+            continue
+        D = np.ascontiguousarray(L["D"], np.float32)
+        codes = np.ascontiguousarray(L["codes"], np.uint8)
+        bias = None if L.get("bias") is None else np.ascontiguousarray(L["bias"], np.float32)
+        keep += [D, codes, bias]
+        M, K, Csp = D.shape
+        if kind == "conv":
+            d.kind, d.Ct, d.kh, d.kw = _lib.LAYER_CONV, codes.shape[0], L["kh"], L["kw"]
+            d.stride, d.pad = L.get("stride", 1), L.get("pad", 0)
+        else:
+            d.kind, d.Ct = _lib.LAYER_FC, codes.shape[1]
+        d.Csp, d.K, d.relu = Csp, K, int(bool(L.get("relu", False)))
+        d.D, d.codes = D.ctypes.data, codes.ctypes.data
+        d.bias = None if bias is None else bias.ctypes.data
+    return arr, keep
+
+
+def serialize_model(layers, in_shape) -> bytes:
+    """A stack (list of dicts: {"kind": "conv"|"fc"|"maxpool", "D", "codes" in
+    the canonical layout, "bias", "kh", "kw", "stride", "pad", "relu"} or
+    {"kind": "maxpool", "k", "s"}, numpy arrays) -> the model blob."""
+    arr, keep = _host_layers(layers)
+    C, H, W = in_shape
+    lib = load()
+    need = ctypes.c_size_t()
+    _lib.check(lib.qcnn_model_serialize(arr, len(arr), C, H, W, None, 0, ctypes.byref(need)),
+               "qcnn_model_serialize")
+    buf = ctypes.create_string_buffer(need.value)
+    _lib.check(lib.qcnn_model_serialize(arr, len(arr), C, H, W, buf, need.value,
+                                        ctypes.byref(need)), "qcnn_model_serialize")
+    return buf.raw[:need.value]
+
+
+def model_info(blob: bytes):
+    """(n_layers, (C, H, W), device bytes) of a blob."""
+    n, C, H, W = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    nb = ctypes.c_size_t()
+    _lib.check(load().qcnn_model_info(blob, len(blob), ctypes.byref(n), ctypes.byref(C),
+                                      ctypes.byref(H), ctypes.byref(W), ctypes.byref(nb)),
+               "qcnn_model_info")
+    return n.value, (C.value, H.value, W.value), nb.value
+
+
+class LoadedNet(Net):
+    """A Net whose parameters live in one device buffer filled from a blob."""
+
+    def __init__(self, blob: bytes, device="cuda", stream=None):
+        n, in_shape, nbytes = model_info(blob)
+        self.buffer = _aligned_bytes(max(nbytes, 1), torch.device(device))
+        arr = (_lib.Layer * n)()
+        _lib.check(load().qcnn_model_upload(blob, len(blob), _ptr(self.buffer), nbytes, arr,
+                                            _stream(stream)), "qcnn_model_upload")
+        self.layers = [None] * n
+        self.in_shape = tuple(in_shape)
+        self._arr = arr
+        C, H, W = self.in_shape
+        oc, oh, ow = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+        _lib.check(load().qcnn_net_output_shape(arr, n, C, H, W, ctypes.byref(oc),
+                                                ctypes.byref(oh), ctypes.byref(ow)),
+                   "qcnn_net_output_shape")
+        self.out_shape = (oc.value, oh.value, ow.value)
+
+    def set_lut(self, lut: str):
+        """Table precision of every PQ layer ("fp32" or "bf16")."""
+        for d in self._arr:
+            if d.kind != _lib.LAYER_MAXPOOL:
+                d.lut_type = _lib.LUT[lut]
+
+
+def load_model(blob_or_path, device="cuda", stream=None) -> LoadedNet:
+    """Load a model blob (bytes, or a file path) onto the GPU."""
+    blob = blob_or_path
+    if not isinstance(blob, (bytes, bytearray)):
+        with open(blob_or_path, "rb") as f:
+            blob = f.read()
+    return LoadedNet(bytes(blob), device, stream)

@@ -63,6 +63,21 @@ _SIGS = {
                                  c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
     "qcnn_net_forward_host": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int,
                                       c_int, c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "qcnn_code_bits": (c_int, [c_int]),
+    "qcnn_model_serialize": (c_int, [ctypes.POINTER(Layer), c_int, c_int, c_int, c_int, c_void_p,
+                                     c_size_t, ctypes.POINTER(c_size_t)]),
+    "qcnn_model_info": (c_int, [c_void_p, c_size_t, ctypes.POINTER(c_int), ctypes.POINTER(c_int),
+                                ctypes.POINTER(c_int), ctypes.POINTER(c_int),
+                                ctypes.POINTER(c_size_t)]),
+    "qcnn_model_upload": (c_int, [c_void_p, c_size_t, c_void_p, c_size_t, ctypes.POINTER(Layer),
+                                  c_void_p]),
+    "qcnn_pack_bits": (c_int, [c_void_p, ctypes.c_longlong, c_int, c_void_p, c_void_p]),
+    "qcnn_unpack_bits": (c_int, [c_void_p, ctypes.c_longlong, c_int, c_void_p, c_void_p]),
+    "qcnn_fc_packed_codes_bytes": (c_size_t, [c_int, c_int, c_int]),
+    "qcnn_fc_pack_codes": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_void_p]),
+    "qcnn_fc_forward_packed": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int,
+                                       c_void_p, c_void_p, c_void_p, c_int, c_int, c_void_p,
+                                       c_size_t, c_void_p]),
     "qcnn_kmeans_workspace_size": (c_int, [c_int, c_int, c_int, c_int, ctypes.POINTER(c_size_t)]),
     "qcnn_kmeans": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_void_p,
                             c_void_p, c_void_p, c_size_t, c_void_p]),

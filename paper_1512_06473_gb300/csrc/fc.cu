@@ -16,6 +16,11 @@
 // (2i, 2i+1) for the same (mm, k) -- both use the same code -- so one load
 // serves two look-ups; the word pitch of a row is odd as above.  Tiles of a
 // single image per lane keep 2-byte entries (pitch NT | 1 halves).
+// Codes can also come bit-packed (b = ceil(log2 K) bits each, every [M][Ct]
+// row padded to a 16-byte pitch): a CTA's slice of a row is then b * CT_CTA
+// / 8 bytes, staged with 16-byte copies, and a lane takes its 4 codes from one
+// funnel shift of two 32-bit words -- 8/b times fewer code bytes from HBM,
+// which is what bounds the layer at batch 1.
 // When the sub-space range is split over several CTAs (to fill the GPU),
 // the partial sums go to the workspace and a second kernel adds them in a
 // fixed order (deterministic), then applies bias and ReLU.
@@ -41,6 +46,9 @@ struct FcArgs {
     int NTX;     // odd pitch of a staged x row (>= NT)
     int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
     int cvec_log2;
+    int cbits;   // 0: one byte per code; else bits per code (packed rows)
+    int cpitch;  // packed: bytes per code row (multiple of 16)
+    int crb;     // bytes per staged code row in shared memory (CT_CTA + 16)
     int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
 };
 
@@ -51,7 +59,9 @@ constexpr int kMchMax = 16;   // sub-spaces per chunk, at most
 struct FcSmem {
     size_t lut, xs, ds, cs, total;
 };
-// row_bytes: bytes of one table row (NTP entries or words)
+// row_bytes: bytes of one table row (NTP entries or words); code rows are
+// staged at a stride of CT_CTA + 16 bytes (byte codes, or a packed slice plus
+// the word the last lane's shift reads past it)
 __host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int row_bytes, int NTX,
                                                  int Csp, int CT_CTA) {
     FcSmem s;
@@ -59,7 +69,7 @@ __host__ __device__ inline FcSmem fc_smem_layout(int MCH, int K, int row_bytes, 
     s.xs = ((size_t)MCH * K * row_bytes + 15) / 16 * 16;
     s.ds = s.xs + ((size_t)2 * MCH * Csp * NTX * 4 + 15) / 16 * 16;
     s.cs = s.ds + ((size_t)2 * MCH * K * Csp * 4 + 15) / 16 * 16;
-    s.total = s.cs + (size_t)2 * MCH * CT_CTA;
+    s.total = s.cs + (size_t)2 * MCH * (CT_CTA + 16);
     return s;
 }
 
@@ -122,8 +132,22 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         const float *dsrc = a.D + (size_t)m0 * a.K * a.Csp;
         for (int e = tid; e < dn; e += kFcThreads) cp_async4(db + e, e < dv ? dsrc + e : a.D, e < dv);
         // codes[m0 + mm][ct0 .. ct0 + CT_CTA) -> cs[b][mm][.]; zero outside
-        uint8_t *cb = cs + (size_t)b * a.MCH * CT_CTA;
-        if (a.cvec > 0) {
+        uint8_t *cb = cs + (size_t)b * a.MCH * a.crb;
+        if (a.cbits) {  // packed rows: this CTA's slice, whole 16-byte copies
+            const int slice = (CT_CTA * a.cbits) >> 3;
+            const int nq = slice >> 4;
+            const size_t off0 = (size_t)blockIdx.x * slice;
+            for (int e = tid; e < a.MCH * nq; e += kFcThreads) {
+                const int mm = e / nq, qq = e - mm * nq;
+                const size_t byte = off0 + (size_t)qq * 16;
+                const bool ok = mm < mch && byte < (size_t)a.cpitch;
+                const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.cpitch + byte : a.codes;
+                const unsigned d = smem_addr(cb + mm * a.crb + qq * 16);
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src),
+                             "r"(ok ? 16 : 0)
+                             : "memory");
+            }
+        } else if (a.cvec > 0) {
             const int row_log2 = kCtCtaLog2 - a.cvec_log2;  // copies per code row
             const int per_row = 1 << row_log2;
             for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
@@ -131,7 +155,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 const int ct = ct0 + q * a.cvec;
                 const bool ok = mm < mch && ct < a.Ct;  // Ct % cvec == 0: all or nothing
                 const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
-                void *dst = cb + mm * CT_CTA + q * a.cvec;
+                void *dst = cb + mm * a.crb + q * a.cvec;
                 const unsigned d = smem_addr(dst);
                 const int sz = ok ? a.cvec : 0;
                 if (a.cvec == 16)
@@ -145,7 +169,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
             for (int e = tid; e < a.MCH * CT_CTA; e += kFcThreads) {
                 const int mm = e / CT_CTA, q = e % CT_CTA;
                 const int ct = ct0 + q;
-                cb[e] = (mm < mch && ct < a.Ct) ? a.codes[(size_t)(m0 + mm) * a.Ct + ct] : 0;
+                cb[mm * a.crb + q] = (mm < mch && ct < a.Ct) ? a.codes[(size_t)(m0 + mm) * a.Ct + ct] : 0;
             }
         }
         cp_async_commit();
@@ -209,12 +233,22 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         __syncthreads();
 
         // gather
-        const uint8_t *cb = cs + (size_t)b * a.MCH * CT_CTA + lane_ct;
+        const uint8_t *cb = cs + (size_t)b * a.MCH * a.crb;
+        const int bit0 = lane_ct * a.cbits;  // packed: first bit of the lane's codes
+        const unsigned cmask = (1u << a.cbits) - 1u;
 #pragma unroll
         for (int mm = 0; mm < kMchMax; ++mm) {
             if (mm < mch) {
-                const unsigned w =
-                    __vminu4(*reinterpret_cast<const unsigned *>(cb + mm * CT_CTA), kmax4);
+                unsigned w;
+                if (a.cbits) {  // 4 codes of b bits -> 4 bytes
+                    const unsigned *cw = reinterpret_cast<const unsigned *>(cb + mm * a.crb);
+                    const unsigned v = __funnelshift_r(cw[bit0 >> 5], cw[(bit0 >> 5) + 1], bit0 & 31);
+                    w = (v & cmask) | (((v >> a.cbits) & cmask) << 8) |
+                        (((v >> (2 * a.cbits)) & cmask) << 16) | (((v >> (3 * a.cbits)) & cmask) << 24);
+                } else {
+                    w = *reinterpret_cast<const unsigned *>(cb + mm * a.crb + lane_ct);
+                }
+                w = __vminu4(w, kmax4);
 #pragma unroll
                 for (int q = 0; q < kCPL; ++q) {
                     const int code = (int)byte_of(w, q);
@@ -335,6 +369,8 @@ FcPlan plan_fc(const FcShape &s) {
         const double per_chunk = (double)MCH * NT * CT_CTA / (fv.BF && fv.NW % 2 == 0 ? 64.0 : 32.0) +
                                  (double)MCH * s.K * NT / 32.0 * 2;
         const double t_smem = waves * cpsplit * per_chunk * cps_sm / 1.2e9 / fv.eff;
+        // (byte codes counted for both code layouts, so that packed and
+        // unpacked calls make the same plan and share one workspace query)
         const double bytes = (double)s.M * s.Ct * n_tiles + 4.0 * s.N * s.Cs * ct_tiles +
                              (splits > 1 ? 8.0 * splits * s.N * s.Ct : 0.0);
         const double t = std::max(t_smem, bytes / 6.0e12) + (splits > 1 ? 3e-6 : 0.0);
@@ -388,6 +424,9 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
              : (s.Ct % 4 == 0 && base % 4 == 0) ? 4
                                                  : 0;
     a.cvec_log2 = a.cvec == 16 ? 4 : a.cvec == 8 ? 3 : 2;
+    a.cbits = s.code_bits;
+    a.cpitch = s.code_bits ? (int)fc_packed_pitch(s.Ct, s.K) : 0;
+    a.crb = p.CT_CTA + 16;
     a.cch_log2 = 0;
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     cudaError_t e =

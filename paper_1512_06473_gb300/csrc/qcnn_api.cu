@@ -81,7 +81,7 @@ bool fc_shape(int N, int Cs, int Ct, int Csp, int K, int lut_type, FcShape *s) {
     if (!fits_int((long long)N * Cs) || !fits_int((long long)N * Ct) ||
         !fits_int((long long)(Cs / Csp) * Ct))
         return false;
-    *s = FcShape{N, Cs, Ct, Csp, K, Cs / Csp, lut_type == QCNN_LUT_BF16};
+    *s = FcShape{N, Cs, Ct, Csp, K, Cs / Csp, lut_type == QCNN_LUT_BF16, 0};
     return true;
 }
 
@@ -214,6 +214,8 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
             if (cs >= INT_MAX) return QCNN_ERR_INVALID_ARG;
             if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, L.lut_type, &st.fc))
                 return QCNN_ERR_INVALID_ARG;
+            if (L.codes_layout == QCNN_CODES_PACKED) st.fc.code_bits = code_bits(L.K);
+            else if (L.codes_layout != QCNN_CODES_CANONICAL) return QCNN_ERR_INVALID_ARG;
             st.fcp = plan_fc(st.fc);
             st.scratch = align_up(st.fcp.partial_bytes, kWsAlign);
             st.oC = L.Ct;
@@ -331,6 +333,21 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct, const float *
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
     return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(workspace),
+                     as_stream(stream));
+}
+
+qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const float *D,
+                                   int Csp, int K, const uint8_t *packed, const float *bias,
+                                   float *y, int relu, int lut_type, void *workspace,
+                                   size_t workspace_bytes, void *stream) {
+    FcShape s;
+    if (!x || !D || !packed || !y || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s))
+        return QCNN_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(packed) % 16 != 0) return QCNN_ERR_INVALID_ARG;
+    s.code_bits = code_bits(K);
+    const FcPlan p = plan_fc(s);
+    if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
+    return launch_fc(s, p, x, D, packed, bias, y, relu, static_cast<float *>(workspace),
                      as_stream(stream));
 }
 

@@ -93,8 +93,17 @@ qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
 // ------------------------------------------------------------------ fc ----
 struct FcShape {
     int N, Cs, Ct, Csp, K, M;
-    int bf16;  // 1: table entries rounded to bfloat16 (QCNN_LUT_BF16)
+    int bf16;       // 1: table entries rounded to bfloat16 (QCNN_LUT_BF16)
+    int code_bits;  // 0: codes [M][Ct] bytes; else bit-packed rows (bits.cu)
 };
+
+int code_bits(int K);                   // ceil(log2 K), at least 1
+size_t fc_packed_pitch(int Ct, int K);  // bytes per packed FC code row
+qcnn_status launch_pack_bits(const uint8_t *codes, long long row_len, long long rows,
+                             long long in_pitch, long long out_pitch, int b, int K, uint8_t *out,
+                             cudaStream_t st);
+qcnn_status launch_unpack_bits(const uint8_t *in, long long n, int b, uint8_t *codes,
+                               cudaStream_t st);
 struct FcPlan {
     int variant;        // kernel table index
     int NT, CT_CTA;     // images and outputs per CTA
