@@ -43,6 +43,8 @@ def parse():
     p.add_argument("--impl", choices=["qcnn", "reference"], default="qcnn")
     p.add_argument("--batch", type=int, default=BATCH)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-extras", action="store_true",
+                   help="skip the model-blob and quantizer measurements")
     p.add_argument("--cpu-sample", type=int, default=0,
                    help="images in the CPU-baseline sample (default: one per worker)")
     return p.parse_args()
@@ -245,6 +247,136 @@ def recorded_traffic(workload, batch, layer):
     return None
 
 
+def extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N, batch1, cm,
+                       with_oracle):
+    """The rows beyond the forward path: the stack loaded from a model blob
+    (codes in ceil(log2 K) bits), and the quantizers (k-means, Eq. 4/6;
+    error correction, Eq. 8-12), each timed on the GPU and, on rank 0 of a
+    single-GPU run, the float64 oracle on one layer beside it."""
+    import numpy as np
+
+    res = {}
+
+    def event_ms(fn, reps, flush_each=True):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ts = []
+        for _ in range(reps):
+            if flush_each:
+                flush.zero_()
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1))
+        return float(np.median(ts))
+
+    # ---- model blob
+    layers = [synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, params)]
+    blob = q.serialize_model(layers, w.in_shape)
+    lnet = q.load_model(blob, dev)
+    lws = lnet.alloc_workspace(N, dev)
+    for _ in range(3):
+        lnet.forward(x, out=out, workspace=lws)
+    torch.cuda.synchronize(dev)
+    steps = max(5, a.steps // 3)
+    ms = event_ms(lambda: lnet.forward(x, out=out, workspace=lws), steps)
+    dense = sum(c.dense_bytes for c in _layer_costs(w, cm))
+    res["model_blob"] = {
+        "bytes": len(blob), "dense_fp32_weight_bytes": int(dense),
+        "compression": round(dense / len(blob), 2),
+        "note": "codes in ceil(log2 K) bits (Table 1 storage), sub-codebooks and biases fp32; "
+                "FC layers of the loaded stack read the bit-packed codes directly",
+        "value": round(N / (ms / 1e3), 1), "unit": "images/s", "ms_per_step": round(ms, 4),
+        "batch1": batch1(lnet)}
+    # fc6 at batch 1, byte codes vs packed rows (L2 flushed: codes come from HBM)
+    j6 = next(j for j, L in enumerate(w.layers) if isinstance(L, synth.FC))
+    L6, P6 = w.layers[j6], params[j6]
+    x6 = torch.from_numpy(synth.relu_normal((1, L6.Cs), 7)).to(dev)
+    D6 = torch.from_numpy(P6["D"]).to(dev)
+    c6 = torch.from_numpy(P6["codes"]).to(dev)
+    p6 = q.fc_pack_codes(c6, L6.K)
+    y6 = torch.empty((1, L6.Ct), device=dev)
+    t_byte = event_ms(lambda: q.fc_forward(x6, D6, c6, out=y6), 20)
+    t_pack = event_ms(lambda: q.fc_forward(x6, D6, p6, out=y6, Ct=L6.Ct), 20)
+    res["model_blob"]["fc6_batch1_us"] = {"byte_codes": round(t_byte * 1e3, 1),
+                                          "packed_codes": round(t_pack * 1e3, 1),
+                                          "code_bytes": [int(c6.numel()), int(p6.numel())]}
+
+    # ---- quantizer: k-means in every sub-space of every PQ layer, 10 rounds
+    rounds = 10
+    jobs = []
+    for j, L in enumerate(w.layers):
+        if isinstance(L, synth.Pool):
+            continue
+        fan = L.Cs * (L.kh * L.kw if isinstance(L, synth.Conv) else 1)
+        shape = (L.Ct, L.Cs, L.kh, L.kw) if isinstance(L, synth.Conv) else (L.Ct, L.Cs)
+        Wd = synth.normal(shape, (2.0 / fan) ** 0.5, 150, j)
+        M = L.Cs // L.Csp
+        if isinstance(L, synth.Conv):
+            pts = Wd.reshape(L.Ct, M, L.Csp, L.kh * L.kw).transpose(1, 0, 3, 2).reshape(M, -1, L.Csp)
+        else:
+            pts = Wd.reshape(L.Ct, M, L.Csp).transpose(1, 0, 2)
+        init = np.stack([pts[m][synth.sample_indices(pts.shape[1], L.K, 151, j, m)]
+                         for m in range(M)])
+        jobs.append((j, L, torch.from_numpy(Wd).to(dev), torch.from_numpy(init).to(dev), Wd, init))
+
+    def quantize_all():
+        for j, L, Wt, It, _, _ in jobs:
+            if isinstance(L, synth.Conv):
+                q.pq_quantize_conv(Wt, L.Csp, L.K, It, rounds)
+            else:
+                q.pq_quantize_fc(Wt, L.Csp, L.K, It, rounds)
+
+    quantize_all()
+    t_q = event_ms(quantize_all, 3, flush_each=False)
+    ops = sum((L.Cs // L.Csp) * L.Ct * (L.kh * L.kw if isinstance(L, synth.Conv) else 1) * L.K
+              * 3 * L.Csp * (rounds + 1) for _, L, *_ in jobs)
+    qres = {"kmeans_alexnet_all_layers_ms": round(t_q, 2), "rounds": rounds,
+            "assign_ops": ops, "assign_gops_per_s": round(ops / (t_q / 1e3) / 1e9, 1),
+            "note": "assignment: 3 binary32 ops per coordinate per (point, centroid); the time "
+                    "includes the sort and the double-precision centroid sums"}
+    # error correction on an fc8-shaped layer (4096 -> 1000, C's 4, K 32), 512 vectors
+    Ne, Cse, Cte, Cspe, Ke = 512, 4096, 1000, 4, 32
+    S = synth.relu_normal((Ne, Cse), 152)
+    We = synth.normal((Cte, Cse), (2.0 / Cse) ** 0.5, 153)
+    T = (S.astype(np.float64) @ We.astype(np.float64).T).astype(np.float32)
+    pe = We.reshape(Cte, Cse // Cspe, Cspe).transpose(1, 0, 2)
+    ie = np.stack([pe[m][synth.sample_indices(Cte, Ke, 154, m)] for m in range(Cse // Cspe)])
+    D0, c0 = q.pq_quantize_fc(torch.from_numpy(We).to(dev), Cspe, Ke,
+                              torch.from_numpy(ie).to(dev), rounds)
+    St, Tt = torch.from_numpy(S).to(dev), torch.from_numpy(T).to(dev)
+    q.ec_quantize_fc(St, Tt, D0, c0, 1, 2)
+    t_ec = event_ms(lambda: q.ec_quantize_fc(St, Tt, D0, c0, 1, 2), 3, flush_each=False)
+    qres["ec_fc8_ms"] = round(t_ec, 2)
+    qres["ec_setup"] = "N=512 calibration vectors, 1 sweep over 1024 sub-spaces, 2 alternations"
+    if with_oracle:
+        import oracle
+        import oracle.ec as oec
+        _, L3, W3t, I3t, W3, I3 = next(t for t in jobs if t[0] == 4)   # conv3
+        t0 = time.perf_counter()
+        oracle.pq_quantize_conv(W3, L3.Csp, L3.K, I3, rounds)
+        qres["oracle_kmeans_conv3_s"] = round(time.perf_counter() - t0, 3)
+        t3 = event_ms(lambda: q.pq_quantize_conv(W3t, L3.Csp, L3.K, I3t, rounds), 3,
+                      flush_each=False)
+        qres["kmeans_conv3_ms"] = round(t3, 3)
+        t0 = time.perf_counter()
+        oec.ec_quantize_fc(S, T, D0.cpu().numpy(), c0.cpu().numpy(), 1, 2)
+        qres["oracle_ec_fc8_s"] = round(time.perf_counter() - t0, 3)
+    res["quantizer"] = qres
+    return res
+
+
+def _layer_costs(w, cm):
+    costs = []
+    for L, (sin, sout) in zip(w.layers, w.shapes()):
+        if isinstance(L, synth.Conv):
+            costs.append(cm.conv_cost(L.Cs, L.Ct, sin[1], sin[2], L.kh, L.kw, sout[1], sout[2],
+                                      L.Csp, L.K))
+        elif isinstance(L, synth.FC):
+            costs.append(cm.fc_cost(L.Cs, L.Ct, L.Csp, L.K))
+    return costs
+
+
 def main():
     a = parse()
     if a.impl == "reference":
@@ -340,21 +472,24 @@ def main():
     bufs = [torch.empty((N, *sout), dtype=torch.float32, device=dev) for (sin, sout) in shapes]
     lws = torch.empty(ws.numel(), dtype=torch.uint8, device=dev)
 
-    def stage_times(qlayers, lut):
+    def stage_times(qlayers, lut, xin=None, obufs=None):
+        xin = x if xin is None else xin
+        obufs = bufs if obufs is None else obufs
+        nb = xin.shape[0]
         stage_ms = [0.0] * len(qlayers)
         for it in range(a.steps + 2):
             flush.zero_()
             ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(qlayers) + 1)]
             ev[0].record(stream)
-            h = x
+            h = xin
             for j, qL in enumerate(qlayers):
-                o = bufs[j]
+                o = obufs[j]
                 if isinstance(qL, q.ConvLayer):
                     q.conv_forward(h, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias,
                                    qL.relu, packed=True, Ct=qL.Ct, out=o, workspace=lws, lut=lut)
                 elif isinstance(qL, q.FCLayer):
-                    q.fc_forward(h.reshape(N, -1), qL.D, qL.codes, qL.bias, qL.relu,
-                                 out=o.reshape(N, -1), workspace=lws, lut=lut)
+                    q.fc_forward(h.reshape(nb, -1), qL.D, qL.codes, qL.bias, qL.relu,
+                                 out=o.reshape(nb, -1), workspace=lws, lut=lut)
                 else:
                     q.maxpool(h, qL.k, qL.s, out=o)
                 ev[j + 1].record(stream)
@@ -464,6 +599,8 @@ def main():
         return res
 
     b1 = batch1(net)
+    bufs1 = [torch.empty((1, *sout), dtype=torch.float32, device=dev) for (sin, sout) in shapes]
+    b1["stage_ms"] = [round(t, 4) for t in stage_times(layers, "fp32", x1, bufs1)]
 
     # ---- bfloat16 tables: the same workload and timing, lut="bf16"
     bf_layers = make_layers("bf16")
@@ -489,6 +626,11 @@ def main():
                     "per look-up and per table entry; not the headline (fp32) number",
             "batch1": batch1(bf_net), "stages": bf_stages}
 
+    extras = {}
+    if not a.no_extras:
+        extras = extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N,
+                                    batch1, cm, rank == 0 and world == 1)
+
     cpu = None
     if pool is not None:
         sample = a.cpu_sample or cores
@@ -513,7 +655,7 @@ def main():
                    "codes": "packed once at model load (outside the timed region)"},
         "dense_equiv_gflops": round(2 * dense_macs * value / 1e9, 1),
         "batch1": b1,
-        "roofline": roofline, "stages": stages, "bf16_lut": bf16,
+        "roofline": roofline, "stages": stages, "bf16_lut": bf16, **extras,
         "cpu_baseline": cpu, "e2e": {k: (round(v, 1) if isinstance(v, float) else v)
                                      for k, v in e2e.items()},
         "gpu_launches": int(launches), "clocks": clk,

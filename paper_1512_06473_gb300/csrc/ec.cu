@@ -48,13 +48,14 @@ __global__ void ec_init_kernel(const float *__restrict__ S, const float *__restr
     }
 }
 
-// Vp[chunk][j][c_t] = sum_{n in chunk} A[n][j] E[n][c_t]; block (0, 0) also
-// writes G = A^T A.  grid (ceil(Ct / 256), ceil(N / kEcChunk)).
+// Vp[chunk][j][c_t] = sum_{n in chunk} A[n][j] E[n][c_t]; the blocks of the
+// first output tile also write the chunk's part of G = A^T A,
+// Gp[chunk][i][j].  grid (ceil(Ct / 256), ceil(N / kEcChunk)).
 __global__ void __launch_bounds__(256) ec_stats_kernel(const float *__restrict__ S, int N, int Cs,
                                                        int Ct, int Csp, int m,
                                                        const double *__restrict__ E,
                                                        double *__restrict__ Vp,
-                                                       double *__restrict__ G) {
+                                                       double *__restrict__ Gp) {
     __shared__ double a[kEcChunk][kMaxCsp];
     const int n0 = blockIdx.y * kEcChunk, nn = min(kEcChunk, N - n0);
     for (int e = threadIdx.x; e < kEcChunk * kMaxCsp; e += blockDim.x) {
@@ -67,6 +68,7 @@ __global__ void __launch_bounds__(256) ec_stats_kernel(const float *__restrict__
         double v[kMaxCsp];
 #pragma unroll
         for (int j = 0; j < kMaxCsp; ++j) v[j] = 0.0;
+#pragma unroll 8
         for (int r = 0; r < nn; ++r) {
             const double e = E[(size_t)(n0 + r) * Ct + ct];
 #pragma unroll
@@ -74,14 +76,22 @@ __global__ void __launch_bounds__(256) ec_stats_kernel(const float *__restrict__
         }
         for (int j = 0; j < Csp; ++j) Vp[((size_t)blockIdx.y * Csp + j) * Ct + ct] = v[j];
     }
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < Csp * Csp) {
+    if (blockIdx.x == 0 && threadIdx.x < Csp * Csp) {
         const int i = threadIdx.x / Csp, j = threadIdx.x % Csp;
         double g = 0.0;
-        for (int n = 0; n < N; ++n)
-            g = fma((double)S[(size_t)n * Cs + (size_t)m * Csp + i],
-                    (double)S[(size_t)n * Cs + (size_t)m * Csp + j], g);
-        G[i * Csp + j] = g;
+        for (int r = 0; r < nn; ++r) g = fma(a[r][i], a[r][j], g);
+        Gp[((size_t)blockIdx.y * Csp + i) * Csp + j] = g;
     }
+}
+
+// G = sum of the chunk parts, in chunk order (one thread per entry).
+__global__ void ec_gram_kernel(int Csp, int nchunks, const double *__restrict__ Gp,
+                               double *__restrict__ G) {
+    const int e = threadIdx.x;
+    if (e >= Csp * Csp) return;
+    double g = 0.0;
+    for (int c = 0; c < nchunks; ++c) g += Gp[(size_t)c * Csp * Csp + e];
+    G[e] = g;
 }
 
 // In-place Cholesky of the Csp x Csp matrix in L (lower triangle used);
@@ -137,22 +147,33 @@ __global__ void __launch_bounds__(256) ec_u_kernel(int N, int Ct, int Csp, int K
     }
 }
 
-// Eq. 11 for every k (one thread each), then q_k = D_k^T G D_k.
+// Eq. 11 for every k (one warp each: lanes take every 32nd member of L_k,
+// then a fixed butterfly adds the lanes), then q_k = D_k^T G D_k.
 __global__ void ec_codeword_kernel(int Ct, int Csp, int K, const double *__restrict__ U,
                                    const int *__restrict__ order, const int *__restrict__ starts,
                                    const double *__restrict__ G, const double *__restrict__ Lf,
                                    double *__restrict__ Dm, double *__restrict__ q) {
-    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    const int k = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
     if (k >= K) return;
     const int s0 = starts[k], s1 = starts[k + 1];
+    double part[kMaxCsp];
+#pragma unroll
+    for (int j = 0; j < kMaxCsp; ++j) part[j] = 0.0;
+    for (int e = s0 + lane; e < s1; e += 32) {
+        const int ct = order[e];
+#pragma unroll
+        for (int j = 0; j < kMaxCsp; ++j)
+            if (j < Csp) part[j] += U[(size_t)j * Ct + ct];
+    }
+#pragma unroll
+    for (int j = 0; j < kMaxCsp; ++j)
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
+    if (lane != 0) return;
     double *d = Dm + (size_t)k * Csp;
     if (s1 > s0) {
         double b[kMaxCsp];
-        for (int j = 0; j < Csp; ++j) {
-            double s = 0.0;
-            for (int e = s0; e < s1; ++e) s += U[(size_t)j * Ct + order[e]];
-            b[j] = s / (double)(s1 - s0);
-        }
+        for (int j = 0; j < Csp; ++j) b[j] = part[j] / (double)(s1 - s0);
         // L y = b, L^T d = y
         for (int i = 0; i < Csp; ++i) {
             double s = b[i];
@@ -234,7 +255,7 @@ __global__ void ec_widen_kernel(const float *__restrict__ in, double *__restrict
 }
 
 struct EcWs {
-    size_t E, Dw, Vp, U, G, Lf, Dold, kold, q, order, starts, flag, total;
+    size_t E, Dw, Vp, Gp, U, G, Lf, Dold, kold, q, order, starts, flag, total;
 };
 
 EcWs ec_ws_layout(int N, int Cs, int Ct, int Csp, int K) {
@@ -249,6 +270,7 @@ EcWs ec_ws_layout(int N, int Cs, int Ct, int Csp, int K) {
     w.E = take((size_t)N * Ct * sizeof(double));
     w.Dw = take((size_t)M * K * Csp * sizeof(double));
     w.Vp = take((size_t)nch * Csp * Ct * sizeof(double));
+    w.Gp = take((size_t)nch * Csp * Csp * sizeof(double));
     w.U = take((size_t)Csp * Ct * sizeof(double));
     w.G = take((size_t)Csp * Csp * sizeof(double));
     w.Lf = take((size_t)Csp * Csp * sizeof(double));
@@ -301,6 +323,7 @@ qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, i
     double *E = reinterpret_cast<double *>(b + L.E);
     double *Dw = reinterpret_cast<double *>(b + L.Dw);
     double *Vp = reinterpret_cast<double *>(b + L.Vp);
+    double *Gp = reinterpret_cast<double *>(b + L.Gp);
     double *U = reinterpret_cast<double *>(b + L.U);
     double *G = reinterpret_cast<double *>(b + L.G);
     double *Lf = reinterpret_cast<double *>(b + L.Lf);
@@ -325,7 +348,9 @@ qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, i
         for (int m = 0; m < M; ++m) {
             double *Dm = Dw + (size_t)m * K * Csp;
             uint8_t *cm = codes + (size_t)m * Ct;
-            ec_stats_kernel<<<sgrid, 256, 0, st>>>(S, N, Cs, Ct, Csp, m, E, Vp, G);
+            ec_stats_kernel<<<sgrid, 256, 0, st>>>(S, N, Cs, Ct, Csp, m, E, Vp, Gp);
+            if ((rc = after_launch()) != QCNN_OK) return rc;
+            ec_gram_kernel<<<1, 64, 0, st>>>(Csp, nch, Gp, G);
             if ((rc = after_launch()) != QCNN_OK) return rc;
             ec_u_kernel<<<cdiv(Ct, 256), 256, 0, st>>>(N, Ct, Csp, K, nch, Vp, G, Dm, cm, U, Dold,
                                                        kold, Lf, flag);
@@ -333,8 +358,8 @@ qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, i
             for (int i = 0; i < inner; ++i) {
                 kmeans_order_kernel<<<1, 1024, 0, st>>>(i == 0 ? kold : cm, Ct, K, order, starts);
                 if ((rc = after_launch()) != QCNN_OK) return rc;
-                ec_codeword_kernel<<<cdiv(K, 128), 128, 0, st>>>(Ct, Csp, K, U, order, starts, G,
-                                                                 Lf, Dm, q);
+                ec_codeword_kernel<<<cdiv(K * 32, 256), 256, 0, st>>>(Ct, Csp, K, U, order,
+                                                                      starts, G, Lf, Dm, q);
                 if ((rc = after_launch()) != QCNN_OK) return rc;
                 ec_assign_kernel<<<cdiv(Ct, 256), 256, 0, st>>>(Ct, Csp, K, U, Dm, q, cm);
                 if ((rc = after_launch()) != QCNN_OK) return rc;
