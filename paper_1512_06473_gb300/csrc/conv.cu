@@ -80,6 +80,13 @@ struct ConvFusedArgs {
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
     int splits, m_per_split;    // sub-space ranges over several CTAs (small batches)
     float *__restrict__ partial;  // [splits][N][Ct][Ho][Wo] when splits > 1
+    // stream-K schedule (large batches): CTA c takes the (tile, sub-space)
+    // units [u0, u1), u = tile * M + m, sk_base units each plus one for the
+    // first sk_extra CTAs; tile = (n * ct_tiles + ct_tile) * row_tiles + row.
+    // A tile cut at the end of CTA c's range leaves two partial pieces,
+    // partial[c][0] (sub-spaces before the cut) and partial[c][1] (after),
+    // each [CT_CTA][TH][Wo]
+    int sk, sk_base, sk_extra, row_tiles, ct_tiles;
 };
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
@@ -130,7 +137,8 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // PIPE  : two table buffers; sub-space m+1's table is built while m is
 //         gathered, with one barrier per sub-space instead of two
 // BF    : bfloat16 pair tables; a slot is then 64 positions (2 per lane)
-template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF>
+// SK    : stream-K schedule (a persistent grid over (tile, sub-space) units)
+template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF, bool SK>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
     constexpr int NT = NW * 32;
     constexpr int E = BF ? 2 : 1;  // positions per lane and slot
@@ -151,18 +159,33 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
-    const int oy0 = blockIdx.x * a.TH;
-    const int ct0 = blockIdx.y * CT_CTA;
-    const int n = blockIdx.z / a.splits, split = blockIdx.z % a.splits;
+    const int split = SK ? 0 : blockIdx.z % a.splits;
+    // tile being staged (sn, soy0, sct0) and tile being computed (cn, coy0, cct0)
+    int sn = blockIdx.z / a.splits, soy0 = blockIdx.x * a.TH, sct0 = blockIdx.y * CT_CTA;
     const int HW = a.H * a.W;
 
     // Halo position h -> offset iy*W + ix inside one input plane, or -1 where
     // the zero padding is; sub-vector slots j >= C'_s stay zero.
-    for (int h = tid; h < HP; h += NT) {
-        const int r = h / pitch, c = h - r * pitch;
-        const int iy = oy0 - a.pad + r, ix = c - a.pad;
-        hoff[h] = (iy >= 0 && iy < a.H && ix >= 0 && ix < a.W) ? iy * a.W + ix : -1;
+    auto make_hoff = [&]() {
+        for (int h = tid; h < HP; h += NT) {
+            const int r = h / pitch, c = h - r * pitch;
+            const int iy = soy0 - a.pad + r, ix = c - a.pad;
+            hoff[h] = (iy >= 0 && iy < a.H && ix >= 0 && ix < a.W) ? iy * a.W + ix : -1;
+        }
+    };
+    long long u = 0, u1 = 0;  // stream-K unit range
+    if constexpr (SK) {
+        const int c = blockIdx.x;
+        u = (long long)c * a.sk_base + min(c, a.sk_extra);
+        u1 = u + a.sk_base + (c < a.sk_extra ? 1 : 0);
+        const long long t = u / a.M;
+        sn = (int)(t / ((long long)a.ct_tiles * a.row_tiles));
+        const int rest = (int)(t - (long long)sn * a.ct_tiles * a.row_tiles);
+        sct0 = (rest / a.row_tiles) * CT_CTA;
+        soy0 = (rest % a.row_tiles) * a.TH;
     }
+    int cn = sn, coy0 = soy0, cct0 = sct0;
+    make_hoff();
     if (a.Csp < CSP4) {
         for (int e = tid; e < 2 * a.xs_floats; e += NT) xs[e] = 0.f;
         for (int e = tid; e < 2 * K * CSP4; e += NT) ds[e] = 0.f;
@@ -172,7 +195,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     // ---- asynchronous staging (callers commit) --------------------------
     auto stage_xd = [&](int m, int b) {  // inputs and sub-codebook of sub-space m
         float *xb = xs + b * a.xs_floats;
-        const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * HW;
+        const float *xn = a.x + ((size_t)sn * a.Cs + (size_t)m * a.Csp) * HW;
         for (int j = 0; j < a.Csp; ++j) {
             for (int h = tid; h < HP; h += NT) {
                 const int off = hoff[h];
@@ -186,7 +209,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     };
     auto stage_codes = [&](int m, int b) {
         uint8_t *cb = cs + (size_t)b * kk * CT_CTA;
-        const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
+        const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + sct0;
         for (int e = tid; e < kk * Q16; e += NT) {
             const int pk = e / Q16, q = e % Q16;
             cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
@@ -329,9 +352,92 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     };
 
+    // ---- epilogue: bias, ReLU, store; or raw partial sums (mode 1: split-M
+    // slice `split`; mode 2: stream-K piece `slot` of boundary `bnd`)
+    auto store = [&](int mode, int bnd, int slot) {
+#pragma unroll
+        for (int c = 0; c < CTW; ++c) {
+            const int ct = cct0 + wc * CTW + c;
+            if (ct >= a.Ct) continue;
+            const float bv = a.bias ? a.bias[ct] : 0.f;
+#pragma unroll
+            for (int p = 0; p < P * E; ++p) {
+                const int l = BF ? (wp * P + (p >> 1)) * 64 + 2 * lane + (p & 1)
+                                 : (wp * P + p) * 32 + lane;
+                const int r = l / pitch, col = l - r * pitch;
+                const int oy = coy0 + r;
+                if (r < a.TH && col < a.Wo && oy < a.Ho) {
+                    const size_t o = (((size_t)cn * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
+                    if (mode == 1) {
+                        a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
+                    } else if (mode == 2) {
+                        const size_t piece = (size_t)CT_CTA * a.TH * a.Wo;
+                        a.partial[((size_t)bnd * 2 + slot) * piece +
+                                  ((size_t)(wc * CTW + c) * a.TH + r) * a.Wo + col] = acc[c][p];
+                    } else {
+                        float v = acc[c][p] + bv;
+                        if (a.relu) v = fmaxf(v, 0.f);
+                        a.y[o] = v;
+                    }
+                }
+            }
+        }
+    };
+
     // sub-spaces [mb, me) of this CTA (all of them unless M is split)
     const int mb = split * a.m_per_split, me = min(a.M, mb + a.m_per_split);
-    if constexpr (!PIPE) {
+    if constexpr (SK) {
+        // ---- stream-K: units [u, u1) in order, u = tile * M + m; the first
+        // and last tile of the range may be cut (partial pieces)
+        int m = (int)(u % a.M);
+        int piece_m0 = m;  // first sub-space of the current piece
+        stage_xd(m, 0);
+        stage_codes(m, 0);
+        cp_async_commit();
+        for (int b = 0;; b ^= 1) {
+            cp_async_wait<0>();
+            __syncthreads();  // unit u staged; gather of the previous unit finished
+            const bool last_of_tile = m == a.M - 1, last_of_range = u + 1 == u1;
+            if (!last_of_range) {
+                if (last_of_tile) {  // the next unit opens a new tile: new halo table
+                    const long long t = (u + 1) / a.M;
+                    sn = (int)(t / ((long long)a.ct_tiles * a.row_tiles));
+                    const int rest = (int)(t - (long long)sn * a.ct_tiles * a.row_tiles);
+                    sct0 = (rest / a.row_tiles) * CT_CTA;
+                    soy0 = (rest % a.row_tiles) * a.TH;
+                    make_hoff();
+                    __syncthreads();
+                }
+                const int mn = last_of_tile ? 0 : m + 1;
+                stage_xd(mn, b ^ 1);
+                stage_codes(mn, b ^ 1);
+                cp_async_commit();
+            }
+            build(b, lut0);
+            __syncthreads();
+            gather(b, lut0);
+            if (last_of_tile || last_of_range) {
+                // whole tile -> y; head of a tile cut at the range end -> piece
+                // 0 of this CTA's boundary; tail of a cut tile -> piece 1 of
+                // the previous CTA's boundary
+                const bool whole = piece_m0 == 0 && last_of_tile;
+                store(whole ? 0 : 2, piece_m0 == 0 ? blockIdx.x : blockIdx.x - 1,
+                      piece_m0 == 0 ? 0 : 1);
+                if (last_of_range) break;
+#pragma unroll
+                for (int c = 0; c < CTW; ++c)
+#pragma unroll
+                    for (int p = 0; p < P * E; ++p) acc[c][p] = 0.f;
+                cn = sn;
+                coy0 = soy0;
+                cct0 = sct0;
+                piece_m0 = 0;
+            }
+            ++u;
+            m = last_of_tile ? 0 : m + 1;
+        }
+        return;
+    } else if constexpr (!PIPE) {
         stage_xd(mb, 0);
         stage_codes(mb, 0);
         cp_async_commit();
@@ -386,29 +492,33 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     }
 
-    // ---- epilogue: bias, ReLU, store (or raw partial sums of a split) -----
-#pragma unroll
-    for (int c = 0; c < CTW; ++c) {
-        const int ct = ct0 + wc * CTW + c;
-        if (ct >= a.Ct) continue;
-        const float bv = a.bias ? a.bias[ct] : 0.f;
-#pragma unroll
-        for (int p = 0; p < P * E; ++p) {
-            const int l = BF ? (wp * P + (p >> 1)) * 64 + 2 * lane + (p & 1)
-                             : (wp * P + p) * 32 + lane;
-            const int r = l / pitch, col = l - r * pitch;
-            const int oy = oy0 + r;
-            if (r < a.TH && col < a.Wo && oy < a.Ho) {
-                const size_t o = (((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
-                if (a.splits > 1) {
-                    a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
-                } else {
-                    float v = acc[c][p] + bv;
-                    if (a.relu) v = fmaxf(v, 0.f);
-                    a.y[o] = v;
-                }
-            }
-        }
+    if constexpr (!SK) store(a.splits > 1 ? 1 : 0, 0, 0);
+}
+
+// Stream-K fix-up: the tile cut at the end of CTA b's range gets
+// y = (sub-spaces before the cut) + (after) + bias, then ReLU.  One CTA per
+// boundary; boundaries that fall between tiles have nothing to do.
+__global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, int extra, int M,
+                                     int row_tiles, int ct_tiles, int TH, int ct_cta, int Ct,
+                                     int Ho, int Wo, const float *__restrict__ bias, int relu,
+                                     float *__restrict__ y) {
+    const int b = blockIdx.x;
+    const long long ub = (long long)(b + 1) * base + min(b + 1, extra);
+    if (ub % M == 0) return;
+    const long long t = ub / M;
+    const int n = (int)(t / ((long long)ct_tiles * row_tiles));
+    const int rest = (int)(t - (long long)n * ct_tiles * row_tiles);
+    const int ct0 = (rest / row_tiles) * ct_cta, oy0 = (rest % row_tiles) * TH;
+    const size_t piece = (size_t)ct_cta * TH * Wo;
+    const float *p0 = part + (size_t)b * 2 * piece, *p1 = p0 + piece;
+    for (int o = threadIdx.x; o < (int)piece; o += blockDim.x) {
+        const int col = o % Wo, r = (o / Wo) % TH, cl = o / (Wo * TH);
+        const int ct = ct0 + cl, oy = oy0 + r;
+        if (ct >= Ct || oy >= Ho) continue;
+        float v = p0[o] + p1[o];
+        if (bias) v += bias[ct];
+        if (relu) v = fmaxf(v, 0.f);
+        y[(((size_t)n * Ct + ct) * Ho + oy) * Wo + col] = v;
     }
 }
 
@@ -432,17 +542,20 @@ __global__ void conv_split_reduce_kernel(const float *__restrict__ partial, int 
 // (GB300, AlexNet conv2-5 and VGG-16 conv3-5 shapes, all lanes counted);
 // build: share of the table-build time left exposed (1 = not overlapped).
 struct FusedVariant {
-    int P, CTW, WP, CSP4, NW, MINB, PIPE, BF;
+    int P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK;
     double eff, build;
     void (*fn)(ConvFusedArgs);
 };
 
 #define QCNN_FUSED(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
-    {P, CTW, WP, C4, NW, MB, PIPE, 0, EFF, BLD,             \
-     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, false>}
+    {P, CTW, WP, C4, NW, MB, PIPE, 0, 0, EFF, BLD,          \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, false, false>}
 #define QCNN_FUSED_BF(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
-    {P, CTW, WP, C4, NW, MB, PIPE, 1, EFF, BLD,                \
-     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, true>}
+    {P, CTW, WP, C4, NW, MB, PIPE, 1, 0, EFF, BLD,             \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, PIPE, true, false>}
+#define QCNN_FUSED_SK(P, CTW, WP, C4, NW, MB, EFF, BLD) \
+    {P, CTW, WP, C4, NW, MB, 0, 0, 1, EFF, BLD,         \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, false, false, true>}
 #define QCNN_FUSED_SET(C4)                                                                       \
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
@@ -457,17 +570,24 @@ struct FusedVariant {
     QCNN_FUSED(4, 8, 1, C4, 16, 1, true, 0.8, 0.3)
 // bfloat16 tables: slots of 64 positions, so half the slots of the fp32
 // tiles cover the same band.  Measured (same shapes): the pair-table build
-// costs about 1.3x the fp32 build, the 32-warp and pipelined tiles never win.
+// costs about 1.3x the fp32 build; pipelined tiles never win (32-warp tiles,
+// slower still and short of registers, are not instantiated).
 #define QCNN_FUSED_BF_SET(C4)                                                      \
     QCNN_FUSED_BF(2, 8, 2, C4, 8, 2, false, 0.45, 1.3),                            \
     QCNN_FUSED_BF(4, 8, 1, C4, 16, 1, false, 1.0, 1.3),                            \
     QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, false, 0.97, 1.3),                          \
-    QCNN_FUSED_BF(2, 8, 1, C4, 32, 1, false, 0.75, 1.3),                           \
-    QCNN_FUSED_BF(4, 4, 1, C4, 32, 1, false, 0.7, 1.3),                            \
     QCNN_FUSED_BF(4, 8, 1, C4, 16, 1, true, 0.6, 0.4),                             \
     QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, true, 0.6, 0.4)
-static const FusedVariant kFused[] = {QCNN_FUSED_SET(4), QCNN_FUSED_SET(8),
-                                      QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8)};
+// stream-K schedules of the fp32 tiles that win on grids with a short last
+// wave (AlexNet's 13x13 layers); bf16 tables gained nothing from it
+#define QCNN_FUSED_SK_SET(C4)                      \
+    QCNN_FUSED_SK(4, 16, 1, C4, 16, 1, 1.0, 1.0),  \
+    QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0)
+static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
+                                      QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
+                                      QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};
+#undef QCNN_FUSED_SK_SET
+#undef QCNN_FUSED_SK
 #undef QCNN_FUSED_BF_SET
 #undef QCNN_FUSED_SET
 #undef QCNN_FUSED_BF
@@ -563,11 +683,43 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
             }
             if (ctas * sp >= 2.0 * sms * cps) break;
         }
+        // Large batches: a stream-K schedule gives every one of the G CTA
+        // slots the same number of (tile, sub-space) units, instead of whole
+        // tiles in ceil(ctas / G) waves; a tile cut between two CTAs costs a
+        // partial-sum round trip and a fix-up launch.
+        const int G = sms * cps;
+        int sk = 0;
+        double sk_units = 0;
+        bool allow_sk = true;
+#ifdef QCNN_TUNING
+        allow_sk = getenv("QCNN_NO_SK") == nullptr;
+#endif
+        // Measured on the AlexNet and VGG shapes: a stream-K unit costs 5-10%
+        // more than a plain one (tile hand-overs, cut tiles), and 20% more
+        // with the build-heavy bf16 tables; it pays only when the last wave
+        // of the plain grid is well short of full.
+        const double wave_fill = ctas / (std::ceil(ctas / G) * G);
+        if (fv.SK) {
+            if (!allow_sk || ctas < G || wave_fill >= 0.9) continue;
+            sk_units = std::ceil(ctas * s.M / G);
+            const double part = 2.0 * 2.0 * (G - 1) * ct_cta * TH * s.Wo * 4.0;
+            score = sk_units * per_m * cps * 1.05 + part / 3000.0 + 6000.0;
+            sk = 1;
+            splits = 1;
+        }
         if (!best.ok || score < best.score) {
             best.splits = splits;
             best.m_per_split = cdiv(s.M, splits);
             best.partial_bytes =
                 splits > 1 ? (size_t)splits * s.N * s.Ct * s.Ho * s.Wo * sizeof(float) : 0;
+            best.sk = sk;
+            if (sk) {
+                const long long units = (long long)s.N * row_tiles * ct_tiles * s.M;
+                best.sk_ctas = G;
+                best.sk_base = (int)(units / G);
+                best.sk_extra = (int)(units % G);
+                best.partial_bytes = (size_t)(G - 1) * 2 * ct_cta * TH * s.Wo * sizeof(float);
+            }
             best.ok = true;
             best.variant = v;
             best.P = fv.P;
@@ -587,9 +739,11 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
 #ifdef QCNN_TUNING
     if (best.ok && getenv("QCNN_PLAN_VERBOSE"))
         fprintf(stderr,
-                "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d pipe=%d TH=%d KS=%d ct_cta=%d smem=%zu\n",
+                "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d pipe=%d TH=%d KS=%d ct_cta=%d smem=%zu "
+                "splits=%d sk=%d sk_ctas=%d base=%d extra=%d\n",
                 best.variant, best.P, best.CTW, best.WP, kFused[best.variant].NW,
-                kFused[best.variant].PIPE, best.TH, best.KS, best.ct_cta, best.smem);
+                kFused[best.variant].PIPE, best.TH, best.KS, best.ct_cta, best.smem, best.splits,
+                best.sk, best.sk_ctas, best.sk_base, best.sk_extra);
 #endif
     return best;
 }
@@ -627,13 +781,27 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.splits = p.splits;
     a.m_per_split = p.m_per_split;
     a.partial = partial_ws;
+    a.sk = p.sk;
+    a.sk_base = p.sk_base;
+    a.sk_extra = p.sk_extra;
+    a.row_tiles = p.row_tiles;
+    a.ct_tiles = p.ct_tiles;
     cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
-    dim3 grid(p.row_tiles, p.ct_tiles, s.N * p.splits);
+    const dim3 grid = p.sk ? dim3(p.sk_ctas, 1, 1) : dim3(p.row_tiles, p.ct_tiles, s.N * p.splits);
     fv.fn<<<grid, fv.NW * 32, p.smem, st>>>(a);
     qcnn_status rc = after_launch();
-    if (rc != QCNN_OK || p.splits == 1) return rc;
+    if (rc != QCNN_OK) return rc;
+    if (p.sk) {
+        if (p.sk_ctas < 2) return QCNN_OK;
+        conv_sk_fixup_kernel<<<p.sk_ctas - 1, 256, 0, st>>>(partial_ws, p.sk_base, p.sk_extra, s.M,
+                                                           p.row_tiles, p.ct_tiles, p.TH,
+                                                           p.ct_cta, s.Ct, s.Ho, s.Wo, bias, relu,
+                                                           y);
+        return after_launch();
+    }
+    if (p.splits == 1) return rc;
     const size_t total = (size_t)s.N * s.Ct * s.Ho * s.Wo;
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
     conv_split_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, total, s.Ct,

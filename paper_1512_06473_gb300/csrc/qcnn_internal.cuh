@@ -46,7 +46,10 @@ struct ConvFusedPlan {
     int row_tiles, ct_tiles;
     int splits = 1;     // CTAs sharing one tile's sub-spaces (small batches)
     int m_per_split;
-    size_t partial_bytes = 0;  // workspace for split partial sums
+    int sk = 0;         // stream-K schedule (large batches): sk_ctas persistent
+    int sk_ctas = 0;    // CTAs over the (tile, sub-space) units, sk_base each
+    int sk_base = 0, sk_extra = 0;  // (+1 for the first sk_extra)
+    size_t partial_bytes = 0;  // workspace for split or stream-K partial sums
     size_t smem;        // dynamic shared memory bytes
     double score;       // estimated cost (lower is better)
 };

@@ -319,3 +319,16 @@ def test_benchmark_layers_bf16(name):
         e_model = rel(model.reshape(ref.shape), ref)
         e_got = rel(host(got).reshape(ref.shape), ref)
         assert e_model <= 3e-3 and e_got <= 1.25 * e_model + 1e-4, (name, i, e_got, e_model)
+
+
+@pytest.mark.parametrize("case", [(64, 64, 13, 13, 384, 3, 3, 1, 1, 4, 128),
+                                  (40, 32, 27, 27, 256, 5, 5, 1, 2, 4, 64)],
+                         ids=lambda c: "x".join(map(str, c)))
+def test_conv_bf16_stream_k(case):
+    """bf16 tables under the stream-K schedule (more tiles than CTA slots)."""
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(33, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    exact, model, emax, S = _conv_refs(x, D, codes, kh, kw, s, p, b)
+    got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), lut="bf16"))
+    check_model(got, model, emax)
+    check_exact(got, exact, S)

@@ -289,3 +289,26 @@ def test_launch_counter_counts_kernels():
     q.fc_forward(x, D, c)
     torch.cuda.synchronize()
     assert q.launch_count() > before
+
+
+# Large batches run a stream-K schedule: persistent CTAs take equal runs of
+# (tile, sub-space) units, tiles cut between two CTAs are summed by a fix-up
+# kernel.  These shapes have more tiles than CTA slots, so they take it.
+STREAM_K = [
+    (64, 64, 13, 13, 384, 3, 3, 1, 1, 4, 128),   # AlexNet conv3-like, M = 16
+    (24, 32, 27, 27, 256, 5, 5, 1, 2, 4, 64),    # conv2-like bands, M = 8
+    (160, 16, 13, 13, 256, 3, 3, 1, 1, 8, 32),   # M = 2: one-unit pieces
+]
+
+
+@pytest.mark.parametrize("case", STREAM_K, ids=lambda c: "x".join(map(str, c)))
+def test_conv_stream_k(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(31, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), relu=True))
+    assert rel(got, ref) <= TOL
+    xi, Di, ci, bi = conv_case(32, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=True)
+    refi = oracle.conv_forward(xi, Di, ci, kh, kw, s, p, bi)
+    goti = host(q.conv_forward(cuda(xi), cuda(Di), cuda(ci), kh, kw, s, p, cuda(bi)))
+    assert np.array_equal(goti.astype(np.float64), refi)
