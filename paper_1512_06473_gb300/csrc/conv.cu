@@ -802,10 +802,15 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
         return after_launch();
     }
     if (p.splits == 1) return rc;
-    const size_t total = (size_t)s.N * s.Ct * s.Ho * s.Wo;
+    return launch_split_reduce(partial_ws, p.splits, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
+                               s.Ho * s.Wo, bias, relu, y, st);
+}
+
+qcnn_status launch_split_reduce(const float *partial, int splits, size_t total, int Ct, int HoWo,
+                                const float *bias, int relu, float *y, cudaStream_t st) {
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
-    conv_split_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, total, s.Ct,
-                                                     s.Ho * s.Wo, bias, relu, y);
+    conv_split_reduce_kernel<<<blocks, 256, 0, st>>>(partial, splits, total, Ct, HoWo, bias, relu,
+                                                     y);
     return after_launch();
 }
 

@@ -306,6 +306,27 @@ __global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, 
     }
 }
 
+// Few outputs, many splits (batch 1): one warp per output; lane l adds the
+// splits l, l + 32, ... in order, then a fixed butterfly adds the lanes.
+__global__ void fc_reduce_warp_kernel(const float *__restrict__ partial, int splits, int N,
+                                      int Ct, const float *__restrict__ bias, int relu,
+                                      float *__restrict__ y) {
+    const size_t total = (size_t)N * Ct;
+    const int lane = threadIdx.x & 31;
+    for (size_t i = ((size_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < total;
+         i += ((size_t)gridDim.x * blockDim.x) >> 5) {
+        float v = 0.f;
+        for (int s = lane; s < splits; s += 32) v += partial[(size_t)s * total + i];
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) {
+            if (bias) v += bias[i % Ct];
+            if (relu) v = fmaxf(v, 0.f);
+            y[i] = v;
+        }
+    }
+}
+
 // eff: measured gather throughput relative to the best variant (GB300,
 // AlexNet fc6-fc8 at batch 128).
 struct FcVariant {
@@ -438,7 +459,13 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     if (rc != QCNN_OK || p.splits == 1) return rc;
     const size_t total = (size_t)s.N * s.Ct;
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
-    fc_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu, y);
+    if (total < 65536 && p.splits >= 16) {
+        const int wblocks = (int)std::min<size_t>((total * 32 + 255) / 256, (size_t)num_sms() * 16);
+        fc_reduce_warp_kernel<<<wblocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu,
+                                                       y);
+    } else {
+        fc_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu, y);
+    }
     return after_launch();
 }
 

@@ -82,6 +82,9 @@ int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
 
 qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K,
                               uint8_t *packed, cudaStream_t st);
+// y = bias + sum of `splits` partial sums [splits][total] (fixed order), then ReLU
+qcnn_status launch_split_reduce(const float *partial, int splits, size_t total, int Ct, int HoWo,
+                                const float *bias, int relu, float *y, cudaStream_t st);
 // partial_ws: p.partial_bytes of workspace (unused when p.splits == 1)
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p,
                               const float *x, const float *D,
