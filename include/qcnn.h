@@ -313,6 +313,36 @@ qcnn_status qcnn_pq_quantize(int kind, const float *W, int Ct, int Cs, int kh, i
  */
 qcnn_status qcnn_ec_quantize_fc_workspace_size(int N, int Cs, int Ct, int Csp, int K,
                                                size_t *bytes);
+
+/*
+ * qcnn_ec_quantize_conv -- quantization with error correction of a conv
+ * layer (Sec. 3.3.2, Appendix B): minimises
+ *     sum_{n,p_t} || sum_{(p_k,p_s)} sum_m (D^(m) B_pk^(m))^T S_{n,p_s}^(m) - T_{n,p_t} ||^2
+ * by block coordinate descent over the sub-spaces m = 0..M-1, `outer`
+ * sweeps, `inner` alternations per sub-space, each
+ *   - a pass over the codewords k = 0..K-1 in order: D_k becomes the
+ *     least-squares fit (Eq. B.6) of what the other codewords leave, in the
+ *     sum of the input sub-vectors at the offsets assigned to k; a codeword
+ *     assigned nowhere keeps its value;
+ *   - a pass over the kernel offsets p_k = 0..kh*kw-1 in order: every
+ *     channel's code at p_k becomes the best single codeword for what the
+ *     other offsets leave (Eq. B.8), ties to the smallest index.
+ * Arithmetic in double; zero padding as in qcnn_conv_forward.
+ *   S [N][Cs][H][W] fp32 (layer input), T [N][Ct][Ho][Wo] fp32 (response of
+ *     the original layer before its bias); device
+ *   D [M][K][Csp] fp32, codes [Ct][kh*kw][M] uint8: the starting point on
+ *     entry (codes >= K are clamped), the result on return
+ * Synchronizes `stream` before returning.  Returns QCNN_ERR_DATA when a
+ * least-squares problem or some G is singular; D and codes are then
+ * unspecified.
+ */
+qcnn_status qcnn_ec_quantize_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh,
+                                                 int kw, int stride, int pad, int Csp, int K,
+                                                 size_t *bytes);
+qcnn_status qcnn_ec_quantize_conv(const float *S, const float *T, int N, int Cs, int H, int W,
+                                  int Ct, int kh, int kw, int stride, int pad, int Csp, int K,
+                                  float *D, uint8_t *codes, int outer, int inner, void *workspace,
+                                  size_t workspace_bytes, void *stream);
 qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, int Ct,
                                 int Csp, int K, float *D, uint8_t *codes, int outer,
                                 int inner, void *workspace, size_t workspace_bytes,

@@ -25,7 +25,7 @@ from . import _lib
 from ._lib import QcnnError, load  # noqa: F401
 
 __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
-           "kmeans", "pq_quantize_fc", "pq_quantize_conv", "ec_quantize_fc",
+           "kmeans", "pq_quantize_fc", "pq_quantize_conv", "ec_quantize_fc", "ec_quantize_conv",
            "code_bits", "pack_bits", "unpack_bits", "fc_pack_codes", "serialize_model",
            "model_info", "load_model",
            "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
@@ -302,6 +302,30 @@ def ec_quantize_fc(S, T, D, codes, outer, inner, stream=None):
     _lib.check(lib.qcnn_ec_quantize_fc(_ptr(S), _ptr(T), N, Cs, Ct, Csp, K, _ptr(D2), _ptr(c2),
                                        int(outer), int(inner), _ptr(ws), wsb, _stream(stream)),
                "qcnn_ec_quantize_fc")
+    return D2, c2
+
+
+def ec_quantize_conv(S, T, D, codes, kh, kw, stride, pad, outer, inner, stream=None):
+    """Error-corrected conv quantization (Appendix B) from (D [M, K, Csp],
+    codes [Ct, kh*kw, M]) on calibration maps S [N, Cs, H, W] and pre-bias
+    responses T [N, Ct, Ho, Wo].  Returns new (D, codes)."""
+    _need(S, "S", torch.float32, 4)
+    _need(T, "T", torch.float32, 4)
+    _need(D, "D", torch.float32, 3)
+    _need(codes, "codes", torch.uint8, 3)
+    N, Cs, H, W = S.shape
+    Ct = T.shape[1]
+    M, K, Csp = D.shape
+    lib = load()
+    nb = ctypes.c_size_t()
+    _lib.check(lib.qcnn_ec_quantize_conv_workspace_size(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp,
+                                                        K, ctypes.byref(nb)),
+               "qcnn_ec_quantize_conv_workspace_size")
+    ws, wsb = _workspace(nb.value, S.device, None)
+    D2, c2 = D.clone(), codes.clone()
+    _lib.check(lib.qcnn_ec_quantize_conv(_ptr(S), _ptr(T), N, Cs, H, W, Ct, kh, kw, stride, pad,
+                                         Csp, K, _ptr(D2), _ptr(c2), int(outer), int(inner),
+                                         _ptr(ws), wsb, _stream(stream)), "qcnn_ec_quantize_conv")
     return D2, c2
 
 

@@ -83,6 +83,9 @@ _SIGS = {
                             c_void_p, c_void_p, c_size_t, c_void_p]),
     "qcnn_pq_quantize_workspace_size": (c_int, [c_int] * 7 + [ctypes.POINTER(c_size_t)]),
     "qcnn_ec_quantize_fc_workspace_size": (c_int, [c_int] * 5 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_ec_quantize_conv_workspace_size": (c_int, [c_int] * 11 + [ctypes.POINTER(c_size_t)]),
+    "qcnn_ec_quantize_conv": (c_int, [c_void_p, c_void_p] + [c_int] * 11 +
+                              [c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t, c_void_p]),
     "qcnn_ec_quantize_fc": (c_int, [c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_int,
                                     c_void_p, c_void_p, c_int, c_int, c_void_p, c_size_t,
                                     c_void_p]),
