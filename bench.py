@@ -349,6 +349,27 @@ def extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N, ba
     t_ec = event_ms(lambda: q.ec_quantize_fc(St, Tt, D0, c0, 1, 2), 3, flush_each=False)
     qres["ec_fc8_ms"] = round(t_ec, 2)
     qres["ec_setup"] = "N=512 calibration vectors, 1 sweep over 1024 sub-spaces, 2 alternations"
+    # error correction of a conv layer (Appendix B), AlexNet conv3 shape with 8
+    # calibration images, from the k-means start
+    j3, L3, W3t, I3t, W3, I3 = next(t for t in jobs if t[0] == 4)
+    Sc = synth.relu_normal((8, L3.Cs, 13, 13), 155)
+    Tc = torch.nn.functional.conv2d(torch.from_numpy(Sc).double(), torch.from_numpy(W3).double(),
+                                    padding=L3.pad).float()
+    Dc0, cc0 = q.pq_quantize_conv(W3t, L3.Csp, L3.K, I3t, rounds)
+    Sct, Tct = torch.from_numpy(Sc).to(dev), Tc.to(dev)
+    Dc1, cc1 = q.ec_quantize_conv(Sct, Tct, Dc0, cc0, L3.kh, L3.kw, 1, L3.pad, 1, 1)
+    t_ecc = event_ms(lambda: q.ec_quantize_conv(Sct, Tct, Dc0, cc0, L3.kh, L3.kw, 1, L3.pad, 1, 1),
+                     2, flush_each=False)
+    qres["ec_conv3_ms"] = round(t_ecc, 1)
+
+    def rel_err(Dq, cq):
+        yq = q.conv_forward(Sct, Dq, cq, L3.kh, L3.kw, 1, L3.pad)
+        return float(((yq.double() - Tct.double()) ** 2).sum() / (Tct.double() ** 2).sum())
+
+    qres["ec_conv3_rel_sq_err"] = {"kmeans": round(rel_err(Dc0, cc0), 5),
+                                   "error_corrected": round(rel_err(Dc1, cc1), 5)}
+    qres["ec_conv3_setup"] = ("8 calibration images 256x13x13 -> 384, C's 4, K 128: one sweep over "
+                              "64 sub-spaces, one alternation (128 codeword steps, 9 offset steps)")
     if with_oracle:
         import oracle
         import oracle.ec as oec
