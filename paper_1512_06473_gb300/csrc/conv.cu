@@ -6,8 +6,13 @@
 //  * conv_fused (stride 1): one CTA owns an image, a band of TH output rows
 //    (all columns) and CT_CTA output channels.  For each sub-space m it
 //    builds the table of every halo position of the band in shared memory
-//    -- layout lut[k][h], h = linear index in the zero-padded halo grid of
-//    row pitch W + 2 pad -- and then gathers from it.  Lanes of a warp take
+//    -- layout lut[k][h], h = linear index in the zero-padded halo grid --
+//    and then gathers from it.  The grid's row pitch is max(W + pad, Wo):
+//    input column ix sits at column ix + pad, and a read past the end of a
+//    row runs on, in linear order, into the next row's `pad` leading zero
+//    columns, so the right padding of one row and the left padding of the
+//    next share one gap (W + pad columns instead of W + 2 pad; fewer lanes
+//    on discarded positions).  Lanes of a warp take
 //    consecutive positions of that padded grid, so for one (c_t, p_k) the
 //    whole warp shares one code k and reads 32 consecutive words of row k:
 //    bank-conflict free, and the kernel offset (ky, kx) is a plain shift
@@ -560,6 +565,7 @@ struct FusedVariant {
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
     QCNN_FUSED(7, 8, 1, C4, 16, 1, false, 1.0, 1.0),                                             \
+    QCNN_FUSED(6, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* a 13-row band of pitch 14 */            \
     QCNN_FUSED(4, 8, 1, C4, 16, 2, false, 0.83, 1.0), /* 2 x 16 warps, 64 registers */          \
     QCNN_FUSED(8, 4, 1, C4, 32, 1, false, 0.82, 1.0), /* 32 warps, 64 registers */              \
     QCNN_FUSED(7, 4, 1, C4, 32, 1, false, 0.89, 1.0),                                            \
@@ -582,7 +588,8 @@ struct FusedVariant {
 // wave (AlexNet's 13x13 layers); bf16 tables gained nothing from it
 #define QCNN_FUSED_SK_SET(C4)                      \
     QCNN_FUSED_SK(4, 16, 1, C4, 16, 1, 1.0, 1.0),  \
-    QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0)
+    QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0),   \
+    QCNN_FUSED_SK(6, 8, 1, C4, 16, 1, 1.0, 1.0)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
                                       QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
                                       QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};
@@ -604,7 +611,10 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
     ConvFusedPlan best;
     if (s.stride != 1 || s.Csp > kMaxCsp) return best;
     const int csp4 = s.Csp <= 4 ? 4 : 8;
-    const int pitch = s.W + 2 * s.pad;
+    // Row pitch of the halo grid: >= W + pad, so that every read past a
+    // row's data lands on zeros (this row's tail or the next row's `pad`
+    // leading columns), and >= Wo, so that a row of outputs fits in a row.
+    const int pitch = std::max(s.W + s.pad, s.Wo);
     const int kk = s.kh * s.kw;
     const int sms = num_sms();
     int dev = 0;
@@ -639,7 +649,9 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         if (TH < 1) continue;
         const int row_tiles = cdiv(s.Ho, TH);
         TH = cdiv(s.Ho, row_tiles);  // balance the bands
-        const int HP = (TH + s.kh - 1) * pitch;
+        // halo positions up to the last one a valid output reads: row
+        // TH + kh - 2, column Wo - 1 + kw - 1 = W + 2 pad - 1
+        const int HP = (TH + s.kh - 2) * pitch + s.W + 2 * s.pad;
         const int reach = (s.kh - 1) * pitch + (s.kw - 1);  // largest kernel offset
         // fp32: KS floats per row, >= every position read; bf16: two copies
         // of RW words per row, RW > every pair word read or written
@@ -649,7 +661,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
             if ((HP - 1) / 2 >= RW) continue;
             KS = 2 * RW;
         } else {
-            KS = ks_for(slots * 32 + reach);
+            KS = ks_for(std::max(slots * 32 + reach, HP));
         }
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;

@@ -38,10 +38,10 @@ struct ConvFusedPlan {
     int variant = -1;   // index into the instantiated kernel table
     int P, CTW, WP;     // slots per warp, channels per warp, warps on positions
     int TH;             // output rows per CTA
-    int pitch;          // W + 2 pad
+    int pitch;          // halo row pitch, max(W + pad, Wo)
     int KS;             // 32-bit words per table row (per sub-codeword; bf16:
                         // both copies, 2 x an odd word count)
-    int HP;             // halo positions with data: (TH + kh - 1) * pitch
+    int HP;             // halo positions built: (TH + kh - 2) * pitch + W + 2 pad
     int ct_cta;         // channels per CTA
     int row_tiles, ct_tiles;
     int splits = 1;     // CTAs sharing one tile's sub-spaces (small batches)
