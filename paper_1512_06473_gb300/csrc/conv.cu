@@ -3,21 +3,23 @@
 //   LUT_n[m][p_s][k] = <x_n^(m)(p_s), D^(m)_k>,  p_s = (oy*s - pad + ky, ox*s - pad + kx)
 //
 // Two kernels compute it:
-//  * conv_fused (stride 1): one CTA owns an image, a band of TH output rows
-//    (all columns) and CT_CTA output channels.  For each sub-space m it
-//    builds the table of every halo position of the band in shared memory
-//    -- layout lut[k][h], h = linear index in the zero-padded halo grid --
-//    and then gathers from it.  The grid's row pitch is max(W + pad, Wo):
-//    input column ix sits at column ix + pad, and a read past the end of a
-//    row runs on, in linear order, into the next row's `pad` leading zero
-//    columns, so the right padding of one row and the left padding of the
-//    next share one gap (W + pad columns instead of W + 2 pad; fewer lanes
-//    on discarded positions).  Lanes of a warp take
-//    consecutive positions of that padded grid, so for one (c_t, p_k) the
+//  * conv_fused (stride 1): outputs live on a padded grid of row pitch
+//    max(W + pad, Wo), output (oy, ox) at linear position l = oy*pitch + ox;
+//    the halo grid has the same pitch, input (iy, ix) at (iy + pad)*pitch +
+//    ix + pad, so output l reads halo position l + ky*pitch + kx at kernel
+//    offset (ky, kx).  A read past the end of a row runs on, in linear
+//    order, into the next row's `pad` leading zero columns: the right
+//    padding of one row and the left padding of the next share one gap.
+//    One CTA owns an image, a run of ST consecutive output positions (a
+//    tile; it need not start or end on a row) and CT_CTA output channels.
+//    For each sub-space m it builds, in shared memory, the table of the
+//    ST + reach halo positions its outputs read -- layout lut[k][h], h
+//    relative to the tile's first position -- and then gathers from it.
+//    Lanes of a warp take consecutive positions, so for one (c_t, p_k) the
 //    whole warp shares one code k and reads 32 consecutive words of row k:
-//    bank-conflict free, and the kernel offset (ky, kx) is a plain shift
-//    ky*pitch + kx of the read address.  Lanes that fall on the padding
-//    columns compute values that are discarded.
+//    bank-conflict free, and the kernel offset is a plain shift of the read
+//    address.  Lanes on padding columns (or past the last output) compute
+//    values that are discarded.
 //    bfloat16 tables (BF): every 32-bit word holds the entries of two
 //    neighbouring positions, (h, h+1), so one load serves two look-ups.  A
 //    kernel offset can be odd, so the table is kept twice: copy 0 holds the
@@ -81,17 +83,17 @@ struct ConvFusedArgs {
     const float *__restrict__ bias;
     float *__restrict__ y;
     int N, Cs, H, W, Ct, kh, kw, pad, Csp, K, M, Ho, Wo;
-    int pitch, TH, KS, HP, CtP, relu;
+    int pitch, ST, KS, HP, CtP, relu;  // ST: output positions per tile
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
     int splits, m_per_split;    // sub-space ranges over several CTAs (small batches)
     float *__restrict__ partial;  // [splits][N][Ct][Ho][Wo] when splits > 1
     // stream-K schedule (large batches): CTA c takes the (tile, sub-space)
     // units [u0, u1), u = tile * M + m, sk_base units each plus one for the
-    // first sk_extra CTAs; tile = (n * ct_tiles + ct_tile) * row_tiles + row.
+    // first sk_extra CTAs; tile = (n * ct_tiles + ct_tile) * pos_tiles + pos.
     // A tile cut at the end of CTA c's range leaves two partial pieces,
     // partial[c][0] (sub-spaces before the cut) and partial[c][1] (after),
-    // each [CT_CTA][TH][Wo]
-    int sk, sk_base, sk_extra, row_tiles, ct_tiles;
+    // each [CT_CTA][ST] over the tile's positions
+    int sk, sk_base, sk_extra, pos_tiles, ct_tiles;
 };
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
@@ -149,6 +151,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     constexpr int CT_CTA = (NW / WP) * CTW;
     constexpr int Q16 = CT_CTA / 16;
+    constexpr int ST = WP * P * 32 * E;  // output positions per tile
     // sub-codewords per lane per build pass (fewer under a 64-register budget)
     constexpr int QB = (NW * MINB >= 32 ? 8 : 16) / CSP4;
     static_assert(CT_CTA % 16 == 0, "channel tile must be a multiple of 16");
@@ -165,16 +168,18 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
     const int split = SK ? 0 : blockIdx.z % a.splits;
-    // tile being staged (sn, soy0, sct0) and tile being computed (cn, coy0, cct0)
-    int sn = blockIdx.z / a.splits, soy0 = blockIdx.x * a.TH, sct0 = blockIdx.y * CT_CTA;
+    // tile being staged (sn, sl0, sct0) and tile being computed (cn, cl0, cct0):
+    // image, first output position, first channel
+    int sn = blockIdx.z / a.splits, sl0 = blockIdx.x * ST, sct0 = blockIdx.y * CT_CTA;
     const int HW = a.H * a.W;
 
-    // Halo position h -> offset iy*W + ix inside one input plane, or -1 where
-    // the zero padding is; sub-vector slots j >= C'_s stay zero.
+    // Halo position h of the tile -> offset iy*W + ix inside one input
+    // plane, or -1 where the zero padding is; sub-vector slots j >= C'_s
+    // stay zero.
     auto make_hoff = [&]() {
         for (int h = tid; h < HP; h += NT) {
-            const int r = h / pitch, c = h - r * pitch;
-            const int iy = soy0 - a.pad + r, ix = c - a.pad;
+            const int g = sl0 + h, r = g / pitch, c = g - r * pitch;
+            const int iy = r - a.pad, ix = c - a.pad;
             hoff[h] = (iy >= 0 && iy < a.H && ix >= 0 && ix < a.W) ? iy * a.W + ix : -1;
         }
     };
@@ -184,12 +189,12 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         u = (long long)c * a.sk_base + min(c, a.sk_extra);
         u1 = u + a.sk_base + (c < a.sk_extra ? 1 : 0);
         const long long t = u / a.M;
-        sn = (int)(t / ((long long)a.ct_tiles * a.row_tiles));
-        const int rest = (int)(t - (long long)sn * a.ct_tiles * a.row_tiles);
-        sct0 = (rest / a.row_tiles) * CT_CTA;
-        soy0 = (rest % a.row_tiles) * a.TH;
+        sn = (int)(t / ((long long)a.ct_tiles * a.pos_tiles));
+        const int rest = (int)(t - (long long)sn * a.ct_tiles * a.pos_tiles);
+        sct0 = (rest / a.pos_tiles) * CT_CTA;
+        sl0 = (rest % a.pos_tiles) * ST;
     }
-    int cn = sn, coy0 = soy0, cct0 = sct0;
+    int cn = sn, cl0 = sl0, cct0 = sct0;
     make_hoff();
     if (a.Csp < CSP4) {
         for (int e = tid; e < 2 * a.xs_floats; e += NT) xs[e] = 0.f;
@@ -369,16 +374,15 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             for (int p = 0; p < P * E; ++p) {
                 const int l = BF ? (wp * P + (p >> 1)) * 64 + 2 * lane + (p & 1)
                                  : (wp * P + p) * 32 + lane;
-                const int r = l / pitch, col = l - r * pitch;
-                const int oy = coy0 + r;
-                if (r < a.TH && col < a.Wo && oy < a.Ho) {
+                const int g = cl0 + l, oy = g / pitch, col = g - oy * pitch;
+                if (col < a.Wo && oy < a.Ho) {
                     const size_t o = (((size_t)cn * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
                     if (mode == 1) {
                         a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
                     } else if (mode == 2) {
-                        const size_t piece = (size_t)CT_CTA * a.TH * a.Wo;
+                        const size_t piece = (size_t)CT_CTA * ST;
                         a.partial[((size_t)bnd * 2 + slot) * piece +
-                                  ((size_t)(wc * CTW + c) * a.TH + r) * a.Wo + col] = acc[c][p];
+                                  (size_t)(wc * CTW + c) * ST + l] = acc[c][p];
                     } else {
                         float v = acc[c][p] + bv;
                         if (a.relu) v = fmaxf(v, 0.f);
@@ -406,10 +410,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             if (!last_of_range) {
                 if (last_of_tile) {  // the next unit opens a new tile: new halo table
                     const long long t = (u + 1) / a.M;
-                    sn = (int)(t / ((long long)a.ct_tiles * a.row_tiles));
-                    const int rest = (int)(t - (long long)sn * a.ct_tiles * a.row_tiles);
-                    sct0 = (rest / a.row_tiles) * CT_CTA;
-                    soy0 = (rest % a.row_tiles) * a.TH;
+                    sn = (int)(t / ((long long)a.ct_tiles * a.pos_tiles));
+                    const int rest = (int)(t - (long long)sn * a.ct_tiles * a.pos_tiles);
+                    sct0 = (rest / a.pos_tiles) * CT_CTA;
+                    sl0 = (rest % a.pos_tiles) * ST;
                     make_hoff();
                     __syncthreads();
                 }
@@ -434,7 +438,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 #pragma unroll
                     for (int p = 0; p < P * E; ++p) acc[c][p] = 0.f;
                 cn = sn;
-                coy0 = soy0;
+                cl0 = sl0;
                 cct0 = sct0;
                 piece_m0 = 0;
             }
@@ -504,22 +508,22 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 // y = (sub-spaces before the cut) + (after) + bias, then ReLU.  One CTA per
 // boundary; boundaries that fall between tiles have nothing to do.
 __global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, int extra, int M,
-                                     int row_tiles, int ct_tiles, int TH, int ct_cta, int Ct,
-                                     int Ho, int Wo, const float *__restrict__ bias, int relu,
-                                     float *__restrict__ y) {
+                                     int pos_tiles, int ct_tiles, int ST, int ct_cta, int Ct,
+                                     int pitch, int Ho, int Wo, const float *__restrict__ bias,
+                                     int relu, float *__restrict__ y) {
     const int b = blockIdx.x;
     const long long ub = (long long)(b + 1) * base + min(b + 1, extra);
     if (ub % M == 0) return;
     const long long t = ub / M;
-    const int n = (int)(t / ((long long)ct_tiles * row_tiles));
-    const int rest = (int)(t - (long long)n * ct_tiles * row_tiles);
-    const int ct0 = (rest / row_tiles) * ct_cta, oy0 = (rest % row_tiles) * TH;
-    const size_t piece = (size_t)ct_cta * TH * Wo;
+    const int n = (int)(t / ((long long)ct_tiles * pos_tiles));
+    const int rest = (int)(t - (long long)n * ct_tiles * pos_tiles);
+    const int ct0 = (rest / pos_tiles) * ct_cta, l0 = (rest % pos_tiles) * ST;
+    const size_t piece = (size_t)ct_cta * ST;
     const float *p0 = part + (size_t)b * 2 * piece, *p1 = p0 + piece;
     for (int o = threadIdx.x; o < (int)piece; o += blockDim.x) {
-        const int col = o % Wo, r = (o / Wo) % TH, cl = o / (Wo * TH);
-        const int ct = ct0 + cl, oy = oy0 + r;
-        if (ct >= Ct || oy >= Ho) continue;
+        const int cl = o / ST, g = l0 + (o - cl * ST);
+        const int ct = ct0 + cl, oy = g / pitch, col = g - oy * pitch;
+        if (ct >= Ct || oy >= Ho || col >= Wo) continue;
         float v = p0[o] + p1[o];
         if (bias) v += bias[ct];
         if (relu) v = fmaxf(v, 0.f);
@@ -565,7 +569,9 @@ struct FusedVariant {
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
     QCNN_FUSED(7, 8, 1, C4, 16, 1, false, 1.0, 1.0),                                             \
-    QCNN_FUSED(6, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* a 13-row band of pitch 14 */            \
+    QCNN_FUSED(6, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* a whole 13x13 map (pitch 14) */         \
+    QCNN_FUSED(5, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* 27x27 maps in 5 tiles (pitch 29) */     \
+    QCNN_FUSED(5, 16, 1, C4, 16, 1, false, 1.0, 1.0),                                            \
     QCNN_FUSED(4, 8, 1, C4, 16, 2, false, 0.83, 1.0), /* 2 x 16 warps, 64 registers */          \
     QCNN_FUSED(8, 4, 1, C4, 32, 1, false, 0.82, 1.0), /* 32 warps, 64 registers */              \
     QCNN_FUSED(7, 4, 1, C4, 32, 1, false, 0.89, 1.0),                                            \
@@ -589,7 +595,8 @@ struct FusedVariant {
 #define QCNN_FUSED_SK_SET(C4)                      \
     QCNN_FUSED_SK(4, 16, 1, C4, 16, 1, 1.0, 1.0),  \
     QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0),   \
-    QCNN_FUSED_SK(6, 8, 1, C4, 16, 1, 1.0, 1.0)
+    QCNN_FUSED_SK(6, 8, 1, C4, 16, 1, 1.0, 1.0),   \
+    QCNN_FUSED_SK(5, 16, 1, C4, 16, 1, 1.0, 1.0)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
                                       QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
                                       QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};
@@ -645,14 +652,14 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         if (fv.CSP4 != csp4 || fv.BF != s.bf16) continue;
         const int slots = fv.WP * fv.P;
         const int E = fv.BF ? 2 : 1;  // positions per lane and slot
-        int TH = std::min(slots * 32 * E / pitch, s.Ho);
-        if (TH < 1) continue;
-        const int row_tiles = cdiv(s.Ho, TH);
-        TH = cdiv(s.Ho, row_tiles);  // balance the bands
-        // halo positions up to the last one a valid output reads: row
-        // TH + kh - 2, column Wo - 1 + kw - 1 = W + 2 pad - 1
-        const int HP = (TH + s.kh - 2) * pitch + s.W + 2 * s.pad;
+        const int ST = slots * 32 * E;  // output positions per tile
+        const int npos = (s.Ho - 1) * pitch + s.Wo;  // through the last output
+        const int pos_tiles = cdiv(npos, ST);
         const int reach = (s.kh - 1) * pitch + (s.kw - 1);  // largest kernel offset
+        // halo positions read by the lanes of a tile; a map shorter than one
+        // tile needs only those of its own positions (lanes past them read
+        // rows that are never written, and their values are discarded)
+        const int HP = std::min(ST, npos) + reach;
         // fp32: KS floats per row, >= every position read; bf16: two copies
         // of RW words per row, RW > every pair word read or written
         int KS;
@@ -661,7 +668,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
             if ((HP - 1) / 2 >= RW) continue;
             KS = 2 * RW;
         } else {
-            KS = ks_for(std::max(slots * 32 + reach, HP));
+            KS = ks_for(ST + reach);
         }
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
@@ -670,7 +677,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         if (smem > (size_t)smem_optin) continue;
         const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
         const int ct_tiles = cdiv(s.Ct, ct_cta);
-        const double ctas = (double)s.N * row_tiles * ct_tiles;
+        const double ctas = (double)s.N * pos_tiles * ct_tiles;
         // work per CTA and sub-space in shared-memory wavefronts (~cycles):
         // gather (incl. lanes on discarded positions and channels past Ct)
         // over the variant's measured efficiency, plus the exposed part of the
@@ -714,7 +721,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         if (fv.SK) {
             if (!allow_sk || ctas < G || wave_fill >= 0.9) continue;
             sk_units = std::ceil(ctas * s.M / G);
-            const double part = 2.0 * 2.0 * (G - 1) * ct_cta * TH * s.Wo * 4.0;
+            const double part = 2.0 * 2.0 * (G - 1) * ct_cta * ST * 4.0;
             score = sk_units * per_m * cps * 1.05 + part / 3000.0 + 6000.0;
             sk = 1;
             splits = 1;
@@ -726,23 +733,23 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
                 splits > 1 ? (size_t)splits * s.N * s.Ct * s.Ho * s.Wo * sizeof(float) : 0;
             best.sk = sk;
             if (sk) {
-                const long long units = (long long)s.N * row_tiles * ct_tiles * s.M;
+                const long long units = (long long)s.N * pos_tiles * ct_tiles * s.M;
                 best.sk_ctas = G;
                 best.sk_base = (int)(units / G);
                 best.sk_extra = (int)(units % G);
-                best.partial_bytes = (size_t)(G - 1) * 2 * ct_cta * TH * s.Wo * sizeof(float);
+                best.partial_bytes = (size_t)(G - 1) * 2 * ct_cta * ST * sizeof(float);
             }
             best.ok = true;
             best.variant = v;
             best.P = fv.P;
             best.CTW = fv.CTW;
             best.WP = fv.WP;
-            best.TH = TH;
+            best.ST = ST;
             best.pitch = pitch;
             best.KS = KS;
             best.HP = HP;
             best.ct_cta = ct_cta;
-            best.row_tiles = row_tiles;
+            best.pos_tiles = pos_tiles;
             best.ct_tiles = ct_tiles;
             best.smem = smem;
             best.score = score;
@@ -751,10 +758,10 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
 #ifdef QCNN_TUNING
     if (best.ok && getenv("QCNN_PLAN_VERBOSE"))
         fprintf(stderr,
-                "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d pipe=%d TH=%d KS=%d ct_cta=%d smem=%zu "
+                "fused plan: v=%d P=%d CTW=%d WP=%d NW=%d pipe=%d ST=%d tiles=%d KS=%d ct_cta=%d smem=%zu "
                 "splits=%d sk=%d sk_ctas=%d base=%d extra=%d\n",
                 best.variant, best.P, best.CTW, best.WP, kFused[best.variant].NW,
-                kFused[best.variant].PIPE, best.TH, best.KS, best.ct_cta, best.smem, best.splits,
+                kFused[best.variant].PIPE, best.ST, best.pos_tiles, best.KS, best.ct_cta, best.smem, best.splits,
                 best.sk, best.sk_ctas, best.sk_base, best.sk_extra);
 #endif
     return best;
@@ -784,7 +791,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.Ho = s.Ho;
     a.Wo = s.Wo;
     a.pitch = p.pitch;
-    a.TH = p.TH;
+    a.ST = p.ST;
     a.KS = p.KS;
     a.HP = p.HP;
     a.CtP = packed_ct(s.Ct);
@@ -796,21 +803,21 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.sk = p.sk;
     a.sk_base = p.sk_base;
     a.sk_extra = p.sk_extra;
-    a.row_tiles = p.row_tiles;
+    a.pos_tiles = p.pos_tiles;
     a.ct_tiles = p.ct_tiles;
     cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
-    const dim3 grid = p.sk ? dim3(p.sk_ctas, 1, 1) : dim3(p.row_tiles, p.ct_tiles, s.N * p.splits);
+    const dim3 grid = p.sk ? dim3(p.sk_ctas, 1, 1) : dim3(p.pos_tiles, p.ct_tiles, s.N * p.splits);
     fv.fn<<<grid, fv.NW * 32, p.smem, st>>>(a);
     qcnn_status rc = after_launch();
     if (rc != QCNN_OK) return rc;
     if (p.sk) {
         if (p.sk_ctas < 2) return QCNN_OK;
         conv_sk_fixup_kernel<<<p.sk_ctas - 1, 256, 0, st>>>(partial_ws, p.sk_base, p.sk_extra, s.M,
-                                                           p.row_tiles, p.ct_tiles, p.TH,
-                                                           p.ct_cta, s.Ct, s.Ho, s.Wo, bias, relu,
-                                                           y);
+                                                           p.pos_tiles, p.ct_tiles, p.ST,
+                                                           p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
+                                                           bias, relu, y);
         return after_launch();
     }
     if (p.splits == 1) return rc;

@@ -32,18 +32,19 @@ struct ConvShape {
     int bf16;  // 1: table entries rounded to bfloat16 (QCNN_LUT_BF16)
 };
 
-// Fused plan: one CTA = (image, band of TH output rows, CT_CTA channels).
+// Fused plan: one CTA = (image, ST consecutive output positions of the
+// padded grid, CT_CTA channels).
 struct ConvFusedPlan {
     bool ok = false;
     int variant = -1;   // index into the instantiated kernel table
     int P, CTW, WP;     // slots per warp, channels per warp, warps on positions
-    int TH;             // output rows per CTA
+    int ST;             // output positions per tile (slots x 32 x positions per lane)
     int pitch;          // halo row pitch, max(W + pad, Wo)
     int KS;             // 32-bit words per table row (per sub-codeword; bf16:
                         // both copies, 2 x an odd word count)
-    int HP;             // halo positions built: (TH + kh - 2) * pitch + W + 2 pad
+    int HP;             // halo positions built: ST + (kh - 1) * pitch + kw - 1
     int ct_cta;         // channels per CTA
-    int row_tiles, ct_tiles;
+    int pos_tiles, ct_tiles;
     int splits = 1;     // CTAs sharing one tile's sub-spaces (small batches)
     int m_per_split;
     int sk = 0;         // stream-K schedule (large batches): sk_ctas persistent
