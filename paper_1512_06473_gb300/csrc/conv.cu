@@ -572,6 +572,7 @@ struct FusedVariant {
     QCNN_FUSED(6, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* a whole 13x13 map (pitch 14) */         \
     QCNN_FUSED(5, 8, 1, C4, 16, 1, false, 1.0, 1.0), /* 27x27 maps in 5 tiles (pitch 29) */     \
     QCNN_FUSED(5, 16, 1, C4, 16, 1, false, 1.0, 1.0),                                            \
+    QCNN_FUSED(6, 16, 1, C4, 12, 1, false, 1.0, 1.0), /* 12 warps: 192 channels */              \
     QCNN_FUSED(4, 8, 1, C4, 16, 2, false, 0.83, 1.0), /* 2 x 16 warps, 64 registers */          \
     QCNN_FUSED(8, 4, 1, C4, 32, 1, false, 0.82, 1.0), /* 32 warps, 64 registers */              \
     QCNN_FUSED(7, 4, 1, C4, 32, 1, false, 0.89, 1.0),                                            \
@@ -596,7 +597,8 @@ struct FusedVariant {
     QCNN_FUSED_SK(4, 16, 1, C4, 16, 1, 1.0, 1.0),  \
     QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0),   \
     QCNN_FUSED_SK(6, 8, 1, C4, 16, 1, 1.0, 1.0),   \
-    QCNN_FUSED_SK(5, 16, 1, C4, 16, 1, 1.0, 1.0)
+    QCNN_FUSED_SK(5, 16, 1, C4, 16, 1, 1.0, 1.0),  \
+    QCNN_FUSED_SK(6, 16, 1, C4, 12, 1, 1.0, 1.0)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
                                       QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
                                       QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};

@@ -59,6 +59,9 @@ CONV_SWEEP = [
     (1, 8, 1, 1, 4, 1, 1, 1, 0, 4, 1),          # 1x1 map, K = 1
     (3, 8, 4, 70, 65, 3, 3, 1, 1, 4, 32),       # map wider than one warp slot
     (1, 8, 58, 3, 16, 3, 3, 1, 1, 8, 16),       # tall, narrow map
+    (1, 8, 6, 7, 12, 1, 1, 1, 1, 4, 16),        # padding wider than the kernel: Wo > W + pad
+    (2, 8, 5, 6, 20, 3, 3, 1, 3, 4, 32),        # pad 3 around a 3x3 kernel
+    (1, 8, 9, 10, 18, 1, 5, 1, 2, 4, 16),       # 1x5 kernel, pad 2 on every side
 ]
 
 
