@@ -505,8 +505,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 }
 
 // Stream-K fix-up: the tile cut at the end of CTA b's range gets
-// y = (sub-spaces before the cut) + (after) + bias, then ReLU.  One CTA per
-// boundary; boundaries that fall between tiles have nothing to do.
+// y = (sub-spaces before the cut) + (after) + bias, then ReLU.  Grid
+// (boundaries, piece / 1024): each thread adds four consecutive piece
+// entries (one channel, four positions) with 16-byte loads; boundaries that
+// fall between tiles have nothing to do.  Entries on discarded positions were
+// never written and are read but not stored.
 __global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, int extra, int M,
                                      int pos_tiles, int ct_tiles, int ST, int ct_cta, int Ct,
                                      int pitch, int Ho, int Wo, const float *__restrict__ bias,
@@ -514,18 +517,26 @@ __global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, i
     const int b = blockIdx.x;
     const long long ub = (long long)(b + 1) * base + min(b + 1, extra);
     if (ub % M == 0) return;
+    const size_t piece = (size_t)ct_cta * ST;  // a multiple of 4: ST % 32 == 0
+    const size_t o4 = ((size_t)blockIdx.y * blockDim.x + threadIdx.x) * 4;
+    if (o4 >= piece) return;
     const long long t = ub / M;
     const int n = (int)(t / ((long long)ct_tiles * pos_tiles));
     const int rest = (int)(t - (long long)n * ct_tiles * pos_tiles);
     const int ct0 = (rest / pos_tiles) * ct_cta, l0 = (rest % pos_tiles) * ST;
-    const size_t piece = (size_t)ct_cta * ST;
     const float *p0 = part + (size_t)b * 2 * piece, *p1 = p0 + piece;
-    for (int o = threadIdx.x; o < (int)piece; o += blockDim.x) {
-        const int cl = o / ST, g = l0 + (o - cl * ST);
-        const int ct = ct0 + cl, oy = g / pitch, col = g - oy * pitch;
-        if (ct >= Ct || oy >= Ho || col >= Wo) continue;
-        float v = p0[o] + p1[o];
-        if (bias) v += bias[ct];
+    const float4 a = *reinterpret_cast<const float4 *>(p0 + o4);
+    const float4 c = *reinterpret_cast<const float4 *>(p1 + o4);
+    const float v4[4] = {a.x + c.x, a.y + c.y, a.z + c.z, a.w + c.w};
+    const int cl = (int)(o4 / ST), ct = ct0 + cl;
+    if (ct >= Ct) return;
+    const float bv = bias ? bias[ct] : 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int g = l0 + (int)(o4 - (size_t)cl * ST) + i;
+        const int oy = g / pitch, col = g - oy * pitch;
+        if (oy >= Ho || col >= Wo) continue;
+        float v = v4[i] + bv;
         if (relu) v = fmaxf(v, 0.f);
         y[(((size_t)n * Ct + ct) * Ho + oy) * Wo + col] = v;
     }
@@ -690,9 +701,13 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         // Small batches: split the sub-spaces of each tile over `splits` CTAs
         // (partial sums through the workspace, then a reduction) when the
         // grid would leave SMs idle.
+        // The 12-warp tiles lose to 16-warp ones when a CTA gets only a few
+        // sub-spaces (measured: AlexNet conv3 at batch 1, 64 splits, 47 us
+        // against 33 us), so they are split at most 8 ways.
+        const int max_sp = fv.NW == 12 ? 8 : 64;
         int splits = 1;
         double score = 0;
-        for (int sp = 1; sp <= std::min(s.M, 64); sp *= 2) {
+        for (int sp = 1; sp <= std::min(s.M, max_sp); sp *= 2) {
             const int mps = cdiv(s.M, sp);
             const int sp_eff = cdiv(s.M, mps);
             const double waves = std::ceil(ctas * sp_eff / (sms * cps));
@@ -816,7 +831,8 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     if (rc != QCNN_OK) return rc;
     if (p.sk) {
         if (p.sk_ctas < 2) return QCNN_OK;
-        conv_sk_fixup_kernel<<<p.sk_ctas - 1, 256, 0, st>>>(partial_ws, p.sk_base, p.sk_extra, s.M,
+        const dim3 fgrid(p.sk_ctas - 1, (unsigned)cdiv(p.ct_cta * p.ST / 4, 256));
+        conv_sk_fixup_kernel<<<fgrid, 256, 0, st>>>(partial_ws, p.sk_base, p.sk_extra, s.M,
                                                            p.pos_tiles, p.ct_tiles, p.ST,
                                                            p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
                                                            bias, relu, y);
