@@ -60,9 +60,28 @@ typedef enum {
     QCNN_ALGO_AUTO = 0,    /* library picks: fused, else chunked, else unfused */
     QCNN_ALGO_FUSED = 1,   /* full table rows of a band in shared memory, stride 1 only */
     QCNN_ALGO_UNFUSED = 2, /* tables materialised in the workspace first      */
-    QCNN_ALGO_CHUNKED = 3  /* table rows built KC sub-codewords at a time in
+    QCNN_ALGO_CHUNKED = 3, /* table rows built KC sub-codewords at a time in
                               shared memory, any stride                      */
+    QCNN_ALGO_FUSED_VARIANT = 256 /* + v: the fused kernel's tile variant v
+                              (0 <= v < qcnn_conv_fused_variant_count()),
+                              bypassing the planner's choice; for tests and
+                              tuning.  QCNN_ERR_UNSUPPORTED when variant v
+                              cannot serve the shape (stride, C'_s width,
+                              table type, shared memory; a stream-K variant
+                              also needs at least as many tiles as CTA
+                              slots)                                       */
 } qcnn_algo;
+
+/*
+ * The fused conv kernel's instantiated tile variants.  info receives
+ * {P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK}: 32-position slots per warp,
+ * output channels per warp, warps along positions, C'_s register width (4
+ * or 8), warps per CTA, CTAs per SM the registers are sized for, two table
+ * buffers (1/0), bfloat16 tables (1/0), stream-K schedule (1/0).
+ * QCNN_ERR_INVALID_ARG for v out of range or a NULL info.
+ */
+int qcnn_conv_fused_variant_count(void);
+qcnn_status qcnn_conv_fused_variant_info(int v, int info[9]);
 
 /*
  * Precision of the look-up-table entries.  FP32: each entry is the fp32 dot
@@ -201,7 +220,8 @@ qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw,
  *   codes  [Ct][kh*kw][M]  uint8 (codes_layout CANONICAL) or the output of
  *          qcnn_conv_pack_codes (PACKED)
  *   bias   [Ct] or NULL;   y [N][Ct][Ho][Wo] fp32, written
- *   algo:  QCNN_ALGO_FUSED needs stride 1, else QCNN_ERR_UNSUPPORTED.
+ *   algo:  QCNN_ALGO_FUSED (and QCNN_ALGO_FUSED_VARIANT + v) needs stride
+ *          1, else QCNN_ERR_UNSUPPORTED.
  *   lut_type: qcnn_lut_type of the table entries; QCNN_LUT_BF16 is served
  *          by the fused and chunked algorithms (UNFUSED returns
  *          QCNN_ERR_UNSUPPORTED).

@@ -177,10 +177,25 @@ def conv_pack_codes(codes: torch.Tensor, K: int, kh: int, kw: int, stream=None) 
     return packed
 
 
+def fused_variants():
+    """The fused conv kernel's tile variants: a list of dicts (index = the
+    variant number accepted by conv_forward's ``algo``)."""
+    lib = load()
+    keys = ("P", "CTW", "WP", "CSP4", "NW", "MINB", "PIPE", "BF", "SK")
+    out = []
+    for v in range(lib.qcnn_conv_fused_variant_count()):
+        info = (ctypes.c_int * 9)()
+        _lib.check(lib.qcnn_conv_fused_variant_info(v, info), "qcnn_conv_fused_variant_info")
+        out.append(dict(zip(keys, list(info))))
+    return out
+
+
 def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, algo="auto",
                  packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32"):
     """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,
-    then ``Ct`` is required) the output of conv_pack_codes."""
+    then ``Ct`` is required) the output of conv_pack_codes.  ``algo`` is
+    "auto", "fused", "unfused", "chunked", or an int v: fused tile variant v
+    of fused_variants()."""
     _need(x, "x", torch.float32, 4)
     _need(D, "D", torch.float32, 3)
     N, Cs, H, W = x.shape
@@ -195,7 +210,7 @@ def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, al
     if bias is not None:
         _need(bias, "bias", torch.float32, 1)
     layout = _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL
-    a = _lib.ALGO[algo]
+    a = _lib.ALGO[algo] if isinstance(algo, str) else _lib.ALGO_FUSED_VARIANT + int(algo)
     lt = _lib.LUT[lut]
     lib = load()
     nb = ctypes.c_size_t()

@@ -13,6 +13,7 @@ c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_vo
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_DATA = 0, 1, 2, 3, 4, 5
 ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3}
+ALGO_FUSED_VARIANT = 256  # + v: fused tile variant v
 CODES_CANONICAL, CODES_PACKED = 0, 1
 LUT = {"fp32": 0, "bf16": 1}
 LAYER_CONV, LAYER_FC, LAYER_MAXPOOL = 0, 1, 2
@@ -47,6 +48,8 @@ _SIGS = {
     "qcnn_conv_packed_codes_bytes": (c_size_t, [c_int, c_int, c_int, c_int]),
     "qcnn_conv_pack_codes": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_void_p,
                                      c_void_p]),
+    "qcnn_conv_fused_variant_count": (c_int, []),
+    "qcnn_conv_fused_variant_info": (c_int, [c_int, ctypes.POINTER(c_int)]),
     "qcnn_conv_workspace_size": (c_int, [c_int] * 14 + [ctypes.POINTER(c_size_t)]),
     "qcnn_conv_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_int,
                                   c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int,

@@ -99,17 +99,16 @@ struct ConvFusedArgs {
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
 // nlut = 2 table buffers when the sub-spaces are software pipelined.
 struct FusedSmem {
-    size_t lut, xs, ds, cs, hoff, total;
+    size_t lut, xs, ds, cs, total;
 };
 __host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats, int csp4,
-                                                       int kk, int ct_cta, int HP, int nlut) {
+                                                       int kk, int ct_cta, int nlut) {
     FusedSmem s;
     s.lut = 0;
     s.xs = ((size_t)nlut * K * KS * 4 + 15) / 16 * 16;
     s.ds = s.xs + (size_t)2 * xs_floats * 4;
     s.cs = s.ds + (size_t)2 * K * csp4 * 4;
-    s.hoff = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
-    s.total = s.hoff + ((size_t)HP * 4 + 15) / 16 * 16;
+    s.total = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
     return s;
 }
 
@@ -147,6 +146,7 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // SK    : stream-K schedule (a persistent grid over (tile, sub-space) units)
 template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF, bool SK>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
+    static_assert(!SK || (!PIPE && !BF), "the stream-K schedule has one fp32 table buffer");
     constexpr int NT = NW * 32;
     constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     constexpr int CT_CTA = (NW / WP) * CTW;
@@ -158,12 +158,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     extern __shared__ __align__(16) unsigned char smem[];
     const int kk = a.kh * a.kw;
     const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
-    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, HP, PIPE ? 2 : 1);
+    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, PIPE ? 2 : 1);
     float *lut0 = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
-    int *hoff = reinterpret_cast<int *>(smem + L.hoff);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
@@ -173,29 +172,22 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     int sn = blockIdx.z / a.splits, sl0 = blockIdx.x * ST, sct0 = blockIdx.y * CT_CTA;
     const int HW = a.H * a.W;
 
-    // Halo position h of the tile -> offset iy*W + ix inside one input
-    // plane, or -1 where the zero padding is; sub-vector slots j >= C'_s
-    // stay zero.
-    auto make_hoff = [&]() {
-        for (int h = tid; h < HP; h += NT) {
-            const int g = sl0 + h, r = g / pitch, c = g - r * pitch;
-            const int iy = r - a.pad, ix = c - a.pad;
-            hoff[h] = (iy >= 0 && iy < a.H && ix >= 0 && ix < a.W) ? iy * a.W + ix : -1;
-        }
+    // stream-K unit uu -> its tile: image n, first position l0, first channel ct0
+    auto tile_of = [&](long long uu, int &n, int &l0, int &ct0) {
+        const long long t = uu / a.M;
+        n = (int)(t / ((long long)a.ct_tiles * a.pos_tiles));
+        const int rest = (int)(t - (long long)n * a.ct_tiles * a.pos_tiles);
+        ct0 = (rest / a.pos_tiles) * CT_CTA;
+        l0 = (rest % a.pos_tiles) * ST;
     };
     long long u = 0, u1 = 0;  // stream-K unit range
     if constexpr (SK) {
         const int c = blockIdx.x;
         u = (long long)c * a.sk_base + min(c, a.sk_extra);
         u1 = u + a.sk_base + (c < a.sk_extra ? 1 : 0);
-        const long long t = u / a.M;
-        sn = (int)(t / ((long long)a.ct_tiles * a.pos_tiles));
-        const int rest = (int)(t - (long long)sn * a.ct_tiles * a.pos_tiles);
-        sct0 = (rest / a.pos_tiles) * CT_CTA;
-        sl0 = (rest % a.pos_tiles) * ST;
+        tile_of(u, sn, sl0, sct0);
     }
     int cn = sn, cl0 = sl0, cct0 = sct0;
-    make_hoff();
     if (a.Csp < CSP4) {
         for (int e = tid; e < 2 * a.xs_floats; e += NT) xs[e] = 0.f;
         for (int e = tid; e < 2 * K * CSP4; e += NT) ds[e] = 0.f;
@@ -203,23 +195,29 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     __syncthreads();
 
     // ---- asynchronous staging (callers commit) --------------------------
-    auto stage_xd = [&](int m, int b) {  // inputs and sub-codebook of sub-space m
+    // Inputs of sub-space m for the halo of the tile (image n, first
+    // position l0): halo position h is input (iy, ix) = (r - pad, c - pad)
+    // with l0 + h = r*pitch + c, zero-filled where that falls in the padding;
+    // sub-vector slots j >= C'_s stay zero.
+    auto stage_xd = [&](int m, int b, int n, int l0) {
         float *xb = xs + b * a.xs_floats;
-        const float *xn = a.x + ((size_t)sn * a.Cs + (size_t)m * a.Csp) * HW;
-        for (int j = 0; j < a.Csp; ++j) {
-            for (int h = tid; h < HP; h += NT) {
-                const int off = hoff[h];
-                cp_async4(xb + h * CSP4 + j, off >= 0 ? xn + (size_t)j * HW + off : a.x, off >= 0);
-            }
+        const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * HW;
+        for (int h = tid; h < HP; h += NT) {
+            const int g = l0 + h, r = g / pitch, c = g - r * pitch;
+            const int iy = r - a.pad, ix = c - a.pad;
+            const bool ok = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+            const float *src = ok ? xn + iy * a.W + ix : a.x;
+            for (int j = 0; j < a.Csp; ++j)
+                cp_async4(xb + h * CSP4 + j, ok ? src + (size_t)j * HW : a.x, ok);
         }
         float *db = ds + b * K * CSP4;
         const float *dm = a.D + (size_t)m * K * a.Csp;
         for (int k = tid; k < K; k += NT)
             for (int j = 0; j < a.Csp; ++j) cp_async4(db + k * CSP4 + j, dm + k * a.Csp + j, true);
     };
-    auto stage_codes = [&](int m, int b) {
+    auto stage_codes = [&](int m, int b, int ct0) {  // codes of sub-space m, channels ct0..
         uint8_t *cb = cs + (size_t)b * kk * CT_CTA;
-        const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + sct0;
+        const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
         for (int e = tid; e < kk * Q16; e += NT) {
             const int pk = e / Q16, q = e % Q16;
             cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
@@ -400,26 +398,18 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         // and last tile of the range may be cut (partial pieces)
         int m = (int)(u % a.M);
         int piece_m0 = m;  // first sub-space of the current piece
-        stage_xd(m, 0);
-        stage_codes(m, 0);
+        stage_xd(m, 0, sn, sl0);
+        stage_codes(m, 0, sct0);
         cp_async_commit();
         for (int b = 0;; b ^= 1) {
             cp_async_wait<0>();
             __syncthreads();  // unit u staged; gather of the previous unit finished
             const bool last_of_tile = m == a.M - 1, last_of_range = u + 1 == u1;
             if (!last_of_range) {
-                if (last_of_tile) {  // the next unit opens a new tile: new halo table
-                    const long long t = (u + 1) / a.M;
-                    sn = (int)(t / ((long long)a.ct_tiles * a.pos_tiles));
-                    const int rest = (int)(t - (long long)sn * a.ct_tiles * a.pos_tiles);
-                    sct0 = (rest / a.pos_tiles) * CT_CTA;
-                    sl0 = (rest % a.pos_tiles) * ST;
-                    make_hoff();
-                    __syncthreads();
-                }
+                if (last_of_tile) tile_of(u + 1, sn, sl0, sct0);  // the next unit opens a new tile
                 const int mn = last_of_tile ? 0 : m + 1;
-                stage_xd(mn, b ^ 1);
-                stage_codes(mn, b ^ 1);
+                stage_xd(mn, b ^ 1, sn, sl0);
+                stage_codes(mn, b ^ 1, sct0);
                 cp_async_commit();
             }
             build(b, lut0);
@@ -447,16 +437,16 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
         return;
     } else if constexpr (!PIPE) {
-        stage_xd(mb, 0);
-        stage_codes(mb, 0);
+        stage_xd(mb, 0, sn, sl0);
+        stage_codes(mb, 0, sct0);
         cp_async_commit();
         for (int m = mb; m < me; ++m) {
             const int b = (m - mb) & 1;
             cp_async_wait<0>();
             __syncthreads();  // stage m visible; gather of m-1 finished everywhere
             if (m + 1 < me) {
-                stage_xd(m + 1, b ^ 1);
-                stage_codes(m + 1, b ^ 1);
+                stage_xd(m + 1, b ^ 1, sn, sl0);
+                stage_codes(m + 1, b ^ 1, sct0);
                 cp_async_commit();
             }
             if constexpr (BF) build_bf16(b, lut0);
@@ -466,9 +456,9 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     } else {
         float *lut1 = lut0 + (size_t)K * KS;
-        stage_xd(mb, 0);
-        if (mb + 1 < me) stage_xd(mb + 1, 1);
-        stage_codes(mb, 0);
+        stage_xd(mb, 0, sn, sl0);
+        if (mb + 1 < me) stage_xd(mb + 1, 1, sn, sl0);
+        stage_codes(mb, 0, sct0);
         cp_async_commit();
         cp_async_wait<0>();
         __syncthreads();
@@ -479,8 +469,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         // code buffer b, inputs of m+1 in staging buffer b^1.
         for (int m = mb; m < me; ++m) {
             const int b = (m - mb) & 1;
-            if (m + 2 < me) stage_xd(m + 2, b);
-            if (m + 1 < me) stage_codes(m + 1, b ^ 1);
+            if (m + 2 < me) stage_xd(m + 2, b, sn, sl0);
+            if (m + 1 < me) stage_codes(m + 1, b ^ 1, sct0);
             cp_async_commit();
             // even warps build first, odd warps gather first: the latency-bound
             // table build of one half overlaps the other half's gather
@@ -627,7 +617,15 @@ static int ks_for(int need) {  // smallest KS >= need with KS % 32 == 1
     return ks;
 }
 
-ConvFusedPlan plan_conv_fused(const ConvShape &s) {
+int conv_fused_variant_count() { return kNumFused; }
+
+void conv_fused_variant_info(int v, int info[9]) {
+    const FusedVariant &f = kFused[v];
+    const int vals[9] = {f.P, f.CTW, f.WP, f.CSP4, f.NW, f.MINB, f.PIPE, f.BF, f.SK};
+    for (int i = 0; i < 9; ++i) info[i] = vals[i];
+}
+
+ConvFusedPlan plan_conv_fused(const ConvShape &s, int force) {
     ConvFusedPlan best;
     if (s.stride != 1 || s.Csp > kMaxCsp) return best;
     const int csp4 = s.Csp <= 4 ? 4 : 8;
@@ -655,12 +653,10 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
     }
 #ifdef QCNN_TUNING  // tuning builds only: force a variant from the environment
     const char *force_env = getenv("QCNN_FUSED_VARIANT");
-    const int force = force_env ? atoi(force_env) : -1;
+    if (force < 0 && force_env) force = atoi(force_env);
 #endif
     for (int v = 0; v < kNumFused; ++v) {
-#ifdef QCNN_TUNING
         if (force >= 0 && v != force) continue;
-#endif
         const FusedVariant &fv = kFused[v];
         if (fv.CSP4 != csp4 || fv.BF != s.bf16) continue;
         const int slots = fv.WP * fv.P;
@@ -686,7 +682,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
         const int xs_floats = cdiv(HP, 4) * 4 * csp4;
         const size_t smem =
-            fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, HP, fv.PIPE ? 2 : 1).total;
+            fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, fv.PIPE ? 2 : 1).total;
         if (smem > (size_t)smem_optin) continue;
         const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
         const int ct_tiles = cdiv(s.Ct, ct_cta);
@@ -736,7 +732,12 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s) {
         // of the plain grid is well short of full.
         const double wave_fill = ctas / (std::ceil(ctas / G) * G);
         if (fv.SK) {
-            if (!allow_sk || ctas < G || wave_fill >= 0.9) continue;
+            // At least as many tiles as CTA slots: every CTA then takes >= M
+            // units, so a tile is cut at most once (two partial pieces).  The
+            // planner's own choice also wants a short last wave on the plain
+            // grid.
+            if (ctas < G) continue;
+            if (force < 0 && (!allow_sk || wave_fill >= 0.9)) continue;
             sk_units = std::ceil(ctas * s.M / G);
             const double part = 2.0 * 2.0 * (G - 1) * ct_cta * ST * 4.0;
             score = sk_units * per_m * cps * 1.05 + part / 3000.0 + 6000.0;

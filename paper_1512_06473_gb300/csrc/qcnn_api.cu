@@ -98,12 +98,21 @@ struct ConvCall {
 qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvCall *c) {
     if (codes_layout != QCNN_CODES_CANONICAL && codes_layout != QCNN_CODES_PACKED)
         return QCNN_ERR_INVALID_ARG;
-    if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED &&
-        algo != QCNN_ALGO_CHUNKED)
+    const bool forced = algo >= QCNN_ALGO_FUSED_VARIANT;
+    if (forced) {
+        if (algo - QCNN_ALGO_FUSED_VARIANT >= conv_fused_variant_count())
+            return QCNN_ERR_INVALID_ARG;
+    } else if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED &&
+               algo != QCNN_ALGO_CHUNKED) {
         return QCNN_ERR_INVALID_ARG;
+    }
     c->s = s;
     c->algo = QCNN_ALGO_UNFUSED;
-    if (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_FUSED) {
+    if (forced) {
+        c->fp = plan_conv_fused(s, algo - QCNN_ALGO_FUSED_VARIANT);
+        if (!c->fp.ok) return QCNN_ERR_UNSUPPORTED;
+        c->algo = QCNN_ALGO_FUSED;
+    } else if (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_FUSED) {
         c->fp = plan_conv_fused(s);
         if (c->fp.ok) c->algo = QCNN_ALGO_FUSED;
         else if (algo == QCNN_ALGO_FUSED) return QCNN_ERR_UNSUPPORTED;
@@ -362,6 +371,14 @@ qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw, i
         return QCNN_ERR_INVALID_ARG;
     if (!fits_int((long long)packed_ct(Ct) * kh * kw * M)) return QCNN_ERR_INVALID_ARG;
     return launch_pack_codes(codes, Ct, kh * kw, M, K, packed, as_stream(stream));
+}
+
+int qcnn_conv_fused_variant_count(void) { return conv_fused_variant_count(); }
+
+qcnn_status qcnn_conv_fused_variant_info(int v, int info[9]) {
+    if (!info || v < 0 || v >= conv_fused_variant_count()) return QCNN_ERR_INVALID_ARG;
+    conv_fused_variant_info(v, info);
+    return QCNN_OK;
 }
 
 qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh, int kw,

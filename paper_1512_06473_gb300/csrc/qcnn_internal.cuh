@@ -55,7 +55,10 @@ struct ConvFusedPlan {
     double score;       // estimated cost (lower is better)
 };
 
-ConvFusedPlan plan_conv_fused(const ConvShape &s);
+// force >= 0: only that variant, without the planner's preference gates
+ConvFusedPlan plan_conv_fused(const ConvShape &s, int force = -1);
+int conv_fused_variant_count();
+void conv_fused_variant_info(int v, int info[9]);
 
 struct ConvUnfusedPlan {
     int NB;             // images per table chunk

@@ -183,3 +183,44 @@ def test_quantizer_argument_checks():
     assert lib.qcnn_kmeans(8, 4, 100, 4, 16, 8, 2, 8, 8, None, 0, None) == _lib.ERR_WORKSPACE
     assert lib.qcnn_pq_quantize(FC, 8, 10, 12, 1, 1, 4, 16, 8, 2, 8, 8, 4096 + 8, 1 << 20,
                                 None) == _lib.ERR_WORKSPACE  # misaligned workspace
+
+
+def test_fused_variant_table():
+    n = lib.qcnn_conv_fused_variant_count()
+    assert n >= 10
+    info = (ctypes.c_int * 9)()
+    seen_sk = seen_pipe = seen_bf = False
+    for v in range(n):
+        assert lib.qcnn_conv_fused_variant_info(v, info) == 0
+        P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK = list(info)
+        assert P >= 1 and (CTW in (4, 8) or CTW % 16 == 0)
+        assert CSP4 in (4, 8) and NW in (8, 12, 16, 32) and MINB in (1, 2)
+        assert (NW // WP) * CTW % 16 == 0
+        seen_sk |= bool(SK)
+        seen_pipe |= bool(PIPE)
+        assert not (SK and (PIPE or BF))
+        seen_bf |= bool(BF)
+    assert seen_sk and seen_pipe and seen_bf
+    assert lib.qcnn_conv_fused_variant_info(n, info) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_conv_fused_variant_info(-1, info) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_conv_fused_variant_info(0, None) == _lib.ERR_INVALID_ARG
+
+
+def test_forced_fused_variant_planning():
+    """Every variant either plans the shape or reports it unsupported; an
+    index past the table is an argument error; strided convs never fuse."""
+    n = lib.qcnn_conv_fused_variant_count()
+    nb = ctypes.c_size_t()
+    shape = (64, 64, 13, 13, 384, 3, 3, 1, 1, 4, 128)
+    ok = 0
+    for v in range(n):
+        rc = lib.qcnn_conv_workspace_size(*shape, 0, _lib.ALGO_FUSED_VARIANT + v, 0,
+                                          ctypes.byref(nb))
+        assert rc in (0, _lib.ERR_UNSUPPORTED)
+        ok += rc == 0
+    assert ok >= 5
+    assert lib.qcnn_conv_workspace_size(*shape, 0, _lib.ALGO_FUSED_VARIANT + n, 0,
+                                        ctypes.byref(nb)) == _lib.ERR_INVALID_ARG
+    strided = (1, 8, 15, 15, 4, 3, 3, 2, 1, 4, 16)
+    assert lib.qcnn_conv_workspace_size(*strided, 0, _lib.ALGO_FUSED_VARIANT, 0,
+                                        ctypes.byref(nb)) == _lib.ERR_UNSUPPORTED

@@ -315,3 +315,37 @@ def test_conv_stream_k(case):
     refi = oracle.conv_forward(xi, Di, ci, kh, kw, s, p, bi)
     goti = host(q.conv_forward(cuda(xi), cuda(Di), cuda(ci), kh, kw, s, p, cuda(bi)))
     assert np.array_equal(goti.astype(np.float64), refi)
+
+
+# Every instantiated fused tile variant, forced through the C ABI (the
+# planner only ever picks some of them).  Integer inputs with |x|, |D| <= 4
+# keep every table entry within 256, so fp32 and bfloat16 tables alike give
+# the exact result.  The batches give the stream-K variants at least as many
+# tiles as CTA slots.
+FORCED = [
+    (80, 16, 13, 13, 384, 3, 3, 1, 1, 4, 128),   # C'_s = 4, 13x13 (one- or two-tile maps)
+    (32, 16, 27, 27, 256, 5, 5, 1, 2, 8, 64),    # C'_s = 8, 27x27 (several tiles)
+]
+
+
+@pytest.mark.parametrize("case", FORCED, ids=lambda c: "x".join(map(str, c)))
+def test_every_fused_variant_is_exact(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    M = Cs // Csp
+    x = synth.small_integers((N, Cs, H, W), -4, 4, 61, 0)
+    D = synth.small_integers((M, K, Csp), -4, 4, 61, 1)
+    b = synth.small_integers((Ct,), -8, 8, 61, 3)
+    codes = synth.uniform_codes((Ct, kh * kw, M), K, 61, 2)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    xd, Dd, cd, bd = cuda(x), cuda(D), cuda(codes), cuda(b)
+    ran = {"sk": 0, "pipe": 0, "bf": 0, "plain": 0}
+    for v, info in enumerate(q.fused_variants()):
+        try:
+            got = q.conv_forward(xd, Dd, cd, kh, kw, s, p, bd, relu=True, algo=v,
+                                 lut="bf16" if info["BF"] else "fp32")
+        except q.QcnnError as e:
+            assert e.status == 2, (v, info)  # QCNN_ERR_UNSUPPORTED: variant cannot serve it
+            continue
+        assert np.array_equal(host(got).astype(np.float64), ref), (v, info)
+        ran["sk" if info["SK"] else "bf" if info["BF"] else "pipe" if info["PIPE"] else "plain"] += 1
+    assert ran["sk"] >= 2 and ran["bf"] >= 2 and ran["plain"] >= 4, ran
