@@ -34,7 +34,9 @@
  *    then unspecified.
  *  - A failed launch returns QCNN_ERR_CUDA; the CUDA error is in
  *    qcnn_last_cuda_error().  The library is stateless apart from that
- *    value and a launch counter, and is safe to call from several threads.
+ *    value, a launch counter and, per device, the copy stream and events of
+ *    qcnn_net_forward_host (created on its first call), and is safe to call
+ *    from several threads.
  */
 #ifndef QCNN_H
 #define QCNN_H
@@ -424,7 +426,11 @@ qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers,
 /*
  * qcnn_net_forward_host -- the same, with x and y in HOST memory (pinned
  * memory gives the fastest copies).  Copies x to the device, runs the
- * stack, copies y back, and synchronizes `stream` before returning.
+ * stack, copies y back, and synchronizes `stream` before returning.  When
+ * N is a multiple of 2 or 4 with at least 8 images per slice, x is copied
+ * in 2 or 4 slices on a separate copy stream of the library, and the first
+ * layer runs on each slice as soon as it has arrived.  Calls of this
+ * function on one device are serialized.
  */
 qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers,
                                   const float *x_host, int N, int C, int H,

@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <atomic>
 #include <climits>
+#include <mutex>
 #include <vector>
 
 namespace qcnn {
@@ -172,6 +173,7 @@ bool ws_ok(const void *ws, size_t have, size_t need) {
 // -------------------------------------------------------------- net plan ---
 struct NetStep {
     int kind;
+    int N;              // batch this step is planned for
     ConvCall conv;
     FcShape fc;
     FcPlan fcp;
@@ -183,10 +185,59 @@ struct NetStep {
 struct NetPlan {
     int N;
     std::vector<NetStep> steps;
+    // host I/O: the input is copied in `chunks` slices of N / chunks images,
+    // and the first layer runs on each slice as soon as it has arrived
+    // (step0c, planned for the slice), overlapping the remaining copies
+    int chunks = 1;
+    NetStep step0c;
     size_t act_floats;  // floats of one ping-pong activation buffer
     size_t scratch;     // max layer scratch
     size_t act_off[2], scratch_off, xin_off, yout_off, total;
 };
+
+qcnn_status plan_step(const qcnn_layer &L, int N, int c, int h, int w, NetStep *out) {
+    NetStep st{};
+    st.kind = L.kind;
+    st.N = N;
+    st.C = c;
+    st.H = h;
+    st.W = w;
+    if (L.kind == QCNN_LAYER_CONV) {
+        if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
+        ConvShape s;
+        if (!conv_shape(N, c, h, w, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K, L.lut_type,
+                        &s))
+            return QCNN_ERR_INVALID_ARG;
+        qcnn_status rc = plan_conv_call(s, L.codes_layout, L.algo, &st.conv);
+        if (rc != QCNN_OK) return rc;
+        st.scratch = st.conv.total;
+        st.oC = L.Ct;
+        st.oH = s.Ho;
+        st.oW = s.Wo;
+    } else if (L.kind == QCNN_LAYER_FC) {
+        if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
+        const long long cs = (long long)c * h * w;
+        if (cs >= INT_MAX) return QCNN_ERR_INVALID_ARG;
+        if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, L.lut_type, &st.fc))
+            return QCNN_ERR_INVALID_ARG;
+        if (L.codes_layout == QCNN_CODES_PACKED) st.fc.code_bits = code_bits(L.K);
+        else if (L.codes_layout != QCNN_CODES_CANONICAL) return QCNN_ERR_INVALID_ARG;
+        st.fcp = plan_fc(st.fc);
+        st.scratch = align_up(st.fcp.partial_bytes, kWsAlign);
+        st.oC = L.Ct;
+        st.oH = 1;
+        st.oW = 1;
+    } else if (L.kind == QCNN_LAYER_MAXPOOL) {
+        if (L.kh <= 0 || L.stride <= 0 || L.kh > h || L.kh > w) return QCNN_ERR_INVALID_ARG;
+        st.oC = c;
+        st.oH = (h - L.kh) / L.stride + 1;
+        st.oW = (w - L.kh) / L.stride + 1;
+    } else {
+        return QCNN_ERR_INVALID_ARG;
+    }
+    *out = st;
+    return QCNN_OK;
+}
 
 qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H, int W,
                      int host_io, NetPlan *np) {
@@ -199,45 +250,9 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
     np->scratch = 0;
     int c = C, h = H, w = W;
     for (int i = 0; i < n_layers; ++i) {
-        const qcnn_layer &L = layers[i];
-        NetStep st{};
-        st.kind = L.kind;
-        st.C = c;
-        st.H = h;
-        st.W = w;
-        if (L.kind == QCNN_LAYER_CONV) {
-            if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
-            ConvShape s;
-            if (!conv_shape(N, c, h, w, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K,
-                            L.lut_type, &s))
-                return QCNN_ERR_INVALID_ARG;
-            qcnn_status rc = plan_conv_call(s, L.codes_layout, L.algo, &st.conv);
-            if (rc != QCNN_OK) return rc;
-            st.scratch = st.conv.total;
-            st.oC = L.Ct;
-            st.oH = s.Ho;
-            st.oW = s.Wo;
-        } else if (L.kind == QCNN_LAYER_FC) {
-            if (!L.D || !L.codes) return QCNN_ERR_INVALID_ARG;
-            const long long cs = (long long)c * h * w;
-            if (cs >= INT_MAX) return QCNN_ERR_INVALID_ARG;
-            if (!fc_shape(N, (int)cs, L.Ct, L.Csp, L.K, L.lut_type, &st.fc))
-                return QCNN_ERR_INVALID_ARG;
-            if (L.codes_layout == QCNN_CODES_PACKED) st.fc.code_bits = code_bits(L.K);
-            else if (L.codes_layout != QCNN_CODES_CANONICAL) return QCNN_ERR_INVALID_ARG;
-            st.fcp = plan_fc(st.fc);
-            st.scratch = align_up(st.fcp.partial_bytes, kWsAlign);
-            st.oC = L.Ct;
-            st.oH = 1;
-            st.oW = 1;
-        } else if (L.kind == QCNN_LAYER_MAXPOOL) {
-            if (L.kh <= 0 || L.stride <= 0 || L.kh > h || L.kh > w) return QCNN_ERR_INVALID_ARG;
-            st.oC = c;
-            st.oH = (h - L.kh) / L.stride + 1;
-            st.oW = (w - L.kh) / L.stride + 1;
-        } else {
-            return QCNN_ERR_INVALID_ARG;
-        }
+        NetStep st;
+        qcnn_status rc = plan_step(layers[i], N, c, h, w, &st);
+        if (rc != QCNN_OK) return rc;
         const long long out = (long long)N * st.oC * st.oH * st.oW;
         if (!fits_int(out)) return QCNN_ERR_INVALID_ARG;
         if (i + 1 < n_layers) np->act_floats = std::max(np->act_floats, (size_t)out);
@@ -246,6 +261,14 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
         h = st.oH;
         w = st.oW;
         np->steps.push_back(st);
+    }
+    np->chunks = 1;
+    if (host_io) {
+        const int ch = (N % 4 == 0 && N / 4 >= 8) ? 4 : (N % 2 == 0 && N / 2 >= 8) ? 2 : 1;
+        if (ch > 1 && plan_step(layers[0], N / ch, C, H, W, &np->step0c) == QCNN_OK) {
+            np->chunks = ch;
+            np->scratch = std::max(np->scratch, np->step0c.scratch);
+        }
     }
     size_t off = 0;
     for (int b = 0; b < 2; ++b) {
@@ -266,30 +289,69 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
     return QCNN_OK;
 }
 
-qcnn_status run_net(const qcnn_layer *layers, const NetPlan &np, const float *x, float *y,
-                    void *ws, cudaStream_t st) {
+qcnn_status run_step(const qcnn_layer &L, const NetStep &s, const float *in, float *out,
+                     void *scratch, cudaStream_t st) {
+    if (s.kind == QCNN_LAYER_CONV)
+        return run_conv(s.conv, in, L.D, L.codes, L.codes_layout, L.bias, out, L.relu, scratch,
+                        st);
+    if (s.kind == QCNN_LAYER_FC)
+        return launch_fc(s.fc, s.fcp, in, L.D, L.codes, L.bias, out, L.relu,
+                         reinterpret_cast<float *>(scratch), st);
+    return launch_maxpool(in, s.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
+}
+
+// Layers [first, n) of the stack; `in` is the input of layer `first`.
+qcnn_status run_net(const qcnn_layer *layers, const NetPlan &np, const float *in, float *y,
+                    void *ws, cudaStream_t st, int first = 0) {
     uint8_t *base = static_cast<uint8_t *>(ws);
     const int n = (int)np.steps.size();
-    const float *in = x;
-    for (int i = 0; i < n; ++i) {
-        const NetStep &s = np.steps[i];
-        const qcnn_layer &L = layers[i];
+    for (int i = first; i < n; ++i) {
         float *out = (i + 1 == n) ? y : reinterpret_cast<float *>(base + np.act_off[i & 1]);
-        void *scratch = base + np.scratch_off;
-        qcnn_status rc = QCNN_OK;
-        if (s.kind == QCNN_LAYER_CONV) {
-            rc = run_conv(s.conv, in, L.D, L.codes, L.codes_layout, L.bias, out, L.relu,
-                          scratch, st);
-        } else if (s.kind == QCNN_LAYER_FC) {
-            rc = launch_fc(s.fc, s.fcp, in, L.D, L.codes, L.bias, out, L.relu,
-                           reinterpret_cast<float *>(scratch), st);
-        } else {
-            rc = launch_maxpool(in, np.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
-        }
+        qcnn_status rc = run_step(layers[i], np.steps[i], in, out, base + np.scratch_off, st);
         if (rc != QCNN_OK) return rc;
         in = out;
     }
     return QCNN_OK;
+}
+
+// Per device: the stream that copies host input slices and the events that
+// order them, created on the first qcnn_net_forward_host call on that device
+// and kept for the life of the process.  The mutex serializes host-I/O calls
+// on one device (each ends with a stream synchronization anyway).
+constexpr int kHostChunksMax = 4;
+struct HostIo {
+    std::mutex mu;
+    bool ok = false;
+    cudaStream_t copy = nullptr;
+    cudaEvent_t start = nullptr, ready[kHostChunksMax] = {};
+};
+
+HostIo *host_io(int dev) {
+    static HostIo slots[64];
+    if (dev < 0 || dev >= 64) return nullptr;
+    return &slots[dev];
+}
+
+bool host_io_init(HostIo &h) {  // called with h.mu held
+    if (h.ok) return true;
+    if (cudaStreamCreateWithFlags(&h.copy, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    bool ok = cudaEventCreateWithFlags(&h.start, cudaEventDisableTiming) == cudaSuccess;
+    for (int c = 0; ok && c < kHostChunksMax; ++c)
+        ok = cudaEventCreateWithFlags(&h.ready[c], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {  // undo, so that a later call starts from scratch
+        cudaGetLastError();
+        for (cudaEvent_t &e : h.ready)
+            if (e) cudaEventDestroy(e), e = nullptr;
+        if (h.start) cudaEventDestroy(h.start), h.start = nullptr;
+        cudaStreamDestroy(h.copy);
+        h.copy = nullptr;
+        return false;
+    }
+    h.ok = true;
+    return true;
 }
 
 }  // namespace
@@ -466,13 +528,48 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
     const NetStep &last = np.steps.back();
     const size_t xb = (size_t)N * C * H * W * sizeof(float);
     const size_t yb = (size_t)N * last.oC * last.oH * last.oW * sizeof(float);
-    rc = cuda_status(cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st));
-    if (rc != QCNN_OK) return rc;
-    rc = run_net(layers, np, xd, yd, workspace, st);
-    if (rc != QCNN_OK) return rc;
-    rc = cuda_status(cudaMemcpyAsync(y_host, yd, yb, cudaMemcpyDeviceToHost, st));
-    if (rc != QCNN_OK) return rc;
-    return cuda_status(cudaStreamSynchronize(st));
+    int dev = 0;
+    HostIo *hio = cudaGetDevice(&dev) == cudaSuccess ? host_io(dev) : nullptr;
+    cudaGetLastError();
+    std::unique_lock<std::mutex> lock;
+    if (np.chunks > 1 && hio) {
+        lock = std::unique_lock<std::mutex>(hio->mu);
+        if (!host_io_init(*hio)) {
+            lock.unlock();
+            hio = nullptr;
+        }
+    }
+    if (np.chunks > 1 && hio) {
+        // slice c of the input is copied on the copy stream (after the work
+        // already queued on `stream`), and the first layer runs on it as soon
+        // as it has arrived, while the later slices are still copying
+        const int nc = np.chunks;
+        const size_t xs = xb / nc;
+        const NetStep &s0 = np.step0c;
+        const size_t ys = (size_t)s0.N * s0.oC * s0.oH * s0.oW;
+        float *y0 = np.steps.size() == 1 ? yd : reinterpret_cast<float *>(base + np.act_off[0]);
+        rc = cuda_status(cudaEventRecord(hio->start, st));
+        if (rc == QCNN_OK) rc = cuda_status(cudaStreamWaitEvent(hio->copy, hio->start, 0));
+        for (int c = 0; c < nc && rc == QCNN_OK; ++c) {
+            rc = cuda_status(cudaMemcpyAsync(reinterpret_cast<uint8_t *>(xd) + c * xs,
+                                             reinterpret_cast<const uint8_t *>(x_host) + c * xs,
+                                             xs, cudaMemcpyHostToDevice, hio->copy));
+            if (rc == QCNN_OK) rc = cuda_status(cudaEventRecord(hio->ready[c], hio->copy));
+        }
+        for (int c = 0; c < nc && rc == QCNN_OK; ++c) {
+            rc = cuda_status(cudaStreamWaitEvent(st, hio->ready[c], 0));
+            if (rc == QCNN_OK)
+                rc = run_step(layers[0], s0, xd + (size_t)c * (xs / sizeof(float)), y0 + c * ys,
+                              base + np.scratch_off, st);
+        }
+        if (rc == QCNN_OK && np.steps.size() > 1) rc = run_net(layers, np, y0, yd, workspace, st, 1);
+    } else {
+        rc = cuda_status(cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st));
+        if (rc == QCNN_OK) rc = run_net(layers, np, xd, yd, workspace, st);
+    }
+    if (rc == QCNN_OK) rc = cuda_status(cudaMemcpyAsync(y_host, yd, yb, cudaMemcpyDeviceToHost, st));
+    const qcnn_status sync = cuda_status(cudaStreamSynchronize(st));
+    return rc != QCNN_OK ? rc : sync;
 }
 
 }  // extern "C"
