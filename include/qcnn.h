@@ -59,11 +59,15 @@ typedef enum {
 } qcnn_status;
 
 typedef enum {
-    QCNN_ALGO_AUTO = 0,    /* library picks: fused, else chunked, else unfused */
+    QCNN_ALGO_AUTO = 0,    /* library picks: fused (stride 1), else phase,
+                              else chunked, else unfused                     */
     QCNN_ALGO_FUSED = 1,   /* full table rows of a band in shared memory, stride 1 only */
     QCNN_ALGO_UNFUSED = 2, /* tables materialised in the workspace first      */
     QCNN_ALGO_CHUNKED = 3, /* table rows built KC sub-codewords at a time in
                               shared memory, any stride                      */
+    QCNN_ALGO_PHASE = 4,   /* full table rows of one stride phase of a tile
+                              at a time in shared memory, any stride (fp32
+                              tables)                                        */
     QCNN_ALGO_FUSED_VARIANT = 256 /* + v: the fused kernel's tile variant v
                               (0 <= v < qcnn_conv_fused_variant_count()),
                               bypassing the planner's choice; for tests and

@@ -194,7 +194,7 @@ def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, al
                  packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32"):
     """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,
     then ``Ct`` is required) the output of conv_pack_codes.  ``algo`` is
-    "auto", "fused", "unfused", "chunked", or an int v: fused tile variant v
+    "auto", "fused", "unfused", "chunked", "phase", or an int v: fused tile variant v
     of fused_variants()."""
     _need(x, "x", torch.float32, 4)
     _need(D, "D", torch.float32, 3)

@@ -12,7 +12,7 @@ from . import build as _build
 c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_uint64
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_DATA = 0, 1, 2, 3, 4, 5
-ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3}
+ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3, "phase": 4}
 ALGO_FUSED_VARIANT = 256  # + v: fused tile variant v
 CODES_CANONICAL, CODES_PACKED = 0, 1
 LUT = {"fp32": 0, "bf16": 1}

@@ -215,12 +215,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         for (int k = tid; k < K; k += NT)
             for (int j = 0; j < a.Csp; ++j) cp_async4(db + k * CSP4 + j, dm + k * a.Csp + j, true);
     };
-    auto stage_codes = [&](int m, int b, int ct0) {  // codes of sub-space m, channels ct0..
+    // codes of sub-space m, channels ct0 ..; 16-byte pieces past the packed
+    // row (CtP, a multiple of 256, may be short of the last tile) are zeros
+    auto stage_codes = [&](int m, int b, int ct0) {
         uint8_t *cb = cs + (size_t)b * kk * CT_CTA;
         const uint8_t *cm = a.codes + (size_t)m * kk * a.CtP + ct0;
         for (int e = tid; e < kk * Q16; e += NT) {
             const int pk = e / Q16, q = e % Q16;
-            cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
+            if (ct0 + q * 16 < a.CtP)
+                cp_async16(cb + pk * CT_CTA + q * 16, cm + (size_t)pk * a.CtP + q * 16);
+            else
+                *reinterpret_cast<uint4 *>(cb + pk * CT_CTA + q * 16) = make_uint4(0, 0, 0, 0);
         }
     };
 

@@ -89,8 +89,9 @@ bool fc_shape(int N, int Cs, int Ct, int Csp, int K, int lut_type, FcShape *s) {
 // ------------------------------------------------------------ conv plan ---
 struct ConvCall {
     ConvShape s;
-    int algo;  // resolved: FUSED, CHUNKED or UNFUSED
+    int algo;  // resolved: FUSED, PHASE, CHUNKED or UNFUSED
     ConvFusedPlan fp;
+    ConvPhasePlan pp;
     ConvChunkPlan cp;
     ConvUnfusedPlan up;
     size_t packed_off, lut_off, total;
@@ -104,7 +105,7 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         if (algo - QCNN_ALGO_FUSED_VARIANT >= conv_fused_variant_count())
             return QCNN_ERR_INVALID_ARG;
     } else if (algo != QCNN_ALGO_AUTO && algo != QCNN_ALGO_FUSED && algo != QCNN_ALGO_UNFUSED &&
-               algo != QCNN_ALGO_CHUNKED) {
+               algo != QCNN_ALGO_CHUNKED && algo != QCNN_ALGO_PHASE) {
         return QCNN_ERR_INVALID_ARG;
     }
     c->s = s;
@@ -117,6 +118,11 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         c->fp = plan_conv_fused(s);
         if (c->fp.ok) c->algo = QCNN_ALGO_FUSED;
         else if (algo == QCNN_ALGO_FUSED) return QCNN_ERR_UNSUPPORTED;
+    }
+    if (c->algo == QCNN_ALGO_UNFUSED && (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_PHASE)) {
+        c->pp = plan_conv_phase(s);
+        if (c->pp.ok) c->algo = QCNN_ALGO_PHASE;
+        else if (algo == QCNN_ALGO_PHASE) return QCNN_ERR_UNSUPPORTED;
     }
     if (c->algo == QCNN_ALGO_UNFUSED && (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_CHUNKED)) {
         c->cp = plan_conv_chunked(s);
@@ -136,6 +142,8 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         off += align_up(c->up.lut_bytes, kWsAlign);
     } else if (c->algo == QCNN_ALGO_CHUNKED) {
         off += c->cp.entries_bytes + c->cp.starts_bytes;
+    } else if (c->algo == QCNN_ALGO_PHASE) {
+        off += align_up(c->pp.partial_bytes, kWsAlign);
     } else {
         off += align_up(c->fp.partial_bytes, kWsAlign);
     }
@@ -157,11 +165,11 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
         if (rc != QCNN_OK) return rc;
         packed = p;
     }
-    if (c.algo == QCNN_ALGO_FUSED)
-        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu,
-                                 reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off),
-                                 st);
     float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
+    if (c.algo == QCNN_ALGO_FUSED)
+        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, lut, st);
+    if (c.algo == QCNN_ALGO_PHASE)
+        return launch_conv_phase(c.s, c.pp, x, D, packed, bias, y, relu, lut, st);
     return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
 }
 

@@ -81,6 +81,22 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
                                 const float *bias, float *y, int relu, void *ws,
                                 cudaStream_t st);
 
+// Stride-phase plan (conv_phase.cu): full table rows of one stride phase of
+// a tile at a time, any stride.
+struct ConvPhasePlan {
+    bool ok = false;
+    int variant = -1;
+    int pitch, dymin, dxmin, HP, KS, ct_cta, pos_tiles, ct_tiles;
+    int splits = 1, units_per_split = 0;  // (sub-space, phase) units per CTA
+    size_t partial_bytes = 0;             // workspace for split partial sums
+    size_t smem;
+    double score;
+};
+ConvPhasePlan plan_conv_phase(const ConvShape &s);
+qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
+                              const float *D, const uint8_t *packed, const float *bias, float *y,
+                              int relu, float *partial_ws, cudaStream_t st);
+
 size_t packed_codes_bytes(int Ct, int kk, int M);
 int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
 

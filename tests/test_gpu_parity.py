@@ -62,11 +62,13 @@ CONV_SWEEP = [
     (1, 8, 6, 7, 12, 1, 1, 1, 1, 4, 16),        # padding wider than the kernel: Wo > W + pad
     (2, 8, 5, 6, 20, 3, 3, 1, 3, 4, 32),        # pad 3 around a 3x3 kernel
     (1, 8, 9, 10, 18, 1, 5, 1, 2, 4, 16),       # 1x5 kernel, pad 2 on every side
+    (2, 8, 17, 19, 40, 5, 5, 3, 2, 4, 64),      # stride 3 with padding: phases of 2x2 .. 1x1
+    (1, 16, 23, 23, 130, 3, 3, 2, 0, 8, 256),   # stride 2, K = 256, ragged channel tile
 ]
 
 
 @pytest.mark.parametrize("case", CONV_SWEEP, ids=lambda c: "x".join(map(str, c)))
-@pytest.mark.parametrize("algo", ["auto", "unfused", "chunked"])
+@pytest.mark.parametrize("algo", ["auto", "unfused", "chunked", "phase"])
 def test_conv_sweep(case, algo):
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
     x, D, codes, b = conv_case(hash(case) % 1000, N, Cs, H, W, Ct, kh, kw, Csp, K)
@@ -87,7 +89,7 @@ def test_conv_fused_forced(case):
     assert rel(host(got), ref) <= TOL
 
 
-@pytest.mark.parametrize("algo", ["fused", "unfused", "chunked"])
+@pytest.mark.parametrize("algo", ["fused", "unfused", "chunked", "phase"])
 def test_conv_integer_bit_exact(algo):
     case = (2, 16, 14, 13, 36, 3, 3, 1, 1, 4, 32)
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
@@ -137,7 +139,7 @@ def test_out_of_range_codes_are_clamped_not_faulting():
     bad = codes.copy()
     bad[::3, ::2, :] = 255
     good = np.minimum(bad, K - 1).astype(np.uint8)
-    for algo in ("fused", "unfused", "chunked"):
+    for algo in ("fused", "unfused", "chunked", "phase"):
         a = host(q.conv_forward(cuda(x), cuda(D), cuda(bad), kh, kw, 1, 1, cuda(b), algo=algo))
         c = host(q.conv_forward(cuda(x), cuda(D), cuda(good), kh, kw, 1, 1, cuda(b), algo=algo))
         assert np.array_equal(a, c)
