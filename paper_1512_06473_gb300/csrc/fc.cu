@@ -212,7 +212,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                         }
                         lw[(mm * a.K + k) * a.NTP + np] = pack_bf16x2(v0, v1);
                     }
-                } else {
+                } else if constexpr (BF) {
                     for (int e = tid; e < a.K * NT; e += kFcThreads) {
                         const int nn = e % NT, k = e / NT;
                         const float *xp = xb + mm * a.Csp * a.NTX + nn;
@@ -221,11 +221,38 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
 #pragma unroll
                         for (int j = 0; j < kMaxCsp; ++j)
                             if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
-                        if constexpr (BF)
-                            reinterpret_cast<unsigned short *>(lut)[(mm * a.K + k) * a.NTP + nn] =
-                                (unsigned short)(pack_bf16x2(v, 0.f) & 0xffffu);
-                        else
+                        reinterpret_cast<unsigned short *>(lut)[(mm * a.K + k) * a.NTP + nn] =
+                            (unsigned short)(pack_bf16x2(v, 0.f) & 0xffffu);
+                    }
+                }
+            }
+            if constexpr (!BF) {
+                // fp32: the chunk's (mm, k, nn) entries with every thread busy --
+                // several sub-spaces side by side when K * NT < the block
+                const int per_mm = a.K * NT;
+                const int lanes_mm = min(per_mm, kFcThreads);
+                const int mm_step = kFcThreads / lanes_mm;
+                const int t_mm = tid / lanes_mm, t_e = tid - t_mm * lanes_mm;
+                if (t_mm < mm_step) {
+                    for (int mm = t_mm; mm < mch; mm += mm_step) {
+                        for (int e = t_e; e < per_mm; e += lanes_mm) {
+                            const int nn = e % NT, k = e / NT;
+                            const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                            const float *dp = db + (mm * a.K + k) * a.Csp;
+                            float v = 0.f;
+                            if (a.Csp == 4) {  // one 16-byte load of the sub-codeword
+                                const float4 d = *reinterpret_cast<const float4 *>(dp);
+                                v = fmaf(xp[0], d.x, v);
+                                v = fmaf(xp[a.NTX], d.y, v);
+                                v = fmaf(xp[2 * a.NTX], d.z, v);
+                                v = fmaf(xp[3 * a.NTX], d.w, v);
+                            } else {
+#pragma unroll
+                                for (int j = 0; j < kMaxCsp; ++j)
+                                    if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
+                            }
                             lut[(mm * a.K + k) * a.NTP + nn] = v;
+                        }
                     }
                 }
             }

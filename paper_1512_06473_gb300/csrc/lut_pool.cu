@@ -63,19 +63,18 @@ qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *
 }
 
 // k x k max-pool, stride s, no padding: one thread per output element.
-__global__ void maxpool_kernel(const float *__restrict__ x, int NC, int H, int W, int k, int s,
+// One thread per output, 32-bit index arithmetic (every element count is
+// below 2^31); neighbouring windows share their overlap through L1.
+__global__ void maxpool_kernel(const float *__restrict__ x, int total, int H, int W, int k, int s,
                                int Ho, int Wo, float *__restrict__ y) {
-    const size_t total = (size_t)NC * Ho * Wo;
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const int ox = (int)(i % Wo);
-        const size_t r = i / Wo;
-        const int oy = (int)(r % Ho);
-        const size_t nc = r / Ho;
-        const float *p = x + (nc * H + (size_t)oy * s) * W + (size_t)ox * s;
-        float v = p[0];
+    const int HoWo = Ho * Wo;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+        const int nc = i / HoWo, o = i - nc * HoWo;
+        const int oy = o / Wo, ox = o - oy * Wo;
+        const float *p = x + (size_t)nc * H * W + oy * s * W + ox * s;
+        float v = __ldg(p);
         for (int dy = 0; dy < k; ++dy)
-            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, __ldg(p + (size_t)dy * W + dx));
+            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, __ldg(p + dy * W + dx));
         y[i] = v;
     }
 }
@@ -83,9 +82,9 @@ __global__ void maxpool_kernel(const float *__restrict__ x, int NC, int H, int W
 qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k, int s, float *y,
                            cudaStream_t st) {
     const int Ho = (H - k) / s + 1, Wo = (W - k) / s + 1;
-    const size_t total = (size_t)N * C * Ho * Wo;
-    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 16);
-    maxpool_kernel<<<blocks, 256, 0, st>>>(x, N * C, H, W, k, s, Ho, Wo, y);
+    const int total = N * C * Ho * Wo;
+    const int blocks = std::max(1, std::min((total + 255) / 256, num_sms() * 8));
+    maxpool_kernel<<<blocks, 256, 0, st>>>(x, total, H, W, k, s, Ho, Wo, y);
     return after_launch();
 }
 
