@@ -54,9 +54,12 @@ __host__ __device__ inline PhaseSmem phase_smem_layout(int K, int KS, int xs_flo
 }
 
 // P: 32-position slots per warp; CTW: channels per warp (even);
-// CSP4: C'_s register width (4 or 8); NW: warps per CTA.
-template <int P, int CTW, int CSP4, int NW>
+// CSP4: C'_s register width (4 or 8); CSPE: C'_s itself when the variant is
+// made for one value (the build then skips the zero slots), else CSP4;
+// NW: warps per CTA.
+template <int P, int CTW, int CSP4, int CSPE, int NW>
 __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs a) {
+    static_assert(CSPE >= 1 && CSPE <= CSP4, "C'_s width");
     constexpr int NT = NW * 32;
     constexpr int ST = P * 32;
     constexpr int CT_CTA = NW * CTW;
@@ -153,7 +156,7 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
                     const int k = q0 + 32 * i + lane;
                     float v = 0.f;
 #pragma unroll
-                    for (int j = 0; j < CSP4; ++j) v = fmaf(xv[j], dk[i][j], v);
+                    for (int j = 0; j < CSPE; ++j) v = fmaf(xv[j], dk[i][j], v);
                     if (k < K) lut[k * KS + h] = v;
                 }
             }
@@ -172,12 +175,12 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
     auto gather = [&](int u) {
         const int m = u / S2, ph = u - m * S2, ay = ph / s, ax = ph - ay * s;
         const uint8_t *cb = cs + (size_t)(m & 1) * kk * CT_CTA + warp * CTW;
-        // first kernel row / column of the phase: (ky - pad) % s == ay
+        // first kernel row / column of the phase: (ky - pad) % s == ay; the
+        // offset (dy, dx) then steps by one with each further row / column
         const int ky0 = (ay + a.pad) % s, kx0 = (ax + a.pad) % s;
-        for (int ky = ky0; ky < a.kh; ky += s) {
-            const int dy = (ky - a.pad - ay) / s;  // exact
-            for (int kx = kx0; kx < a.kw; kx += s) {
-                const int dx = (kx - a.pad - ax) / s;
+        const int dy0 = (ky0 - a.pad - ay) / s, dx0 = (kx0 - a.pad - ax) / s;  // exact
+        for (int ky = ky0, dy = dy0; ky < a.kh; ky += s, ++dy) {
+            for (int kx = kx0, dx = dx0; kx < a.kw; kx += s, ++dx) {
                 const int pk = ky * a.kw + kx;
                 // the warp's CTW codes: 32-bit words, or 16-bit pairs when
                 // CTW is not a multiple of 4; clamped into [0, K)
@@ -249,20 +252,21 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
 
 // ---------------------------------------------------------- variant table --
 struct PhaseVariant {
-    int P, CTW, CSP4, NW;
+    int P, CTW, CSP4, CSPE, NW;
     void (*fn)(PhaseArgs);
 };
-#define QCNN_PHASE(P, CTW, C4, NW) {P, CTW, C4, NW, conv_phase_kernel<P, CTW, C4, NW>}
+#define QCNN_PHASE(P, CTW, C4, CE, NW) {P, CTW, C4, CE, NW, conv_phase_kernel<P, CTW, C4, CE, NW>}
 static const PhaseVariant kPhase[] = {
-    QCNN_PHASE(7, 6, 4, 16),   // 96 channels (AlexNet conv1), 224 positions
-    QCNN_PHASE(7, 8, 4, 12),
-    QCNN_PHASE(6, 8, 4, 12),
-    QCNN_PHASE(4, 8, 4, 12),
-    QCNN_PHASE(6, 8, 4, 16),   // 128 channels
-    QCNN_PHASE(4, 16, 4, 16),  // 256 channels
-    QCNN_PHASE(6, 8, 8, 12),
-    QCNN_PHASE(6, 8, 8, 16),
-    QCNN_PHASE(4, 16, 8, 16),
+    QCNN_PHASE(7, 6, 4, 3, 16),   // C'_s = 3, 96 channels (AlexNet conv1), 224 positions
+    QCNN_PHASE(7, 6, 4, 4, 16),
+    QCNN_PHASE(7, 8, 4, 4, 12),
+    QCNN_PHASE(6, 8, 4, 4, 12),
+    QCNN_PHASE(4, 8, 4, 4, 12),
+    QCNN_PHASE(6, 8, 4, 4, 16),   // 128 channels
+    QCNN_PHASE(4, 16, 4, 4, 16),  // 256 channels
+    QCNN_PHASE(6, 8, 8, 8, 12),
+    QCNN_PHASE(6, 8, 8, 8, 16),
+    QCNN_PHASE(4, 16, 8, 8, 16),
 };
 #undef QCNN_PHASE
 constexpr int kNumPhase = sizeof(kPhase) / sizeof(kPhase[0]);
@@ -297,7 +301,7 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s) {
     const int U = s.M * s.stride * s.stride;
     for (int v = 0; v < kNumPhase; ++v) {
         const PhaseVariant &pv = kPhase[v];
-        if (pv.CSP4 != csp4) continue;
+        if (pv.CSP4 != csp4 || s.Csp > pv.CSPE) continue;
         const int ST = pv.P * 32;
         const int HP = std::min(ST, npos) + reach;
         const int KS = phase_ks(ST + reach);
@@ -326,6 +330,8 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s) {
             }
             if (ctas * sp >= 2.0 * sms) break;
         }
+        // a variant made for this C'_s exactly is preferred at equal cost
+        if (pv.CSPE == s.Csp && pv.CSPE < pv.CSP4) score *= 0.97;
         if (!best.ok || score < best.score) {
             best.ok = true;
             best.variant = v;
