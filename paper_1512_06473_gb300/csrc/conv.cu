@@ -146,7 +146,7 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 // SK    : stream-K schedule (a persistent grid over (tile, sub-space) units)
 template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF, bool SK>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
-    static_assert(!SK || (!PIPE && !BF), "the stream-K schedule has one fp32 table buffer");
+    static_assert(!SK || !PIPE, "the stream-K schedule has one table buffer");
     constexpr int NT = NW * 32;
     constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     constexpr int CT_CTA = (NW / WP) * CTW;
@@ -417,7 +417,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 stage_codes(mn, b ^ 1, sct0);
                 cp_async_commit();
             }
-            build(b, lut0);
+            if constexpr (BF) build_bf16(b, lut0);
+            else build(b, lut0);
             __syncthreads();
             gather(b, lut0);
             if (last_of_tile || last_of_range) {
@@ -571,6 +572,9 @@ struct FusedVariant {
 #define QCNN_FUSED_SK(P, CTW, WP, C4, NW, MB, EFF, BLD) \
     {P, CTW, WP, C4, NW, MB, 0, 0, 1, EFF, BLD,         \
      conv_fused_kernel<P, CTW, WP, C4, NW, MB, false, false, true>}
+#define QCNN_FUSED_BF_SK(P, CTW, WP, C4, NW, MB, EFF, BLD) \
+    {P, CTW, WP, C4, NW, MB, 0, 1, 1, EFF, BLD,            \
+     conv_fused_kernel<P, CTW, WP, C4, NW, MB, false, true, true>}
 #define QCNN_FUSED_SET(C4)                                                                       \
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
@@ -604,11 +608,16 @@ struct FusedVariant {
     QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0),   \
     QCNN_FUSED_SK(6, 8, 1, C4, 16, 1, 1.0, 1.0),   \
     QCNN_FUSED_SK(5, 16, 1, C4, 16, 1, 1.0, 1.0),  \
-    QCNN_FUSED_SK(6, 16, 1, C4, 12, 1, 1.0, 1.0)
+    QCNN_FUSED_SK(6, 16, 1, C4, 12, 1, 1.0, 1.0),  \
+    QCNN_FUSED_BF_SK(3, 16, 1, C4, 12, 1, 1.0, 1.3), /* bf16: a whole 13x13 map */ \
+    QCNN_FUSED_BF_SK(3, 8, 1, C4, 16, 1, 1.0, 1.3),                               \
+    QCNN_FUSED_BF_SK(2, 16, 1, C4, 16, 1, 1.0, 1.3),                              \
+    QCNN_FUSED_BF_SK(4, 8, 1, C4, 16, 1, 1.0, 1.3)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
                                       QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
                                       QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};
 #undef QCNN_FUSED_SK_SET
+#undef QCNN_FUSED_BF_SK
 #undef QCNN_FUSED_SK
 #undef QCNN_FUSED_BF_SET
 #undef QCNN_FUSED_SET
