@@ -601,8 +601,8 @@ struct FusedVariant {
     QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, false, 0.97, 1.3),                          \
     QCNN_FUSED_BF(4, 8, 1, C4, 16, 1, true, 0.6, 0.4),                             \
     QCNN_FUSED_BF(2, 16, 1, C4, 16, 1, true, 0.6, 0.4)
-// stream-K schedules of the fp32 tiles that win on grids with a short last
-// wave (AlexNet's 13x13 layers); bf16 tables gained nothing from it
+// stream-K schedules of the tiles that win on grids with a short last wave
+// (AlexNet's 27x27 and 13x13 layers), fp32 and bf16 tables
 #define QCNN_FUSED_SK_SET(C4)                      \
     QCNN_FUSED_SK(4, 16, 1, C4, 16, 1, 1.0, 1.0),  \
     QCNN_FUSED_SK(7, 8, 1, C4, 16, 1, 1.0, 1.0),   \
