@@ -61,7 +61,8 @@ typedef enum {
 typedef enum {
     QCNN_ALGO_AUTO = 0,    /* library picks: fused (stride 1), else phase,
                               else chunked, else unfused                     */
-    QCNN_ALGO_FUSED = 1,   /* full table rows of a band in shared memory, stride 1 only */
+    QCNN_ALGO_FUSED = 1,   /* full table rows of a tile of output positions in
+                              shared memory, stride 1 only                   */
     QCNN_ALGO_UNFUSED = 2, /* tables materialised in the workspace first      */
     QCNN_ALGO_CHUNKED = 3, /* table rows built KC sub-codewords at a time in
                               shared memory, any stride                      */
