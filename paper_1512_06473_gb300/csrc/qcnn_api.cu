@@ -297,6 +297,65 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
     return QCNN_OK;
 }
 
+// Net plans are cached per (device, batch, input shape, layer shapes and
+// options): planning a stack costs tens of microseconds on the host, which is
+// a tenth of a batch-1 forward.  Layer pointers only enter the key as
+// NULL / non-NULL (the plan depends on shapes alone).  At most kPlanCache
+// entries, oldest replaced first; the mutex guards the table.
+constexpr size_t kPlanCache = 16;
+struct PlanKey {
+    std::vector<int> v;
+    bool operator==(const PlanKey &o) const { return v == o.v; }
+};
+struct PlanCache {
+    std::mutex mu;
+    std::vector<std::pair<PlanKey, NetPlan>> entries;
+    size_t next = 0;
+};
+PlanCache &plan_cache() {
+    static PlanCache c;
+    return c;
+}
+
+qcnn_status plan_net_cached(const qcnn_layer *layers, int n_layers, int N, int C, int H, int W,
+                            int host_io, NetPlan *np) {
+    if (!layers || n_layers <= 0 || n_layers > 4096)
+        return plan_net(layers, n_layers, N, C, H, W, host_io, np);
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        dev = -1;
+    }
+    PlanKey key;
+    key.v.reserve(7 + 14 * (size_t)n_layers);
+    key.v.insert(key.v.end(), {dev, n_layers, N, C, H, W, host_io});
+    for (int i = 0; i < n_layers; ++i) {
+        const qcnn_layer &L = layers[i];
+        key.v.insert(key.v.end(), {L.kind, L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp, L.K, L.relu,
+                                   L.algo, L.codes_layout, L.lut_type, L.D != nullptr,
+                                   L.codes != nullptr});
+    }
+    PlanCache &pc = plan_cache();
+    {
+        std::lock_guard<std::mutex> g(pc.mu);
+        for (const auto &e : pc.entries)
+            if (e.first == key) {
+                *np = e.second;
+                return QCNN_OK;
+            }
+    }
+    const qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, host_io, np);
+    if (rc != QCNN_OK) return rc;
+    std::lock_guard<std::mutex> g(pc.mu);
+    if (pc.entries.size() < kPlanCache) {
+        pc.entries.emplace_back(std::move(key), *np);
+    } else {
+        pc.entries[pc.next] = {std::move(key), *np};
+        pc.next = (pc.next + 1) % kPlanCache;
+    }
+    return QCNN_OK;
+}
+
 qcnn_status run_step(const qcnn_layer &L, const NetStep &s, const float *in, float *out,
                      void *scratch, cudaStream_t st) {
     if (s.kind == QCNN_LAYER_CONV)
@@ -492,7 +551,7 @@ qcnn_status qcnn_net_output_shape(const qcnn_layer *layers, int n_layers, int C,
                                   int *out_C, int *out_H, int *out_W) {
     if (!out_C || !out_H || !out_W) return QCNN_ERR_INVALID_ARG;
     NetPlan np;
-    qcnn_status rc = plan_net(layers, n_layers, 1, C, H, W, 0, &np);
+    qcnn_status rc = plan_net_cached(layers, n_layers, 1, C, H, W, 0, &np);
     if (rc != QCNN_OK) return rc;
     *out_C = np.steps.back().oC;
     *out_H = np.steps.back().oH;
@@ -504,7 +563,7 @@ qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers, int 
                                     int W, int host_io, size_t *bytes) {
     if (!bytes) return QCNN_ERR_INVALID_ARG;
     NetPlan np;
-    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, host_io, &np);
+    qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, host_io, &np);
     if (rc != QCNN_OK) return rc;
     *bytes = np.total;
     return QCNN_OK;
@@ -515,7 +574,7 @@ qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers, const float
                              size_t workspace_bytes, void *stream) {
     if (!x || !y) return QCNN_ERR_INVALID_ARG;
     NetPlan np;
-    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, 0, &np);
+    qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, 0, &np);
     if (rc != QCNN_OK) return rc;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
     return run_net(layers, np, x, y, workspace, as_stream(stream));
@@ -526,7 +585,7 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
                                   size_t workspace_bytes, void *stream) {
     if (!x_host || !y_host) return QCNN_ERR_INVALID_ARG;
     NetPlan np;
-    qcnn_status rc = plan_net(layers, n_layers, N, C, H, W, 1, &np);
+    qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, 1, &np);
     if (rc != QCNN_OK) return rc;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);

@@ -198,7 +198,7 @@ def test_fused_variant_table():
         assert (NW // WP) * CTW % 16 == 0
         seen_sk |= bool(SK)
         seen_pipe |= bool(PIPE)
-        assert not (SK and (PIPE or BF))
+        assert not (SK and PIPE)  # stream-K runs one table buffer
         seen_bf |= bool(BF)
     assert seen_sk and seen_pipe and seen_bf
     assert lib.qcnn_conv_fused_variant_info(n, info) == _lib.ERR_INVALID_ARG
