@@ -98,18 +98,22 @@ constexpr int kEccThreads = 256;
 constexpr int kEccStat = kMaxCsp * kMaxCsp + kMaxCsp;  // G (Csp x Csp) + V (Csp)
 
 // Block reduction of `cnt` doubles per thread into vals[0..cnt) of thread 0,
-// in a fixed tree order.
+// in a fixed order: a shuffle tree inside each warp, then the warps' sums in
+// warp order.  sh holds kEccStat doubles per warp.
 __device__ void ecc_block_reduce(double *vals, int cnt, double *sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     for (int c = 0; c < cnt; ++c) {
-        sh[threadIdx.x] = vals[c];
-        __syncthreads();
-        for (int s = blockDim.x / 2; s > 0; s >>= 1) {
-            if ((int)threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
-            __syncthreads();
-        }
-        if (threadIdx.x == 0) vals[c] = sh[0];
-        __syncthreads();
+        double v = vals[c];
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+        if (lane == 0) sh[warp * kEccStat + c] = v;
     }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (int c = 0; c < cnt; ++c) {
+            double t = sh[c];
+            for (int w = 1; w < nw; ++w) t += sh[w * kEccStat + c];
+            vals[c] = t;
+        }
 }
 
 // D pass, codeword k: per block, G_k and V over the segments b, b + B, ...
@@ -118,10 +122,11 @@ __global__ void __launch_bounds__(kEccThreads) ecc_dstats_kernel(
     const int *__restrict__ order, const int *__restrict__ seg_ct,
     const int *__restrict__ seg_start, const int *__restrict__ seg_len,
     const int *__restrict__ nseg, double *__restrict__ part) {
-    __shared__ double sh[kEccThreads];
+    __shared__ double sh[(kEccThreads / 32) * kEccStat];
     double acc[kEccStat];
     for (int c = 0; c < kEccStat; ++c) acc[c] = 0.0;
     const int ns = nseg[k];
+    if ((int)blockIdx.x >= ns) return;  // no segment for this block: its part is not read
     const int items = g.N * g.P;
     for (int sgi = blockIdx.x; sgi < ns; sgi += gridDim.x) {
         const int ct = seg_ct[(size_t)k * g.Ct + sgi];
@@ -166,27 +171,32 @@ __device__ bool ecc_cholesky(double *L, int n) {
     return true;
 }
 
-// D pass, codeword k: add the block parts in order, solve, update D_k;
-// delta = D_k,new - D_k,old (zero when k has no pairs).
+// D pass, codeword k: add the parts of the blocks that had segments, in
+// block order (one thread per statistic), solve, update D_k;
+// delta = D_k,new - D_k,old (zero when k has no pairs).  Launch with at least
+// kEccStat threads.
 __global__ void ecc_dsolve_kernel(EcConvGeo g, int m, int k, int nblocks,
                                   const double *__restrict__ part, const int *__restrict__ nseg,
                                   double *__restrict__ Dw, double *__restrict__ delta,
                                   int *__restrict__ flag) {
+    __shared__ double tot[kEccStat];
+    const int C = g.Csp, cnt = C * C + C;
+    const int nb = min(nblocks, nseg[k]);
+    for (int c = threadIdx.x; c < cnt; c += blockDim.x) {
+        double t = 0.0;
+        for (int blk = 0; blk < nb; ++blk) t += part[(size_t)blk * kEccStat + c];
+        tot[c] = t;
+    }
+    __syncthreads();
     if (threadIdx.x != 0) return;
-    const int C = g.Csp;
     double *d = Dw + ((size_t)m * g.K + k) * C;
     if (nseg[k] == 0) {
         for (int j = 0; j < C; ++j) delta[j] = 0.0;
         return;
     }
     double L[kMaxCsp * kMaxCsp], b[kMaxCsp];
-    for (int c = 0; c < C * C; ++c) L[c] = 0.0;
-    for (int j = 0; j < C; ++j) b[j] = 0.0;
-    for (int blk = 0; blk < nblocks; ++blk) {
-        const double *p = part + (size_t)blk * kEccStat;
-        for (int c = 0; c < C * C; ++c) L[c] += p[c];
-        for (int j = 0; j < C; ++j) b[j] += p[C * C + j];
-    }
+    for (int c = 0; c < C * C; ++c) L[c] = tot[c];
+    for (int j = 0; j < C; ++j) b[j] = tot[C * C + j];
     if (!ecc_cholesky(L, C)) {
         *flag = 1;
         for (int j = 0; j < C; ++j) delta[j] = 0.0;
@@ -521,7 +531,7 @@ qcnn_status qcnn_ec_quantize_conv(const float *S, const float *T, int N, int Cs,
                     ecc_dstats_kernel<<<kEccBlocks, kEccThreads, 0, st>>>(
                         S, g, m, k, E, order, seg_ct, seg_start, seg_len, nseg, part);
                     if ((rc = chk()) != QCNN_OK) return rc;
-                    ecc_dsolve_kernel<<<1, 32, 0, st>>>(g, m, k, kEccBlocks, part, nseg, Dw, delta,
+                    ecc_dsolve_kernel<<<1, 96, 0, st>>>(g, m, k, kEccBlocks, part, nseg, Dw, delta,
                                                         flag);
                     if ((rc = chk()) != QCNN_OK) return rc;
                     ecc_dupdate_kernel<<<kEccBlocks, kEccThreads, 0, st>>>(
