@@ -167,6 +167,32 @@ def test_net_rejects_mismatched_layer():
         == _lib.ERR_INVALID_ARG
 
 
+def test_net_plan_cache_keys_on_every_planning_input():
+    """Net plans are cached; a change of batch, host I/O, a layer option or a
+    NULL pointer must not be answered from the cache."""
+    w = synth.alexnet()
+    arr = _layers(w)
+    sizes = {}
+    for N in (1, 2, 128):
+        for host_io in (0, 1):
+            nb = ctypes.c_size_t()
+            for _ in range(2):  # the second call is served from the cache
+                assert lib.qcnn_net_workspace_size(arr, len(arr), N, 3, 227, 227, host_io,
+                                                   ctypes.byref(nb)) == 0
+                sizes.setdefault((N, host_io), nb.value)
+                assert sizes[(N, host_io)] == nb.value
+    assert len(set(sizes.values())) == len(sizes)
+    a, b = ctypes.c_size_t(), ctypes.c_size_t()
+    assert lib.qcnn_net_workspace_size(arr, len(arr), 1, 3, 227, 227, 0, ctypes.byref(a)) == 0
+    arr[0].algo = 2  # conv1 through the unfused path: its tables live in the workspace
+    assert lib.qcnn_net_workspace_size(arr, len(arr), 1, 3, 227, 227, 0, ctypes.byref(b)) == 0
+    assert b.value > a.value
+    arr[0].algo = 0
+    arr[4].D = None
+    assert lib.qcnn_net_workspace_size(arr, len(arr), 1, 3, 227, 227, 0, ctypes.byref(b)) \
+        == _lib.ERR_INVALID_ARG
+
+
 def test_quantizer_argument_checks():
     nb = ctypes.c_size_t()
     FC, CONV = _lib.LAYER_FC, _lib.LAYER_CONV
