@@ -34,9 +34,10 @@
  *    then unspecified.
  *  - A failed launch returns QCNN_ERR_CUDA; the CUDA error is in
  *    qcnn_last_cuda_error().  The library is stateless apart from that
- *    value, a launch counter and, per device, the copy stream and events of
- *    qcnn_net_forward_host (created on its first call), and is safe to call
- *    from several threads.
+ *    value, a launch counter, a cache of qcnn_net_* plans (keyed by device,
+ *    batch, input shape and the layers' shapes and options) and, per device,
+ *    the copy stream and events of qcnn_net_forward_host (created on its
+ *    first call), and is safe to call from several threads.
  */
 #ifndef QCNN_H
 #define QCNN_H
