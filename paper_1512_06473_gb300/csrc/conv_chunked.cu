@@ -180,27 +180,28 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
                     if (QPT > 1 || tid > 0) h1[q - 1] = hv;
                 }
             }
-            return;
-        }
-        for (int kl = 0; kl < kc; ++kl) {
-            float dk[CSPT];
+        } else {
+            for (int kl = 0; kl < kc; ++kl) {
+                float dk[CSPT];
 #pragma unroll
-            for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
-            float *row = L + kl * g.SK + tid;
+                for (int j = 0; j < CSPT; ++j) dk[j] = ds[(k0 + kl) * CSPT + j];
+                float *row = L + kl * g.SK + tid;
 #pragma unroll
-            for (int qi = 0; qi + 1 < QPT; qi += 2) {
-                float2 v = make_float2(0.f, 0.f);
+                for (int qi = 0; qi + 1 < QPT; qi += 2) {
+                    float2 v = make_float2(0.f, 0.f);
 #pragma unroll
-                for (int j = 0; j < CSPT; ++j)
-                    v = __ffma2_rn(make_float2(xr[qi][j], xr[qi + 1][j]), make_float2(dk[j], dk[j]), v);
-                row[qi * kChunkThreads] = v.x;
-                row[(qi + 1) * kChunkThreads] = v.y;
-            }
-            if constexpr (QPT % 2 == 1) {
-                float v = 0.f;
+                    for (int j = 0; j < CSPT; ++j)
+                        v = __ffma2_rn(make_float2(xr[qi][j], xr[qi + 1][j]),
+                                       make_float2(dk[j], dk[j]), v);
+                    row[qi * kChunkThreads] = v.x;
+                    row[(qi + 1) * kChunkThreads] = v.y;
+                }
+                if constexpr (QPT % 2 == 1) {
+                    float v = 0.f;
 #pragma unroll
-                for (int j = 0; j < CSPT; ++j) v = fmaf(xr[QPT - 1][j], dk[j], v);
-                row[(QPT - 1) * kChunkThreads] = v;
+                    for (int j = 0; j < CSPT; ++j) v = fmaf(xr[QPT - 1][j], dk[j], v);
+                    row[(QPT - 1) * kChunkThreads] = v;
+                }
             }
         }
     };
