@@ -384,6 +384,52 @@ def extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N, ba
         oec.ec_quantize_fc(S, T, D0.cpu().numpy(), c0.cpu().numpy(), 1, 2)
         qres["oracle_ec_fc8_s"] = round(time.perf_counter() - t0, 3)
     res["quantizer"] = qres
+
+    # ---- the other workloads (parity cases of the tests), each net at its
+    # batches: forward time (L2 flushed), images/s, dense-equivalent GFLOP/s
+    # and the whole net's fraction of the shared-memory roofline
+    peak_smem = 152 * 128 * 2070e6
+    cfgs = {}
+    for name in sorted(synth.WORKLOADS):
+        wk = synth.WORKLOADS[name]
+        if name == w.name:
+            continue
+        pk = wk.params()
+        lay = []
+        for L, P in zip(wk.layers, pk):
+            if isinstance(L, synth.Conv):
+                codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
+                lay.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
+                                       torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
+                                       L.stride, L.pad, L.relu, packed=True))
+            elif isinstance(L, synth.FC):
+                lay.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
+                                     torch.from_numpy(P["codes"]).to(dev),
+                                     torch.from_numpy(P["bias"]).to(dev), L.relu))
+            else:
+                lay.append(q.PoolLayer(L.k, L.s))
+        in_shape = tuple(wk.in_shape) if len(wk.in_shape) == 3 else (wk.in_shape[0], 1, 1)
+        wnet = q.Net(lay, in_shape)
+        costs = _layer_costs(wk, cm)
+        dense = sum(c.dense_macs for c in costs)
+        alg = 4.0 * sum(c.lookups + c.lut_entries for c in costs)
+        per = []
+        for B in wk.batches:
+            xb = torch.from_numpy(wk.input(B, 3).reshape(B, *in_shape)).to(dev)
+            wws = wnet.alloc_workspace(B, dev)
+            wout = wnet._out(B, dev)
+            for _ in range(3):
+                wnet.forward(xb, out=wout, workspace=wws)
+            torch.cuda.synchronize(dev)
+            ms_b = event_ms(lambda: wnet.forward(xb, out=wout, workspace=wws), 10)
+            per.append({"batch": B, "ms": round(ms_b, 4), "images_per_s": round(B / (ms_b / 1e3), 1),
+                        "dense_equiv_gflops": round(2 * dense * B / (ms_b / 1e3) / 1e9, 1),
+                        "frac_smem": round(alg * B / (ms_b / 1e3) / peak_smem, 4)})
+        cfgs[name] = per
+    res["configs"] = {"note": "each workload's whole net, device-resident input, L2 flushed "
+                              "before every forward; frac_smem = 4 B x (look-ups + table "
+                              "entries) per second over 152 x 128 B x 2070 MHz",
+                      "workloads": cfgs}
     return res
 
 
