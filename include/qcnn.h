@@ -29,6 +29,11 @@
  *  - Limits: 1 <= Csp <= 8, 1 <= K <= 256, Cs % Csp == 0, every size > 0 and
  *    every element count below 2^31.  Outside them: QCNN_ERR_INVALID_ARG,
  *    returned before any work is enqueued.
+ *  - Alignment: fp32 arrays 4-byte aligned, bfloat16 tables 2-byte aligned,
+ *    PACKED code arrays (conv QCNN_CODES_PACKED, and FC rows from
+ *    qcnn_fc_pack_codes) 16-byte aligned; workspaces 256-byte aligned.  A
+ *    misaligned array gives QCNN_ERR_INVALID_ARG (a misaligned workspace
+ *    QCNN_ERR_WORKSPACE) before any work is enqueued.
  *  - Codes >= K are a caller error.  Kernels clamp every index into [0, K),
  *    so such codes never cause an out-of-bounds access, but the outputs are
  *    then unspecified.

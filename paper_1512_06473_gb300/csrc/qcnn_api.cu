@@ -54,6 +54,24 @@ inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s
 
 bool fits_int(long long v) { return v > 0 && v < (long long)INT_MAX; }
 
+// Device arrays are read with accesses of their element size (4-byte
+// cp.async for fp32) and PACKED code arrays with 16-byte copies, so a
+// misaligned pointer is refused on the host rather than faulting a kernel.
+// NULL passes (NULL-ness is checked where it matters).
+bool aligned(const void *p, uintptr_t a) { return reinterpret_cast<uintptr_t>(p) % a == 0; }
+bool f32_ok(const void *p) { return aligned(p, 4); }
+
+// The device pointers of every layer of a stack, for qcnn_net_forward*.
+bool layer_pointers_ok(const qcnn_layer *layers, int n) {
+    for (int i = 0; i < n; ++i) {
+        const qcnn_layer &L = layers[i];
+        if (L.kind == QCNN_LAYER_MAXPOOL) continue;
+        if (!f32_ok(L.D) || !f32_ok(L.bias)) return false;
+        if (L.codes_layout == QCNN_CODES_PACKED && !aligned(L.codes, 16)) return false;
+    }
+    return true;
+}
+
 bool pq_ok(int Cs, int Csp, int K) {
     return Cs > 0 && Csp >= 1 && Csp <= kMaxCsp && K >= 1 && K <= kMaxK && Cs % Csp == 0;
 }
@@ -446,6 +464,8 @@ qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W, const fl
     if (!x || !D || !lut || N <= 0 || H <= 0 || W <= 0 || !pq_ok(Cs, Csp, K) ||
         !lut_type_ok(lut_type))
         return QCNN_ERR_INVALID_ARG;
+    if (!f32_ok(x) || !f32_ok(D) || !aligned(lut, lut_type == QCNN_LUT_BF16 ? 2 : 4))
+        return QCNN_ERR_INVALID_ARG;
     const long long P = (long long)H * W;
     if (!fits_int((long long)N * Cs * P) || !fits_int((long long)N * (Cs / Csp) * P * K))
         return QCNN_ERR_INVALID_ARG;
@@ -468,6 +488,7 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct, const float *
     FcShape s;
     if (!x || !D || !codes || !y || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
+    if (!f32_ok(x) || !f32_ok(D) || !f32_ok(y) || !f32_ok(bias)) return QCNN_ERR_INVALID_ARG;
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
     return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(workspace),
@@ -481,7 +502,8 @@ qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const 
     FcShape s;
     if (!x || !D || !packed || !y || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
-    if (reinterpret_cast<uintptr_t>(packed) % 16 != 0) return QCNN_ERR_INVALID_ARG;
+    if (!aligned(packed, 16) || !f32_ok(x) || !f32_ok(D) || !f32_ok(y) || !f32_ok(bias))
+        return QCNN_ERR_INVALID_ARG;
     s.code_bits = code_bits(K);
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
@@ -532,6 +554,9 @@ qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int C
     if (!x || !D || !codes || !y ||
         !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
+    if (!f32_ok(x) || !f32_ok(D) || !f32_ok(y) || !f32_ok(bias) ||
+        (codes_layout == QCNN_CODES_PACKED && !aligned(codes, 16)))
+        return QCNN_ERR_INVALID_ARG;
     ConvCall c;
     qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
@@ -543,6 +568,7 @@ qcnn_status qcnn_maxpool(const float *x, int N, int C, int H, int W, int k, int 
                          void *stream) {
     if (!x || !y || N <= 0 || C <= 0 || H <= 0 || W <= 0 || k <= 0 || s <= 0 || k > H || k > W)
         return QCNN_ERR_INVALID_ARG;
+    if (!f32_ok(x) || !f32_ok(y)) return QCNN_ERR_INVALID_ARG;
     if (!fits_int((long long)N * C * H * W)) return QCNN_ERR_INVALID_ARG;
     return launch_maxpool(x, N, C, H, W, k, s, y, as_stream(stream));
 }
@@ -572,10 +598,11 @@ qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers, int 
 qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers, const float *x, int N,
                              int C, int H, int W, float *y, void *workspace,
                              size_t workspace_bytes, void *stream) {
-    if (!x || !y) return QCNN_ERR_INVALID_ARG;
+    if (!x || !y || !f32_ok(x) || !f32_ok(y)) return QCNN_ERR_INVALID_ARG;
     NetPlan np;
     qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, 0, &np);
     if (rc != QCNN_OK) return rc;
+    if (!layer_pointers_ok(layers, n_layers)) return QCNN_ERR_INVALID_ARG;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
     return run_net(layers, np, x, y, workspace, as_stream(stream));
 }
@@ -587,6 +614,7 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
     NetPlan np;
     qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, 1, &np);
     if (rc != QCNN_OK) return rc;
+    if (!layer_pointers_ok(layers, n_layers)) return QCNN_ERR_INVALID_ARG;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
     uint8_t *base = static_cast<uint8_t *>(workspace);

@@ -250,3 +250,52 @@ def test_forced_fused_variant_planning():
     strided = (1, 8, 15, 15, 4, 3, 3, 2, 1, 4, 16)
     assert lib.qcnn_conv_workspace_size(*strided, 0, _lib.ALGO_FUSED_VARIANT, 0,
                                         ctypes.byref(nb)) == _lib.ERR_UNSUPPORTED
+
+
+# The calls below pass made-up device addresses; each one must be refused by
+# the host-side checks.  On a machine with a GPU a missing check would launch
+# a kernel on them, so the test only runs where no device is visible.
+_no_device = pytest.mark.skipif(__import__("torch").cuda.is_available(),
+                                reason="passes made-up device addresses")
+
+
+@_no_device
+def test_misaligned_pointers_are_refused_before_launch():
+    A16, A4, ODD = 4096, 4100, 4098  # 16-byte aligned, 4-byte aligned, 2-byte aligned
+    INV = _lib.ERR_INVALID_ARG
+    PACKED = 1
+    # conv: fp32 arrays need 4-byte alignment, PACKED codes 16-byte alignment
+    conv = lambda x, D, codes, y, bias, layout: lib.qcnn_conv_forward(
+        x, 2, 8, 9, 9, 4, 3, 3, 1, 1, D, 4, 16, codes, layout, bias, y, 0, 0, 0, None, 0, None)
+    assert conv(A16, A16, A4, A16, None, PACKED) == INV
+    assert conv(ODD, A16, A16, A16, None, PACKED) == INV
+    assert conv(A16, ODD, A16, A16, None, PACKED) == INV
+    assert conv(A16, A16, A16, ODD, None, PACKED) == INV
+    assert conv(A16, A16, A16, A16, ODD, PACKED) == INV
+    # FC
+    fc = lambda x, D, codes, y, bias: lib.qcnn_fc_forward(x, 2, 12, 4, D, 3, 16, codes, bias, y,
+                                                           0, 0, None, 0, None)
+    assert fc(ODD, A16, A16, A16, None) == INV
+    assert fc(A16, A16, A16, A16, ODD) == INV
+    assert lib.qcnn_fc_forward_packed(A16, 2, 12, 4, A16, 3, 16, A4, None, A16, 0, 0, None, 0,
+                                      None) == INV
+    # table build: fp32 entries 4-byte, bfloat16 entries 2-byte aligned
+    assert lib.qcnn_lut_build(A16, 1, 12, 1, 1, A16, 3, 16, ODD, 0, None) == INV
+    assert lib.qcnn_lut_build(A16, 1, 12, 1, 1, A16, 3, 16, A16 + 1, 1, None) == INV
+    assert lib.qcnn_maxpool(ODD, 1, 4, 8, 8, 2, 2, A16, None) == INV
+    # a stack: the layers' D / bias and PACKED codes, and the net's x / y
+    w = synth.alexnet()
+    arr = _layers(w)
+    for L in arr:
+        if L.kind != 2:
+            L.D, L.codes, L.codes_layout = A16, A16, PACKED
+    nb = ctypes.c_size_t()
+    assert lib.qcnn_net_workspace_size(arr, len(arr), 1, 3, 227, 227, 0, ctypes.byref(nb)) == 0
+    assert lib.qcnn_net_forward(arr, len(arr), ODD, 1, 3, 227, 227, A16, None, 0, None) == INV
+    arr[2].codes = A4  # conv2's PACKED codes
+    assert lib.qcnn_net_forward(arr, len(arr), A16, 1, 3, 227, 227, A16, None, 0, None) == INV
+    arr[2].codes = A16
+    arr[len(arr) - 1].bias = ODD  # fc8's bias
+    host = (ctypes.c_float * 4)()
+    assert lib.qcnn_net_forward_host(arr, len(arr), ctypes.addressof(host), 1, 3, 227, 227,
+                                     ctypes.addressof(host), None, 0, None) == INV
