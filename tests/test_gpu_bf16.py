@@ -193,6 +193,7 @@ FC_BF16 = [
     (70, 2304, 513, 4, 32),     # many chunks, splits
     (1, 9216, 4096, 4, 32),     # fc6 at batch 1 (2-byte entries)
     (128, 4096, 1000, 4, 32),   # fc8 at batch 128
+    (100, 6144, 1030, 6, 64),   # 16 images per lane, ragged images and outputs
 ]
 
 

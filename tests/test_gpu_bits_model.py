@@ -41,6 +41,7 @@ def test_fc_pack_rows(M, Ct, K):
     (33, 128, 520, 4, 256),      # 8-bit codes
     (2, 64, 100, 8, 2),          # 1-bit codes
     (70, 2304, 513, 4, 5),       # 3-bit codes, splits
+    (100, 6144, 1030, 6, 64),    # 6-bit codes, 16 images per lane
 ])
 @pytest.mark.parametrize("lut", ["fp32", "bf16"])
 def test_fc_packed_codes_match_byte_codes(N, Cs, Ct, Csp, K, lut):

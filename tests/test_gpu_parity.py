@@ -161,6 +161,8 @@ FC_SWEEP = [
     (5, 40, 64, 1, 2),          # Csp = 1
     (70, 2304, 513, 4, 32),     # many chunks, splits
     (1, 9216, 4096, 4, 32),     # fc6 at batch 1
+    (128, 4096, 1000, 4, 32),   # fc8 at batch 128: 16 images x 4 outputs per lane
+    (100, 6144, 1030, 6, 64),   # the same tile, ragged images and outputs, C's = 6
 ]
 
 
