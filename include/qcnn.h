@@ -187,7 +187,7 @@ qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const 
                                    size_t workspace_bytes, void *stream);
 
 /*
- * qcnn_fc_forward_noalloc -- the same result as qcnn_fc_forward, for callers
+ * qcnn_fc_forward_noalloc -- the FC response of qcnn_fc_forward, for callers
  * that cannot hand the library any device memory: code running inside
  * another runtime's execution step, where that runtime owns all device
  * memory and forbids allocation, or a foreign-function caller with no device
@@ -197,9 +197,12 @@ qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const 
  *   process exits.  The call allocates nothing.  The first call on each
  *   device looks up the array's device address (cudaGetSymbolAddress), so
  *   make that first call before any stream capture.
- *   Limit: when qcnn_fc_workspace_size(...) for these sizes exceeds
- *   QCNN_FC_NOALLOC_SCRATCH_BYTES the call returns QCNN_ERR_WORKSPACE and
- *   enqueues nothing.
+ *   Plan: that of qcnn_fc_forward, except that no split count is used
+ *   whose partial sums would exceed QCNN_FC_NOALLOC_SCRATCH_BYTES (one
+ *   split needs none), so every size runs; where qcnn_fc_forward would
+ *   split further, this call is slower and its sums are added in another
+ *   order (a difference within fp32 rounding; identical plans give
+ *   bit-identical results).
  *   All calls share the array: calls that overlap on the GPU (different
  *   streams or host threads without ordering) race and give wrong results.
  *   Nothing in it needs clearing: each call writes what it reads back.

@@ -377,7 +377,7 @@ constexpr int kNumFc = sizeof(kFcVariants) / sizeof(kFcVariants[0]);
 // odd table-row pitch in the unit the kernel indexes (see FcArgs::NTP)
 static int fc_ntp(int NT, int bf16) { return (bf16 && NT % 2 == 0 ? NT / 2 : NT) | 1; }
 
-FcPlan plan_fc(const FcShape &s) {
+FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
     FcPlan best{};
     double best_t = 1e300;
     const int sms = num_sms();
@@ -410,6 +410,10 @@ FcPlan plan_fc(const FcShape &s) {
         const int tiles = n_tiles * ct_tiles;
         const int target = 2 * sms * cps_sm;
         int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
+        // at most max_partial_bytes of partial sums [splits][N][Ct]
+        const size_t per_split = (size_t)s.N * s.Ct * sizeof(float);
+        const size_t cap = max_partial_bytes / per_split;
+        if (splits > 1 && (size_t)splits > cap) splits = cap >= 2 ? (int)cap : 1;
         const int cpsplit = cdiv(n_chunks, splits);
         splits = cdiv(n_chunks, cpsplit);
         const double ctas = (double)tiles * splits;

@@ -50,20 +50,12 @@ qcnn_status scratch_address(void **out) {
 
 }  // namespace
 
+// The plan is qcnn_fc_forward's, except that split counts whose partial sums
+// would not fit the fixed scratch are not used (one split needs none).
 extern "C" qcnn_status qcnn_fc_forward_noalloc(const float *x, int N, int Cs, int Ct,
                                                const float *D, int Csp, int K,
                                                const uint8_t *codes, const float *bias,
                                                float *y, int relu, void *stream) {
-    size_t need = 0;
-    qcnn_status rc = qcnn_fc_workspace_size(N, Cs, Ct, Csp, K, QCNN_LUT_FP32, &need);
-    if (rc != QCNN_OK) return rc;
-    if (!x || !D || !codes || !y) return QCNN_ERR_INVALID_ARG;
-    if (need > kScratchBytes) return QCNN_ERR_WORKSPACE;  // larger than the fixed scratch
-    void *scratch = nullptr;
-    if (need > 0) {
-        rc = scratch_address(&scratch);
-        if (rc != QCNN_OK) return rc;
-    }
-    return qcnn_fc_forward(x, N, Cs, Ct, D, Csp, K, codes, bias, y, relu, QCNN_LUT_FP32, scratch,
-                           need, stream);
+    return qcnn::fc_forward_limited(x, N, Cs, Ct, D, Csp, K, codes, bias, y, relu, kScratchBytes,
+                                    scratch_address, reinterpret_cast<cudaStream_t>(stream));
 }

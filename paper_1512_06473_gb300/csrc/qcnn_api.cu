@@ -441,6 +441,28 @@ bool host_io_init(HostIo &h) {  // called with h.mu held
 
 }  // namespace
 
+namespace qcnn {
+
+qcnn_status fc_forward_limited(const float *x, int N, int Cs, int Ct, const float *D, int Csp,
+                               int K, const uint8_t *codes, const float *bias, float *y,
+                               int relu, size_t max_partial_bytes,
+                               qcnn_status (*get_scratch)(void **), cudaStream_t st) {
+    FcShape s;
+    if (!x || !D || !codes || !y || !fc_shape(N, Cs, Ct, Csp, K, QCNN_LUT_FP32, &s))
+        return QCNN_ERR_INVALID_ARG;
+    if (!f32_ok(x) || !f32_ok(D) || !f32_ok(y) || !f32_ok(bias)) return QCNN_ERR_INVALID_ARG;
+    const FcPlan p = plan_fc(s, max_partial_bytes);
+    void *scratch = nullptr;
+    if (p.partial_bytes > 0) {
+        if (p.partial_bytes > max_partial_bytes) return QCNN_ERR_WORKSPACE;
+        const qcnn_status rc = get_scratch(&scratch);
+        if (rc != QCNN_OK) return rc;
+    }
+    return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(scratch), st);
+}
+
+}  // namespace qcnn
+
 extern "C" {
 
 const char *qcnn_status_string(qcnn_status s) {

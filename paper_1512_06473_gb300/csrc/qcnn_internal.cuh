@@ -141,7 +141,16 @@ struct FcPlan {
     size_t smem;
     size_t partial_bytes;  // workspace for split partial sums (0 if splits == 1)
 };
-FcPlan plan_fc(const FcShape &s);
+// max_partial_bytes: no split count whose partial sums need more is chosen
+// (1 split, without partial sums, always fits)
+FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes = ~(size_t)0);
+// FC forward whose split partial sums live in caller-independent scratch of
+// at most max_partial_bytes; get_scratch is asked for its device address
+// only when the plan needs it (qcnn_fc_forward_noalloc)
+qcnn_status fc_forward_limited(const float *x, int N, int Cs, int Ct, const float *D, int Csp,
+                               int K, const uint8_t *codes, const float *bias, float *y,
+                               int relu, size_t max_partial_bytes,
+                               qcnn_status (*get_scratch)(void **), cudaStream_t st);
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x,
                       const float *D, const uint8_t *codes, const float *bias,
                       float *y, int relu, float *partial_ws, cudaStream_t st);
