@@ -713,7 +713,7 @@ def main():
         return 0
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "images/s", "n_gpus": world,
-        "steps": a.steps, "warmup": a.warmup, "ms_per_step": round(ms_per_step, 4),
+        "steps": a.steps, "warmup": max(a.warmup, 3), "ms_per_step": round(ms_per_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded images, random-init codebooks/codes/biases)",
         "config": {"workload": WORKLOAD, "global_batch": N * world, "per_gpu_batch": N,
