@@ -308,6 +308,24 @@ def test_net_forward_host_sliced_input():
         assert rel(yh.numpy(), dev) <= TOL
 
 
+@pytest.mark.parametrize("name", ["conv3x3_64x56x56_b1", "fc_512x256_b8", "alexnet_fc678"])
+def test_net_forward_host_sliced_single_layer_and_fc_first(name):
+    """Host input in four slices of 8 images for a one-layer stack (the
+    first layer's slices are the final output) and for stacks whose first
+    layer is FC (slices of flattened rows)."""
+    w = synth.WORKLOADS[name]
+    params = w.params()
+    net = build_net(w, params, packed=True)
+    N = 32
+    x = w.input(N, 7).reshape((N,) + net.in_shape)
+    dev = host(net.forward(cuda(x)))
+    xh = torch.from_numpy(x).pin_memory()
+    yh = torch.empty(dev.shape, dtype=torch.float32).pin_memory()
+    ws = net.alloc_workspace(N, host_io=True)
+    net.forward_host(xh, yh, ws)
+    assert rel(yh.numpy(), dev) <= TOL
+
+
 def test_launch_counter_counts_kernels():
     x = cuda(synth.normal((2, 32), 1.0, 1))
     D = cuda(synth.normal((8, 16, 4), 1.0, 2))
