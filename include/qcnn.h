@@ -159,6 +159,17 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
                             size_t workspace_bytes, void *stream);
 
 /*
+ * qcnn_fc_plan_info -- the plan qcnn_fc_forward (and qcnn_fc_forward_packed)
+ * would run, worked out on the host.  info receives: [0] images per CTA,
+ * [1] outputs per CTA, [2] CTAs sharing the sub-spaces of one tile (1: no
+ * partial sums), [3] sub-spaces per shared-memory chunk, [4] CTAs of the
+ * main kernel.  QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for a
+ * NULL info.
+ */
+qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K,
+                              int lut_type, int info[5]);
+
+/*
  * Bit-packed codes: the storage model of Table 1 (Sec. 3.4), each code in
  * b = qcnn_code_bits(K) = ceil(log2 K) bits (at least 1).  Stream layout:
  * code i occupies stream bits [i*b, (i+1)*b), its bit t at stream bit
@@ -254,6 +265,27 @@ qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W,
                               const float *bias, float *y, int relu, int algo,
                               int lut_type, void *workspace,
                               size_t workspace_bytes, void *stream);
+
+/*
+ * qcnn_conv_plan_info -- the launch plan qcnn_conv_forward would run for
+ * these arguments, worked out on the host like every plan (no work is
+ * enqueued and no device memory is touched).  It is for tests, tuning and
+ * logs.  info receives:
+ *   [0] the algorithm run: QCNN_ALGO_FUSED, _PHASE, _CHUNKED or _UNFUSED;
+ *   [1] its kernel variant (FUSED: the index of
+ *       qcnn_conv_fused_variant_info), -1 for UNFUSED;
+ *   [2] output positions per tile (FUSED, PHASE; else 0);
+ *   [3] output channels per CTA (0 for UNFUSED);
+ *   [4] CTAs sharing the sub-spaces of one tile (1: no partial sums);
+ *   [5] 1 when the FUSED kernel runs the stream-K schedule, else 0;
+ *   [6] CTAs of the main kernel (0 for UNFUSED).
+ * Errors are those of qcnn_conv_workspace_size, plus QCNN_ERR_INVALID_ARG
+ * for a NULL info.
+ */
+qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh,
+                                int kw, int stride, int pad, int Csp, int K,
+                                int codes_layout, int algo, int lut_type,
+                                int info[7]);
 
 /*
  * qcnn_maxpool -- k x k max-pool, stride s, no padding, floor output size

@@ -190,6 +190,34 @@ def fused_variants():
     return out
 
 
+_ALGO_NAMES = {v: k for k, v in _lib.ALGO.items()}
+
+
+def conv_plan(N, Cs, H, W, Ct, kh, kw, stride=1, pad=0, Csp=4, K=128, algo="auto",
+              packed=True, lut="fp32"):
+    """The plan conv_forward would run for these sizes (qcnn_conv_plan_info),
+    worked out on the host: a dict with the algorithm's name, its kernel
+    variant, positions per tile, channels per CTA, splits, stream-K and CTAs."""
+    a = _lib.ALGO[algo] if isinstance(algo, str) else _lib.ALGO_FUSED_VARIANT + int(algo)
+    info = (ctypes.c_int * 7)()
+    _lib.check(load().qcnn_conv_plan_info(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K,
+                                          _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL,
+                                          a, _lib.LUT[lut], info), "qcnn_conv_plan_info")
+    keys = ("algo", "variant", "positions", "channels", "splits", "stream_k", "ctas")
+    d = dict(zip(keys, list(info)))
+    d["algo"] = _ALGO_NAMES[d["algo"]]
+    return d
+
+
+def fc_plan(N, Cs, Ct, Csp=4, K=32, lut="fp32"):
+    """The plan fc_forward would run (qcnn_fc_plan_info): images and outputs
+    per CTA, splits, sub-spaces per chunk and CTAs."""
+    info = (ctypes.c_int * 5)()
+    _lib.check(load().qcnn_fc_plan_info(N, Cs, Ct, Csp, K, _lib.LUT[lut], info),
+               "qcnn_fc_plan_info")
+    return dict(zip(("images", "outputs", "splits", "chunk", "ctas"), list(info)))
+
+
 def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, algo="auto",
                  packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32"):
     """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,

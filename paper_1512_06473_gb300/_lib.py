@@ -50,6 +50,8 @@ _SIGS = {
                                      c_void_p]),
     "qcnn_conv_fused_variant_count": (c_int, []),
     "qcnn_conv_fused_variant_info": (c_int, [c_int, ctypes.POINTER(c_int)]),
+    "qcnn_conv_plan_info": (c_int, [c_int] * 14 + [ctypes.POINTER(c_int)]),
+    "qcnn_fc_plan_info": (c_int, [c_int] * 6 + [ctypes.POINTER(c_int)]),
     "qcnn_conv_workspace_size": (c_int, [c_int] * 14 + [ctypes.POINTER(c_size_t)]),
     "qcnn_conv_forward": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_int,
                                   c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int,

@@ -339,6 +339,7 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s) {
             best.dymin = dymin;
             best.dxmin = dxmin;
             best.HP = HP;
+            best.ST = ST;
             best.KS = KS;
             best.ct_cta = ct_cta;
             best.pos_tiles = pos_tiles;

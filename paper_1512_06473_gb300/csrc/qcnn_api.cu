@@ -567,6 +567,57 @@ qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh
     return QCNN_OK;
 }
 
+qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int kw, int stride,
+                                int pad, int Csp, int K, int codes_layout, int algo,
+                                int lut_type, int info[7]) {
+    ConvShape s;
+    if (!info || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
+        return QCNN_ERR_INVALID_ARG;
+    ConvCall c;
+    const qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    if (rc != QCNN_OK) return rc;
+    for (int i = 0; i < 7; ++i) info[i] = 0;
+    info[0] = c.algo;
+    if (c.algo == QCNN_ALGO_FUSED) {
+        const ConvFusedPlan &p = c.fp;
+        info[1] = p.variant;
+        info[2] = p.ST;
+        info[3] = p.ct_cta;
+        info[4] = p.splits;
+        info[5] = p.sk;
+        info[6] = p.sk ? p.sk_ctas : p.pos_tiles * p.ct_tiles * s.N * p.splits;
+    } else if (c.algo == QCNN_ALGO_PHASE) {
+        const ConvPhasePlan &p = c.pp;
+        info[1] = p.variant;
+        info[2] = p.ST;
+        info[3] = p.ct_cta;
+        info[4] = p.splits;
+        info[6] = p.pos_tiles * p.ct_tiles * s.N * p.splits;
+    } else if (c.algo == QCNN_ALGO_CHUNKED) {
+        const ConvChunkPlan &p = c.cp;
+        info[1] = p.variant;
+        info[3] = p.ct_cta;
+        info[4] = 1;
+        info[6] = p.row_tiles * p.ct_tiles * s.N;
+    } else {
+        info[1] = -1;
+        info[4] = 1;
+    }
+    return QCNN_OK;
+}
+
+qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_type, int info[5]) {
+    FcShape s;
+    if (!info || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s)) return QCNN_ERR_INVALID_ARG;
+    const FcPlan p = plan_fc(s);
+    info[0] = p.NT;
+    info[1] = p.CT_CTA;
+    info[2] = p.splits;
+    info[3] = p.MCH;
+    info[4] = p.ct_tiles * p.n_tiles * p.splits;
+    return QCNN_OK;
+}
+
 qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int Ct, int kh,
                               int kw, int stride, int pad, const float *D, int Csp, int K,
                               const uint8_t *codes, int codes_layout, const float *bias,

@@ -87,6 +87,7 @@ struct ConvPhasePlan {
     bool ok = false;
     int variant = -1;
     int pitch, dymin, dxmin, HP, KS, ct_cta, pos_tiles, ct_tiles;
+    int ST = 0;                           // output positions per tile
     int splits = 1, units_per_split = 0;  // (sub-space, phase) units per CTA
     size_t partial_bytes = 0;             // workspace for split partial sums
     size_t smem;

@@ -299,3 +299,72 @@ def test_misaligned_pointers_are_refused_before_launch():
     host = (ctypes.c_float * 4)()
     assert lib.qcnn_net_forward_host(arr, len(arr), ctypes.addressof(host), 1, 3, 227, 227,
                                      ctypes.addressof(host), None, 0, None) == INV
+
+
+# ---- the planners' choices (host only) ------------------------------------
+# The plans the measured launch list of the AlexNet-shaped benchmark shows
+# (batch 128) and the batch-1 split plans, pinned so that a planner change
+# that moves a layer off its measured-best kernel fails here, without a GPU.
+# Without a device the planners assume GB300's 152 SMs and 227 KB of shared
+# memory per block; another GPU would plan differently.
+def _gb300_or_no_device():
+    torch = __import__("torch")
+    return (not torch.cuda.is_available()
+            or torch.cuda.get_device_properties(0).multi_processor_count == 152)
+
+
+_planner = pytest.mark.skipif(not _gb300_or_no_device(), reason="plans are for 152 SMs")
+ALEX_CONV = {"conv1": (3, 227, 227, 96, 11, 11, 4, 0, 3), "conv2": (96, 27, 27, 256, 5, 5, 1, 2, 4),
+             "conv3": (256, 13, 13, 384, 3, 3, 1, 1, 4), "conv4": (384, 13, 13, 384, 3, 3, 1, 1, 4),
+             "conv5": (384, 13, 13, 256, 3, 3, 1, 1, 4)}
+ALEX_FC = {"fc6": (9216, 4096), "fc7": (4096, 4096), "fc8": (4096, 1000)}
+
+
+@_planner
+def test_alexnet_batch128_plans():
+    import paper_1512_06473_gb300 as q
+    V = q.fused_variants()
+    p = q.conv_plan(128, *ALEX_CONV["conv1"], K=128)
+    assert (p["algo"], p["positions"], p["channels"], p["splits"]) == ("phase", 224, 96, 1)
+    assert p["ctas"] == 14 * 128  # 14 tiles of 224 positions of the pitch-57 phase grid
+    want = {"conv2": (5, 16, 16), "conv3": (6, 16, 12), "conv4": (6, 16, 12), "conv5": (6, 8, 16)}
+    for name, (P, CTW, NW) in want.items():
+        p = q.conv_plan(128, *ALEX_CONV[name], K=128)
+        v = V[p["variant"]]
+        assert p["algo"] == "fused" and p["stream_k"] == 1 and p["ctas"] == 152, name
+        assert (v["P"], v["CTW"], v["NW"], v["SK"], v["BF"]) == (P, CTW, NW, 1, 0), name
+        assert p["channels"] == CTW * NW and p["positions"] == 32 * P
+    for name, (Cs, Ct) in ALEX_FC.items():
+        f = q.fc_plan(128, Cs, Ct)
+        assert (f["images"], f["outputs"]) == (16, 1024), name
+        assert f["splits"] > 1 and f["ctas"] == f["splits"] * 8 * -(-Ct // 1024)
+
+
+@_planner
+def test_batch1_plans_split_the_subspaces():
+    import paper_1512_06473_gb300 as q
+    for name, shape in ALEX_CONV.items():
+        p = q.conv_plan(1, *shape, K=128)
+        assert p["algo"] == ("phase" if name == "conv1" else "fused"), name
+        assert p["splits"] > 1 and p["stream_k"] == 0 and p["ctas"] >= 64, (name, p)
+    for name, (Cs, Ct) in ALEX_FC.items():
+        f = q.fc_plan(1, Cs, Ct)
+        assert f["images"] == 1 and f["splits"] >= 64, (name, f)
+
+
+def test_plan_info_arguments():
+    info7, info5 = (ctypes.c_int * 7)(), (ctypes.c_int * 5)()
+    args = (2, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 1)
+    assert lib.qcnn_conv_plan_info(*args, 0, 0, None) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_conv_plan_info(*args, 0, 0, info7) == _lib.OK
+    assert info7[0] == 1 and info7[4] >= 1  # fused, stride 1
+    # the fused kernel is stride-1 only; the unfused path has no bfloat16 tables
+    assert lib.qcnn_conv_plan_info(2, 8, 9, 9, 4, 3, 3, 2, 1, 4, 16, 1, 1, 0, info7) \
+        == _lib.ERR_UNSUPPORTED
+    assert lib.qcnn_conv_plan_info(*args, 2, 1, info7) == _lib.ERR_UNSUPPORTED
+    assert lib.qcnn_conv_plan_info(*args, 2, 0, info7) == _lib.OK
+    assert (info7[0], info7[1], info7[6]) == (2, -1, 0)
+    assert lib.qcnn_fc_plan_info(2, 12, 4, 3, 16, 0, None) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_plan_info(2, 10, 4, 3, 16, 0, info5) == _lib.ERR_INVALID_ARG
+    assert lib.qcnn_fc_plan_info(2, 12, 4, 3, 16, 0, info5) == _lib.OK
+    assert info5[4] == info5[2] * -(-2 // info5[0]) * -(-4 // info5[1])
