@@ -444,6 +444,38 @@ def _layer_costs(w, cm):
     return costs
 
 
+def stage_rooflines(w, cm, stage_ms, N, smem_gbs, hbm_gbs):
+    """Per-layer fraction of the stage roofline at batch N.  The roof time is
+    the slower of two: the algorithmic shared-memory bytes (4 B per look-up and
+    per table entry, Table 1 counts) at the shared-memory peak, and the
+    algorithmic HBM bytes (input and output activations once, one byte per
+    code, the sub-codebooks) at the measured copy bandwidth.  At batch 1 the
+    FC layers are HBM-bound (their codes), the conv layers shared-memory
+    bound; a max-pool is HBM-bound."""
+    out = []
+    for j, (L, (sin, sout)) in enumerate(zip(w.layers, w.shapes())):
+        t = stage_ms[j] / 1e3
+        act = 4.0 * N * (math.prod(sin) + math.prod(sout))
+        if isinstance(L, synth.Pool):
+            out.append({"layer": j, "kind": "maxpool", "ms": round(stage_ms[j], 4),
+                        "bound": "hbm", "frac": round(act / (hbm_gbs * 1e9) / t, 4)})
+            continue
+        M = L.Cs // L.Csp
+        if isinstance(L, synth.Conv):
+            c = cm.conv_cost(L.Cs, L.Ct, sin[1], sin[2], L.kh, L.kw, sout[1], sout[2], L.Csp,
+                             L.K)
+            codes = L.Ct * L.kh * L.kw * M
+        else:
+            c = cm.fc_cost(L.Cs, L.Ct, L.Csp, L.K)
+            codes = L.Ct * M
+        t_hbm = (act + codes + 4.0 * M * L.K * L.Csp) / (hbm_gbs * 1e9)
+        t_smem = 4.0 * N * (c.lookups + c.lut_entries) / (smem_gbs * 1e9)
+        out.append({"layer": j, "kind": L.kind, "ms": round(stage_ms[j], 4),
+                    "bound": "hbm" if t_hbm > t_smem else "smem",
+                    "frac": round(max(t_hbm, t_smem) / t, 4)})
+    return out
+
+
 def main():
     a = parse()
     if a.impl == "reference":
@@ -668,6 +700,10 @@ def main():
     b1 = batch1(net)
     bufs1 = [torch.empty((1, *sout), dtype=torch.float32, device=dev) for (sin, sout) in shapes]
     b1["stage_ms"] = [round(t, 4) for t in stage_times(layers, "fp32", x1, bufs1)]
+    hbm_gbs = float(peaks.get("hbm_gbs") or 6800.0)
+    b1["stages"] = stage_rooflines(w, cm, b1["stage_ms"], 1, smem_peak_gbs, hbm_gbs)
+    b1["roofline_note"] = (f"per stage: the slower of shared-memory bytes at {smem_peak_gbs:.0f} "
+                           f"GB/s and HBM bytes at {hbm_gbs:.0f} GB/s (measured copy)")
 
     # ---- bfloat16 tables: the same workload and timing, lut="bf16"
     bf_layers = make_layers("bf16")
