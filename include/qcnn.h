@@ -60,8 +60,11 @@ typedef enum {
     QCNN_ERR_UNSUPPORTED = 2, /* valid request this build cannot serve      */
     QCNN_ERR_WORKSPACE = 3,   /* workspace smaller than the query asked for */
     QCNN_ERR_CUDA = 4,        /* a CUDA call or kernel launch failed        */
-    QCNN_ERR_DATA = 5         /* input data unusable (rank-deficient
+    QCNN_ERR_DATA = 5,        /* input data unusable (rank-deficient
                                  calibration set of qcnn_ec_quantize_fc)    */
+    QCNN_ERR_DEVICE_CHECK = 6 /* debug builds: a kernel found a code >= K or
+                                 an index outside its arrays (see
+                                 qcnn_device_check)                         */
 } qcnn_status;
 
 typedef enum {
@@ -122,6 +125,35 @@ int qcnn_last_cuda_error(void);
 
 /* Number of kernels this library has launched in this process so far. */
 uint64_t qcnn_launch_count(void);
+
+/*
+ * Device checks of the debug build.  The library can be built with
+ * QCNN_DEBUG_CHECKS (libqcnn_debug.so); its kernels then test, as they run,
+ * what the release kernels only clamp:
+ *   QCNN_CHECK_CODE   a code >= K was read (the codes k_m(c_t) of Eq. 5 and
+ *                     k_m(c_t, p_k) of Eq. 7 index K sub-codewords);
+ *   QCNN_CHECK_TABLE  a look-up-table read in shared memory fell outside the
+ *                     table the kernel built;
+ *   QCNN_CHECK_GLOBAL a device-memory access fell outside its array.
+ * A kernel that finds one ORs its bit into a device record and carries on
+ * with the clamped value, so nothing faults.  The record is read, and
+ * cleared, at the next synchronizing call: qcnn_device_check below, and the
+ * calls that synchronize their stream anyway (qcnn_net_forward_host,
+ * qcnn_ec_quantize_fc, qcnn_ec_quantize_conv, qcnn_model_upload), which then
+ * return QCNN_ERR_DEVICE_CHECK instead of QCNN_OK.
+ *
+ * qcnn_debug_checks: 1 in a debug build, 0 in a release build.
+ * qcnn_device_check: synchronizes `stream`; returns QCNN_ERR_DEVICE_CHECK
+ *   when the record holds any bit (stored in *flags when flags is not NULL),
+ *   and clears it.  In a release build it only synchronizes (*flags = 0).
+ *   The record is per process and device-wide: work on other streams since
+ *   the last check is included.
+ */
+#define QCNN_CHECK_CODE 1u
+#define QCNN_CHECK_TABLE 2u
+#define QCNN_CHECK_GLOBAL 4u
+int qcnn_debug_checks(void);
+qcnn_status qcnn_device_check(void *stream, unsigned *flags);
 
 /*
  * qcnn_lut_build -- the look-up tables alone (Sec. 3.1, the paragraph after
@@ -207,7 +239,11 @@ qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const 
  *   the library, held in the memory of every GPU that loads it until the
  *   process exits.  The call allocates nothing.  The first call on each
  *   device looks up the array's device address (cudaGetSymbolAddress), so
- *   make that first call before any stream capture.
+ *   make that first call before any stream capture.  The address is kept
+ *   per device together with the id of the CUDA context it belongs to; if
+ *   that context is replaced (cudaDeviceReset, or any teardown of the
+ *   primary context), the next call looks it up again, and that call too
+ *   must then come before any stream capture.
  *   Plan: that of qcnn_fc_forward, except that no split count is used
  *   whose partial sums would exceed QCNN_FC_NOALLOC_SCRATCH_BYTES (one
  *   split needs none), so every size runs; where qcnn_fc_forward would

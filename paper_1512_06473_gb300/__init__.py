@@ -22,13 +22,14 @@ from typing import List, Optional, Sequence
 import torch
 
 from . import _lib
-from ._lib import QcnnError, load  # noqa: F401
+from ._lib import QcnnError, load, set_debug  # noqa: F401
 
 __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpool",
            "kmeans", "pq_quantize_fc", "pq_quantize_conv", "ec_quantize_fc", "ec_quantize_conv",
            "code_bits", "pack_bits", "unpack_bits", "fc_pack_codes", "serialize_model",
            "model_info", "load_model",
-           "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load"]
+           "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load",
+           "set_debug", "debug_checks", "device_check"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -58,6 +59,24 @@ def _workspace(nbytes: int, device, workspace: Optional[torch.Tensor]):
     ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
     off = (-ws.data_ptr()) % 256
     return ws[off:off + nbytes], nbytes
+
+
+def debug_checks() -> bool:
+    """True when the binding calls the debug build (set_debug(True))."""
+    return bool(load().qcnn_debug_checks())
+
+
+def device_check(stream=None) -> int:
+    """Synchronize the stream and return the debug build's device-check flags
+    since the last check (QCNN_CHECK_CODE 1: a code >= K was read;
+    QCNN_CHECK_TABLE 2: a table read outside the built table;
+    QCNN_CHECK_GLOBAL 4: a device-memory access outside its array), clearing
+    them.  Always 0 with the release build."""
+    flags = ctypes.c_uint(0)
+    st = load().qcnn_device_check(_stream(stream), ctypes.byref(flags))
+    if st not in (_lib.OK, _lib.ERR_DEVICE_CHECK):
+        _lib.check(st, "qcnn_device_check")
+    return int(flags.value)
 
 
 def launch_count() -> int:

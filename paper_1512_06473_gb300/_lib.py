@@ -12,6 +12,8 @@ from . import build as _build
 c_int, c_size_t, c_void_p, c_uint64 = ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_uint64
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_DATA = 0, 1, 2, 3, 4, 5
+ERR_DEVICE_CHECK = 6
+CHECK_CODE, CHECK_TABLE, CHECK_GLOBAL = 1, 2, 4  # qcnn_device_check flag bits
 ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3, "phase": 4}
 ALGO_FUSED_VARIANT = 256  # + v: fused tile variant v
 CODES_CANONICAL, CODES_PACKED = 0, 1
@@ -37,6 +39,8 @@ _SIGS = {
     "qcnn_status_string": (ctypes.c_char_p, [c_int]),
     "qcnn_last_cuda_error": (c_int, []),
     "qcnn_launch_count": (c_uint64, []),
+    "qcnn_debug_checks": (c_int, []),
+    "qcnn_device_check": (c_int, [c_void_p, ctypes.POINTER(ctypes.c_uint)]),
     "qcnn_lut_build": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                                c_void_p, c_int, c_void_p]),
     "qcnn_fc_workspace_size": (c_int, [c_int, c_int, c_int, c_int, c_int, c_int,
@@ -100,7 +104,9 @@ _SIGS = {
 }
 
 _lock = threading.Lock()
-_lib = None
+_lib = None          # the library the binding calls (release unless debug is on)
+_release = None
+_debug = None
 
 
 def header_functions(path: str | None = None):
@@ -111,21 +117,43 @@ def header_functions(path: str | None = None):
     return sorted(set(re.findall(r"\b(qcnn_[a-z0-9_]+)\s*\(", text)))
 
 
+def _bind(so: str):
+    lib = ctypes.CDLL(so)
+    for name, (res, args) in _SIGS.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
 def load(path: str | None = None):
-    """Load (building first when the sources are newer) and bind libqcnn.so."""
-    global _lib
+    """The bound library the binding calls: libqcnn.so (built first when the
+    sources are newer), or the debug build after set_debug(True).  With a
+    path, bind that file and return it without making it current."""
+    global _lib, _release
     with _lock:
-        if _lib is not None and path is None:
-            return _lib
-        so = path or _build.build()
-        lib = ctypes.CDLL(so)
-        for name, (res, args) in _SIGS.items():
-            f = getattr(lib, name)
-            f.restype = res
-            f.argtypes = args
-        if path is None:
-            _lib = lib
-        return lib
+        if path is not None:
+            return _bind(path)
+        if _lib is None:
+            _release = _bind(_build.build())
+            _lib = _release
+        return _lib
+
+
+def set_debug(enabled: bool):
+    """Route every later call of the binding to libqcnn_debug.so (the build
+    whose kernels record codes >= K and out-of-range indices, read back by
+    device_check) or back to libqcnn.so."""
+    global _lib, _release, _debug
+    with _lock:
+        if enabled:
+            if _debug is None:
+                _debug = _bind(_build.build_debug())
+            _lib = _debug
+        else:
+            if _release is None:
+                _release = _bind(_build.build())
+            _lib = _release
 
 
 def check(status: int, what: str):

@@ -38,6 +38,7 @@ __global__ void pack_bits_kernel(const uint8_t *__restrict__ codes, long long n,
                 const long long s = byte * 8 + t;
                 const long long ci = s / b;
                 if (ci < row_len) {
+                    QCNN_CHECK((unsigned)c[ci] <= (unsigned)kmax, QCNN_CHECK_CODE);
                     const unsigned code = min((unsigned)c[ci], (unsigned)kmax);
                     v |= ((code >> (s - ci * b)) & 1u) << t;
                 }

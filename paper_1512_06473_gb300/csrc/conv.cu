@@ -51,6 +51,7 @@ size_t packed_codes_bytes(int Ct, int kk, int M) {
 // packed[m][pk][ct] = min(codes[ct][pk][m], K - 1); zero for ct >= Ct.
 __global__ void pack_codes_kernel(const uint8_t *__restrict__ codes, int Ct, int kk,
                                   int M, int K, int CtP, uint8_t *__restrict__ packed) {
+    grid_dep_sync();
     const size_t total = (size_t)M * kk * CtP;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -61,6 +62,7 @@ __global__ void pack_codes_kernel(const uint8_t *__restrict__ codes, int Ct, int
         unsigned v = 0;
         if (ct < Ct) {
             v = codes[((size_t)ct * kk + pk) * M + m];
+            QCNN_CHECK(v < (unsigned)K, QCNN_CHECK_CODE);
             v = v < (unsigned)K ? v : (unsigned)(K - 1);
         }
         packed[i] = (uint8_t)v;
@@ -71,8 +73,8 @@ qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K
                               uint8_t *packed, cudaStream_t st) {
     const size_t total = packed_codes_bytes(Ct, kk, M);
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
-    pack_codes_kernel<<<blocks, 256, 0, st>>>(codes, Ct, kk, M, K, packed_ct(Ct), packed);
-    return after_launch();
+    return launch_pdl(pack_codes_kernel, dim3(blocks), dim3(256), 0, st, codes, Ct, kk, M, K,
+                      packed_ct(Ct), packed);
 }
 
 // ==================================================================== fused
@@ -163,6 +165,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
+    grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
@@ -342,13 +345,18 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 unsigned w[CTW / 4];
                 load_code_words<CTW>(cb + pk * CT_CTA, w);
 #pragma unroll
-                for (int i = 0; i < CTW / 4; ++i) w[i] = __vminu4(w[i], kmax4);
+                for (int i = 0; i < CTW / 4; ++i) {
+                    QCNN_CHECK(__vcmpgtu4(w[i], kmax4) == 0u, QCNN_CHECK_CODE);
+                    w[i] = __vminu4(w[i], kmax4);
+                }
                 const int off = ky * pitch + kx;
                 const int base4 =
                     BF ? lane_off4 + (off >> 1) * 4 + (off & 1) * K * KS4 : lane_off4 + off * 4;
 #pragma unroll
                 for (int c = 0; c < CTW; ++c) {
                     const unsigned code = byte_of(w[c >> 2], c & 3);
+                    QCNN_CHECK((int)code * KS4 + base4 + (P - 1) * 128 + 4 <= K * KS * 4,
+                               QCNN_CHECK_TABLE);
                     const unsigned char *row = lutb + (int)code * KS4 + base4;
                     if constexpr (BF) {
 #pragma unroll
@@ -380,6 +388,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 const int g = cl0 + l, oy = g / pitch, col = g - oy * pitch;
                 if (col < a.Wo && oy < a.Ho) {
                     const size_t o = (((size_t)cn * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
+                    QCNN_CHECK(o < (size_t)a.N * a.Ct * a.Ho * a.Wo, QCNN_CHECK_GLOBAL);
                     if (mode == 1) {
                         a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
                     } else if (mode == 2) {
@@ -506,10 +515,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
 // entries (one channel, four positions) with 16-byte loads; boundaries that
 // fall between tiles have nothing to do.  Entries on discarded positions were
 // never written and are read but not stored.
-__global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, int extra, int M,
+__global__ void conv_sk_fixup_kernel(const float *part, int base, int extra, int M,
                                      int pos_tiles, int ct_tiles, int ST, int ct_cta, int Ct,
                                      int pitch, int Ho, int Wo, const float *__restrict__ bias,
                                      int relu, float *__restrict__ y) {
+    grid_dep_sync();
     const int b = blockIdx.x;
     const long long ub = (long long)(b + 1) * base + min(b + 1, extra);
     if (ub % M == 0) return;
@@ -539,10 +549,11 @@ __global__ void conv_sk_fixup_kernel(const float *__restrict__ part, int base, i
 }
 
 // y = bias + sum over splits of the partial sums, in split order; then ReLU.
-__global__ void conv_split_reduce_kernel(const float *__restrict__ partial, int splits,
+__global__ void conv_split_reduce_kernel(const float *partial, int splits,
                                          size_t total, int Ct, int HoWo,
                                          const float *__restrict__ bias, int relu,
                                          float *__restrict__ y) {
+    grid_dep_sync();
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
         float v = 0.f;
@@ -841,17 +852,15 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
     const dim3 grid = p.sk ? dim3(p.sk_ctas, 1, 1) : dim3(p.pos_tiles, p.ct_tiles, s.N * p.splits);
-    fv.fn<<<grid, fv.NW * 32, p.smem, st>>>(a);
-    qcnn_status rc = after_launch();
+    qcnn_status rc = launch_pdl(fv.fn, grid, dim3(fv.NW * 32), p.smem, st, a);
     if (rc != QCNN_OK) return rc;
     if (p.sk) {
         if (p.sk_ctas < 2) return QCNN_OK;
         const dim3 fgrid(p.sk_ctas - 1, (unsigned)cdiv(p.ct_cta * p.ST / 4, 256));
-        conv_sk_fixup_kernel<<<fgrid, 256, 0, st>>>(partial_ws, p.sk_base, p.sk_extra, s.M,
-                                                           p.pos_tiles, p.ct_tiles, p.ST,
-                                                           p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
-                                                           bias, relu, y);
-        return after_launch();
+        return launch_pdl(conv_sk_fixup_kernel, fgrid, dim3(256), 0, st,
+                          static_cast<const float *>(partial_ws), p.sk_base, p.sk_extra, s.M,
+                          p.pos_tiles, p.ct_tiles, p.ST, p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
+                          bias, relu, y);
     }
     if (p.splits == 1) return rc;
     return launch_split_reduce(partial_ws, p.splits, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
@@ -861,16 +870,15 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
 qcnn_status launch_split_reduce(const float *partial, int splits, size_t total, int Ct, int HoWo,
                                 const float *bias, int relu, float *y, cudaStream_t st) {
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
-    conv_split_reduce_kernel<<<blocks, 256, 0, st>>>(partial, splits, total, Ct, HoWo, bias, relu,
-                                                     y);
-    return after_launch();
+    return launch_pdl(conv_split_reduce_kernel, dim3(blocks), dim3(256), 0, st, partial, splits,
+                      total, Ct, HoWo, bias, relu, y);
 }
 
 // ================================================================== unfused
 // Tables of a chunk of NB images in the stride-phase-split layout
 //   lut[nb][m][k][ay][ax][py][px],  iy = py*s + ay,  ix = px*s + ax.
 struct UnfusedLutArgs {
-    const float *__restrict__ x;
+    const float *x;  // usually the output of the kernel before: coherent loads
     const float *__restrict__ D;
     float *__restrict__ lut;
     int n0, NB, Cs, H, W, s, Csp, K, M, HQ, WQ;
@@ -878,6 +886,7 @@ struct UnfusedLutArgs {
 
 __global__ void __launch_bounds__(256) conv_unfused_lut_kernel(const UnfusedLutArgs a) {
     extern __shared__ __align__(16) float dsm[];  // D[m] : [K][Csp]
+    grid_dep_sync();
     const int m = blockIdx.y, nb = blockIdx.z;
     const int n = a.n0 + nb;
     for (int e = threadIdx.x; e < a.K * a.Csp + kMaxCsp; e += blockDim.x)
@@ -899,7 +908,7 @@ __global__ void __launch_bounds__(256) conv_unfused_lut_kernel(const UnfusedLutA
 #pragma unroll
     for (int j = 0; j < kMaxCsp; ++j) {
         // the address stays inside x even for the lanes j >= Csp that are discarded
-        const float v = __ldg(xp + (size_t)min(j, a.Csp - 1) * a.H * a.W);
+        const float v = xp[(size_t)min(j, a.Csp - 1) * a.H * a.W];
         xv[j] = (in && j < a.Csp) ? v : 0.f;
     }
     float *out = a.lut + ((size_t)nb * a.M + m) * a.K * (size_t)PQ + q;
@@ -914,8 +923,8 @@ __global__ void __launch_bounds__(256) conv_unfused_lut_kernel(const UnfusedLutA
 }
 
 struct UnfusedGatherArgs {
-    const float *__restrict__ lut;
-    const uint8_t *__restrict__ codes;  // packed [M][kk][CtP]
+    const float *lut;                   // written by the kernel before
+    const uint8_t *codes;               // packed [M][kk][CtP] (maybe by the kernel before)
     const float *__restrict__ bias;
     float *__restrict__ y;
     int n0, Ct, CtP, H, W, kh, kw, s, pad, K, M, Ho, Wo, HQ, WQ, relu;
@@ -927,6 +936,7 @@ constexpr int kUnfSL = 2;    // 32-column slots per warp
 
 // grid: x = row tile (8 rows, one per warp) * col tile, y = channel tile, z = image in chunk
 __global__ void __launch_bounds__(256) conv_unfused_gather_kernel(const UnfusedGatherArgs a) {
+    grid_dep_sync();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int rt = blockIdx.x / a.col_tiles, ctile = blockIdx.x % a.col_tiles;
     const int oy = rt * 8 + warp;
@@ -962,8 +972,11 @@ __global__ void __launch_bounds__(256) conv_unfused_gather_kernel(const UnfusedG
                     off[sl] = ((ay * a.s + ax) * a.HQ + py) * a.WQ + ox[sl] + dx;
                 }
                 const uint8_t *cp = a.codes + ((size_t)m * kk + ky * a.kw + kx) * a.CtP + ct0;
-                const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(cp));
+                const uint4 cw = *reinterpret_cast<const uint4 *>(cp);
                 const unsigned kmax4 = (unsigned)(a.K - 1) * 0x01010101u;
+                QCNN_CHECK((__vcmpgtu4(cw.x, kmax4) | __vcmpgtu4(cw.y, kmax4) |
+                            __vcmpgtu4(cw.z, kmax4) | __vcmpgtu4(cw.w, kmax4)) == 0u,
+                           QCNN_CHECK_CODE);
                 const unsigned w[4] = {__vminu4(cw.x, kmax4), __vminu4(cw.y, kmax4),
                                        __vminu4(cw.z, kmax4), __vminu4(cw.w, kmax4)};
 #pragma unroll
@@ -971,8 +984,11 @@ __global__ void __launch_bounds__(256) conv_unfused_gather_kernel(const UnfusedG
                     const unsigned code = byte_of(w[c >> 2], c & 3);
                     const float *row = lm + (size_t)code * PQ;
 #pragma unroll
-                    for (int sl = 0; sl < kUnfSL; ++sl)
-                        if (ok[sl]) acc[c][sl] += __ldg(row + off[sl]);
+                    for (int sl = 0; sl < kUnfSL; ++sl) {
+                        QCNN_CHECK(!ok[sl] || (size_t)code * PQ + off[sl] < (size_t)a.K * PQ,
+                                   QCNN_CHECK_TABLE);
+                        if (ok[sl]) acc[c][sl] += row[off[sl]];
+                    }
                 }
             }
         }
@@ -1016,16 +1032,14 @@ qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p, co
         UnfusedLutArgs la{x, D, lut_ws, n0, nb, s.Cs, s.H, s.W, s.stride, s.Csp, s.K, s.M,
                           p.HQ, p.WQ};
         dim3 g1(cdiv(PQ, 256), s.M, nb);
-        conv_unfused_lut_kernel<<<g1, 256, ((size_t)s.K * s.Csp + kMaxCsp) * sizeof(float),
-                                  st>>>(la);
-        qcnn_status rc = after_launch();
+        qcnn_status rc = launch_pdl(conv_unfused_lut_kernel, g1, dim3(256),
+                                    ((size_t)s.K * s.Csp + kMaxCsp) * sizeof(float), st, la);
         if (rc != QCNN_OK) return rc;
         UnfusedGatherArgs ga{lut_ws, packed, bias, y, n0, s.Ct, packed_ct(s.Ct), s.H, s.W,
                              s.kh, s.kw, s.stride, s.pad, s.K, s.M, s.Ho, s.Wo, p.HQ, p.WQ,
                              relu, col_tiles};
         dim3 g2(cdiv(s.Ho, 8) * col_tiles, cdiv(s.Ct, kUnfCTW), nb);
-        conv_unfused_gather_kernel<<<g2, 256, 0, st>>>(ga);
-        rc = after_launch();
+        rc = launch_pdl(conv_unfused_gather_kernel, g2, dim3(256), 0, st, ga);
         if (rc != QCNN_OK) return rc;
     }
     return QCNN_OK;

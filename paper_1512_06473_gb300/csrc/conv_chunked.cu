@@ -70,6 +70,7 @@ __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed,
                                   int Ct, int kk, int M, int K, ChunkGeom g,
                                   uint32_t *__restrict__ entries, int *__restrict__ starts) {
     extern __shared__ int psh[];  // wcount[NW][NCH], bstart[NCH + 1]
+    grid_dep_sync();
     const int nw = blockDim.x / 32;
     int *wcount = psh, *bstart = psh + nw * g.NCH;
     const int i = blockIdx.x;
@@ -78,6 +79,7 @@ __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed,
     int code = 0, b = -1;
     if (pk < kk) {
         code = packed ? codes[((size_t)m * kk + pk) * CtP + ct] : codes[((size_t)ct * kk + pk) * M + m];
+        QCNN_CHECK(code < K, QCNN_CHECK_CODE);
         code = min(code, K - 1);
         b = code / g.KC;
     }
@@ -112,10 +114,10 @@ __global__ void chunk_prep_kernel(const uint8_t *__restrict__ codes, int packed,
 
 // ---------------------------------------------------------------- kernel --
 struct ChunkArgs {
-    const float *__restrict__ x;
+    const float *x;  // usually the output of the kernel before: coherent loads
     const float *__restrict__ D;
-    const uint32_t *__restrict__ entries;
-    const int *__restrict__ starts;
+    const uint32_t *entries;  // written by chunk_prep_kernel just before
+    const int *starts;
     const float *__restrict__ bias;
     float *__restrict__ y;
     int N, Cs, H, W, Ct, Csp, K, M, Ho, Wo, kk, ct_cta, relu;
@@ -129,6 +131,7 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
     const ChunkGeom &g = a.g;
     float *lut = csm;  // fp32 [KC][SK]; bf16 [2][KC][SKW] words
     float *ds = csm + (BF ? (size_t)2 * g.KC * g.SKW : (size_t)g.KC * g.SK);  // [K][CSPT]
+    grid_dep_sync();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int oy0 = blockIdx.x * g.TH;
     const int ct0 = blockIdx.y * a.ct_cta;
@@ -214,10 +217,13 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
             const int ct = ctw0 + c;
             if (ct < a.Ct) {
                 const size_t row = (size_t)m * a.Ct + ct;
-                const int e0 = __ldg(a.starts + row * (g.NCH + 1) + ch);
-                const int e1 = __ldg(a.starts + row * (g.NCH + 1) + ch + 1);
+                const int e0 = a.starts[row * (g.NCH + 1) + ch];
+                const int e1 = a.starts[row * (g.NCH + 1) + ch + 1];
                 const uint32_t *ep = a.entries + row * a.kk;
                 auto look = [&](const unsigned char *b) {
+                    QCNN_CHECK(b + (P - 1) * 128 + 4 <=
+                                   reinterpret_cast<const unsigned char *>(L) + 4 * g.KC * g.SK,
+                               QCNN_CHECK_TABLE);
                     if constexpr (BF) {
 #pragma unroll
                         for (int p = 0; p < P; ++p)
@@ -231,11 +237,11 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
                 };
                 int e = e0;
                 for (; e + 1 < e1; e += 2) {
-                    const unsigned o0 = __ldg(ep + e), o1 = __ldg(ep + e + 1);
+                    const unsigned o0 = ep[e], o1 = ep[e + 1];
                     look(lb + o0);
                     look(lb + o1);
                 }
-                if (e < e1) look(lb + __ldg(ep + e));
+                if (e < e1) look(lb + ep[e]);
             }
         }
     };
@@ -258,7 +264,7 @@ __global__ void __launch_bounds__(kChunkThreads, 1) conv_chunked_kernel(const Ch
                                      (ok ? iy : 0)) * a.W + (ok ? ix : 0);
 #pragma unroll
             for (int j = 0; j < CSPT; ++j) {
-                const float v = __ldg(xp + (size_t)min(j, a.Csp - 1) * a.H * a.W);
+                const float v = xp[(size_t)min(j, a.Csp - 1) * a.H * a.W];
                 xr[qi][j] = (ok && j < a.Csp) ? v : 0.f;
             }
         }
@@ -427,9 +433,9 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
     const int kk = s.kh * s.kw;
     const int pthreads = cdiv(kk, 32) * 32;
     const size_t psmem = ((size_t)(pthreads / 32) * g.NCH + g.NCH + 1) * sizeof(int);
-    chunk_prep_kernel<<<s.M * s.Ct, pthreads, psmem, st>>>(codes, codes_packed, packed_ct(s.Ct),
-                                                          s.Ct, kk, s.M, s.K, g, entries, starts);
-    qcnn_status rc = after_launch();
+    qcnn_status rc = launch_pdl(chunk_prep_kernel, dim3(s.M * s.Ct), dim3(pthreads), psmem, st,
+                                codes, codes_packed, packed_ct(s.Ct), s.Ct, kk, s.M, s.K, g,
+                                entries, starts);
     if (rc != QCNN_OK) return rc;
     ChunkArgs a;
     a.x = x;
@@ -456,8 +462,7 @@ qcnn_status launch_conv_chunked(const ConvShape &s, const ConvChunkPlan &p, cons
         cudaFuncSetAttribute(cv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
     dim3 grid(p.row_tiles, p.ct_tiles, s.N);
-    cv.fn<<<grid, kChunkThreads, p.smem, st>>>(a);
-    return after_launch();
+    return launch_pdl(cv.fn, grid, dim3(kChunkThreads), p.smem, st, a);
 }
 
 }  // namespace qcnn

@@ -74,6 +74,7 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
+    grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int l0 = blockIdx.x * ST, ct0 = blockIdx.y * CT_CTA;
@@ -197,10 +198,16 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
                         w[i] = (unsigned)h[2 * i] | (2 * i + 1 < CTW / 2 ? (unsigned)h[2 * i + 1] << 16 : 0u);
                 }
 #pragma unroll
-                for (int i = 0; i < (CTW + 3) / 4; ++i) w[i] = __vminu4(w[i], kmax4);
+                for (int i = 0; i < (CTW + 3) / 4; ++i) {
+                    QCNN_CHECK(__vcmpgtu4(w[i], kmax4) == 0u, QCNN_CHECK_CODE);
+                    w[i] = __vminu4(w[i], kmax4);
+                }
                 const int off4 = ((dy - a.dymin) * pitch + (dx - a.dxmin)) * 4;
 #pragma unroll
                 for (int c = 0; c < CTW; ++c) {
+                    QCNN_CHECK((int)byte_of(w[c >> 2], c & 3) * KS4 + off4 + lane * 4 +
+                                       (P - 1) * 128 + 4 <= K * KS4,
+                               QCNN_CHECK_TABLE);
                     const unsigned char *row = lutb + (int)byte_of(w[c >> 2], c & 3) * KS4 + off4;
                     accumulate<P>(acc[c], [&](int p) {
                         return *reinterpret_cast<const float *>(row + p * 128);
@@ -239,6 +246,7 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
             const int g = l0 + p * 32 + lane, oy = g / pitch, ox = g - oy * pitch;
             if (ox >= a.Wo || oy >= a.Ho) continue;
             const size_t o = (((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + ox;
+            QCNN_CHECK(o < (size_t)a.N * a.Ct * a.Ho * a.Wo, QCNN_CHECK_GLOBAL);
             if (a.splits > 1) {
                 a.partial[(size_t)split * a.N * a.Ct * a.Ho * a.Wo + o] = acc[c][p];
             } else {
@@ -394,8 +402,7 @@ qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const 
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
     const dim3 grid(p.pos_tiles, p.ct_tiles, s.N * p.splits);
-    pv.fn<<<grid, pv.NW * 32, p.smem, st>>>(a);
-    qcnn_status rc = after_launch();
+    qcnn_status rc = launch_pdl(pv.fn, grid, dim3(pv.NW * 32), p.smem, st, a);
     if (rc != QCNN_OK || p.splits == 1) return rc;
     return launch_split_reduce(partial_ws, p.splits, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
                                s.Ho * s.Wo, bias, relu, y, st);

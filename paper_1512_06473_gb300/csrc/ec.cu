@@ -374,7 +374,7 @@ qcnn_status qcnn_ec_quantize_fc(const float *S, const float *T, int N, int Cs, i
     if ((rc = cuda_status(cudaMemcpyAsync(&h_flag, flag, sizeof(int), cudaMemcpyDeviceToHost,
                                           st))) != QCNN_OK)
         return rc;
-    if ((rc = cuda_status(cudaStreamSynchronize(st))) != QCNN_OK) return rc;
+    if ((rc = sync_and_check(st)) != QCNN_OK) return rc;
     return h_flag ? QCNN_ERR_DATA : QCNN_OK;
 }
 

@@ -387,7 +387,10 @@ __global__ void ecc_bupdate_kernel(const float *__restrict__ S, EcConvGeo g, int
 __global__ void ecc_clamp_kernel(uint8_t *__restrict__ codes, long long n, int K) {
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (long long)gridDim.x * blockDim.x)
-        if (codes[i] >= K) codes[i] = (uint8_t)(K - 1);
+        if (codes[i] >= K) {
+            QCNN_CHECK(false, QCNN_CHECK_CODE);
+            codes[i] = (uint8_t)(K - 1);
+        }
 }
 
 __global__ void ecc_cast_kernel(const double *__restrict__ in, float *__restrict__ out,
@@ -560,7 +563,7 @@ qcnn_status qcnn_ec_quantize_conv(const float *S, const float *T, int N, int Cs,
     if ((rc = cuda_status(cudaMemcpyAsync(&h_flag, flag, sizeof(int), cudaMemcpyDeviceToHost, st))) !=
         QCNN_OK)
         return rc;
-    if ((rc = cuda_status(cudaStreamSynchronize(st))) != QCNN_OK) return rc;
+    if ((rc = sync_and_check(st)) != QCNN_OK) return rc;
     return h_flag ? QCNN_ERR_DATA : QCNN_OK;
 }
 

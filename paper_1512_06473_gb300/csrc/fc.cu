@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
+    grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wn = warp % WN, wc = warp / WN;
@@ -275,10 +276,13 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 } else {
                     w = *reinterpret_cast<const unsigned *>(cb + mm * a.crb + lane_ct);
                 }
+                QCNN_CHECK(__vcmpgtu4(w, kmax4) == 0u, QCNN_CHECK_CODE);
                 w = __vminu4(w, kmax4);
 #pragma unroll
                 for (int q = 0; q < kCPL; ++q) {
                     const int code = (int)byte_of(w, q);
+                    QCNN_CHECK((mm * a.K + code + 1) * a.NTP <= a.MCH * a.K * a.NTP,
+                               QCNN_CHECK_TABLE);
                     if constexpr (PAIRS) {
                         const unsigned *row = reinterpret_cast<const unsigned *>(lut) +
                                               (mm * a.K + code) * a.NTP + nbase / 2;
@@ -320,8 +324,9 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     }
 }
 
-__global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, int N, int Ct,
+__global__ void fc_reduce_kernel(const float *partial, int splits, int N, int Ct,
                                  const float *__restrict__ bias, int relu, float *__restrict__ y) {
+    grid_dep_sync();
     const size_t total = (size_t)N * Ct;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -335,9 +340,10 @@ __global__ void fc_reduce_kernel(const float *__restrict__ partial, int splits, 
 
 // Few outputs, many splits (batch 1): one warp per output; lane l adds the
 // splits l, l + 32, ... in order, then a fixed butterfly adds the lanes.
-__global__ void fc_reduce_warp_kernel(const float *__restrict__ partial, int splits, int N,
-                                      int Ct, const float *__restrict__ bias, int relu,
+__global__ void fc_reduce_warp_kernel(const float *partial, int splits, int N, int Ct,
+                                      const float *__restrict__ bias, int relu,
                                       float *__restrict__ y) {
+    grid_dep_sync();
     const size_t total = (size_t)N * Ct;
     const int lane = threadIdx.x & 31;
     for (size_t i = ((size_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < total;
@@ -487,19 +493,18 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
     dim3 grid(p.ct_tiles, p.n_tiles, p.splits);
-    fv.fn<<<grid, kFcThreads, p.smem, st>>>(a);
-    qcnn_status rc = after_launch();
+    qcnn_status rc = launch_pdl(fv.fn, grid, dim3(kFcThreads), p.smem, st, a);
     if (rc != QCNN_OK || p.splits == 1) return rc;
     const size_t total = (size_t)s.N * s.Ct;
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
     if (total < 65536 && p.splits >= 16) {
         const int wblocks = (int)std::min<size_t>((total * 32 + 255) / 256, (size_t)num_sms() * 16);
-        fc_reduce_warp_kernel<<<wblocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu,
-                                                       y);
-    } else {
-        fc_reduce_kernel<<<blocks, 256, 0, st>>>(partial_ws, p.splits, s.N, s.Ct, bias, relu, y);
+        return launch_pdl(fc_reduce_warp_kernel, dim3(wblocks), dim3(256), 0, st,
+                          static_cast<const float *>(partial_ws), p.splits, s.N, s.Ct, bias,
+                          relu, y);
     }
-    return after_launch();
+    return launch_pdl(fc_reduce_kernel, dim3(blocks), dim3(256), 0, st,
+                      static_cast<const float *>(partial_ws), p.splits, s.N, s.Ct, bias, relu, y);
 }
 
 }  // namespace qcnn

@@ -14,6 +14,8 @@
 // overlap on the GPU (other streams, other host threads) race on it.
 #include "qcnn_internal.cuh"
 
+#include <cuda.h>
+
 #include <mutex>
 
 namespace {
@@ -28,23 +30,66 @@ static __device__ __align__(256) float g_fc_scratch[kScratchBytes / sizeof(float
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mutex;
-void *g_scratch_addr[kMaxDevices] = {};
+struct ScratchAddr {
+    void *addr = nullptr;
+    unsigned long long ctx_id = 0;  // context the address belongs to
+};
+ScratchAddr g_scratch[kMaxDevices];
 
-// Device address of the scratch array on the current device; looked up once
-// per device (the first call on each device does it).
+// Unique id of the calling thread's current CUDA context (cuCtxGetId), or 0
+// when there is none or it cannot be had.  The driver functions are reached
+// through the runtime's entry-point query, so the library needs no link to
+// the driver library.  A device's primary context that is destroyed
+// (cudaDeviceReset) and created again gets a new id, and with it the module
+// holding the scratch array is loaded again at another address.
+unsigned long long current_context_id() {
+    using GetCurrent = CUresult (*)(CUcontext *);
+    using GetId = CUresult (*)(CUcontext, unsigned long long *);
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(f);
+        f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(f);
+        cudaGetLastError();
+    });
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx ||
+        get_id(ctx, &id) != CUDA_SUCCESS)
+        return 0;
+    return id;
+}
+
+// Device address of the scratch array in the current context.  It is
+// looked up (cudaGetSymbolAddress) on the first call on each device and
+// again whenever that device's context has changed since (or its id is
+// unavailable); otherwise the cached address is used.
 qcnn_status scratch_address(void **out) {
     int dev = -1;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return qcnn::cuda_status(e);
     if (dev < 0 || dev >= kMaxDevices) return QCNN_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_mutex);
-    if (!g_scratch_addr[dev]) {
+    ScratchAddr &c = g_scratch[dev];
+    const unsigned long long id = current_context_id();
+    if (!c.addr || id == 0 || id != c.ctx_id) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_fc_scratch);
         if (e != cudaSuccess || !p) return qcnn::cuda_status(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
-        g_scratch_addr[dev] = p;
+        c.addr = p;
+        c.ctx_id = current_context_id();  // the lookup may have created the context
     }
-    *out = g_scratch_addr[dev];
+    *out = c.addr;
     return QCNN_OK;
 }
 

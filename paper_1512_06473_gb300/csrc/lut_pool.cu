@@ -22,6 +22,7 @@ __global__ void __launch_bounds__(256) lut_build_kernel(const float *__restrict_
                                                         int Csp, int K, int M,
                                                         T *__restrict__ lut) {
     __shared__ float xs[kLutUnits][kMaxCsp];
+    grid_dep_sync();
     const int n = blockIdx.y;
     const long long units = (long long)M * P;
     const long long u0 = (long long)blockIdx.x * kLutUnits;
@@ -55,26 +56,28 @@ qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *
     const long long units = (long long)M * P;
     dim3 grid((unsigned)((units + kLutUnits - 1) / kLutUnits), N);
     if (bf16)
-        lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M,
-                                               static_cast<__nv_bfloat16 *>(lut));
-    else
-        lut_build_kernel<<<grid, 256, 0, st>>>(x, Cs, P, D, Csp, K, M, static_cast<float *>(lut));
-    return after_launch();
+        return launch_pdl(lut_build_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, x, Cs, P, D,
+                          Csp, K, M, static_cast<__nv_bfloat16 *>(lut));
+    return launch_pdl(lut_build_kernel<float>, grid, dim3(256), 0, st, x, Cs, P, D, Csp, K, M,
+                      static_cast<float *>(lut));
 }
 
 // k x k max-pool, stride s, no padding: one thread per output element.
 // One thread per output, 32-bit index arithmetic (every element count is
-// below 2^31); neighbouring windows share their overlap through L1.
-__global__ void maxpool_kernel(const float *__restrict__ x, int total, int H, int W, int k, int s,
-                               int Ho, int Wo, float *__restrict__ y) {
+// below 2^31); neighbouring windows share their overlap through L1.  x is
+// usually the output of the kernel just before, so it is read with plain
+// (coherent) loads.
+__global__ void maxpool_kernel(const float *x, int total, int H, int W, int k, int s, int Ho,
+                               int Wo, float *__restrict__ y) {
+    grid_dep_sync();
     const int HoWo = Ho * Wo;
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
         const int nc = i / HoWo, o = i - nc * HoWo;
         const int oy = o / Wo, ox = o - oy * Wo;
         const float *p = x + (size_t)nc * H * W + oy * s * W + ox * s;
-        float v = __ldg(p);
+        float v = p[0];
         for (int dy = 0; dy < k; ++dy)
-            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, __ldg(p + dy * W + dx));
+            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, p[dy * W + dx]);
         y[i] = v;
     }
 }
@@ -84,8 +87,8 @@ qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k, in
     const int Ho = (H - k) / s + 1, Wo = (W - k) / s + 1;
     const int total = N * C * Ho * Wo;
     const int blocks = std::max(1, std::min((total + 255) / 256, num_sms() * 8));
-    maxpool_kernel<<<blocks, 256, 0, st>>>(x, total, H, W, k, s, Ho, Wo, y);
-    return after_launch();
+    return launch_pdl(maxpool_kernel, dim3(blocks), dim3(256), 0, st, x, total, H, W, k, s, Ho, Wo,
+                      y);
 }
 
 }  // namespace qcnn

@@ -326,7 +326,7 @@ qcnn_status qcnn_model_upload(const void *blob, size_t bytes, void *device_buffe
     }
     // the staging areas are reused layer after layer and the blob is read by
     // the copies: finish before returning
-    return cuda_status(cudaStreamSynchronize(st));
+    return sync_and_check(st);
 }
 
 }  // extern "C"

@@ -27,6 +27,62 @@ qcnn_status after_launch() {
     return cuda_status(cudaGetLastError());
 }
 
+// State of programmatic launches on this host thread: 0 outside a call
+// scope (plain launches), 1 in a scope before its first launch (plain), 2 in
+// a scope after it (programmatic).
+thread_local int t_pdl = 0;
+
+PdlScope::PdlScope() : saved(t_pdl) { t_pdl = 1; }
+PdlScope::~PdlScope() { t_pdl = saved; }
+
+void pdl_break() {
+    if (t_pdl == 2) t_pdl = 1;
+}
+
+bool pdl_next_launch() {
+    if (t_pdl == 0) return false;
+    const bool programmatic = t_pdl == 2;
+    t_pdl = 2;
+    return programmatic;
+}
+
+// Readers of the translation units' device-check records (debug builds
+// register one per unit at load time; release builds none).
+std::mutex &check_mutex() {
+    static std::mutex m;
+    return m;
+}
+std::vector<CheckReader> &check_readers() {
+    static std::vector<CheckReader> v;
+    return v;
+}
+
+void register_check_reader(CheckReader r) {
+    std::lock_guard<std::mutex> g(check_mutex());
+    check_readers().push_back(r);
+}
+
+qcnn_status collect_device_checks(unsigned *flags) {
+    std::lock_guard<std::mutex> g(check_mutex());
+    qcnn_status rc = QCNN_OK;
+    for (CheckReader r : check_readers()) {
+        const qcnn_status s = r(flags);
+        if (rc == QCNN_OK) rc = s;
+    }
+    return rc;
+}
+
+qcnn_status sync_and_check(cudaStream_t st) {
+    qcnn_status rc = cuda_status(cudaStreamSynchronize(st));
+    if (rc != QCNN_OK) return rc;
+#ifdef QCNN_DEBUG_CHECKS
+    unsigned flags = 0;
+    if ((rc = collect_device_checks(&flags)) != QCNN_OK) return rc;
+    if (flags) return QCNN_ERR_DEVICE_CHECK;
+#endif
+    return QCNN_OK;
+}
+
 int num_sms() {
     static std::atomic<int> cached[64] = {};
     int dev = 0;
@@ -458,6 +514,7 @@ qcnn_status fc_forward_limited(const float *x, int N, int Cs, int Ct, const floa
         const qcnn_status rc = get_scratch(&scratch);
         if (rc != QCNN_OK) return rc;
     }
+    PdlScope pdl;
     return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(scratch), st);
 }
 
@@ -473,8 +530,28 @@ const char *qcnn_status_string(qcnn_status s) {
         case QCNN_ERR_WORKSPACE: return "workspace too small or misaligned";
         case QCNN_ERR_CUDA: return "CUDA error";
         case QCNN_ERR_DATA: return "input data unusable (rank-deficient calibration set)";
+        case QCNN_ERR_DEVICE_CHECK:
+            return "a kernel found a code >= K or an index outside its arrays (debug build)";
     }
     return "unknown status";
+}
+
+int qcnn_debug_checks(void) {
+#ifdef QCNN_DEBUG_CHECKS
+    return 1;
+#else
+    return 0;
+#endif
+}
+
+qcnn_status qcnn_device_check(void *stream, unsigned *flags) {
+    if (flags) *flags = 0;
+    qcnn_status rc = cuda_status(cudaStreamSynchronize(as_stream(stream)));
+    if (rc != QCNN_OK) return rc;
+    unsigned f = 0;
+    if ((rc = collect_device_checks(&f)) != QCNN_OK) return rc;
+    if (flags) *flags = f;
+    return f ? QCNN_ERR_DEVICE_CHECK : QCNN_OK;
 }
 
 int qcnn_last_cuda_error(void) { return g_last_cuda_error.load(); }
@@ -491,6 +568,7 @@ qcnn_status qcnn_lut_build(const float *x, int N, int Cs, int H, int W, const fl
     const long long P = (long long)H * W;
     if (!fits_int((long long)N * Cs * P) || !fits_int((long long)N * (Cs / Csp) * P * K))
         return QCNN_ERR_INVALID_ARG;
+    PdlScope pdl;
     return launch_lut_build(x, N, Cs, (int)P, D, Csp, K, lut, lut_type == QCNN_LUT_BF16,
                             as_stream(stream));
 }
@@ -513,6 +591,7 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct, const float *
     if (!f32_ok(x) || !f32_ok(D) || !f32_ok(y) || !f32_ok(bias)) return QCNN_ERR_INVALID_ARG;
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
+    PdlScope pdl;
     return launch_fc(s, p, x, D, codes, bias, y, relu, static_cast<float *>(workspace),
                      as_stream(stream));
 }
@@ -529,6 +608,7 @@ qcnn_status qcnn_fc_forward_packed(const float *x, int N, int Cs, int Ct, const 
     s.code_bits = code_bits(K);
     const FcPlan p = plan_fc(s);
     if (!ws_ok(workspace, workspace_bytes, p.partial_bytes)) return QCNN_ERR_WORKSPACE;
+    PdlScope pdl;
     return launch_fc(s, p, x, D, packed, bias, y, relu, static_cast<float *>(workspace),
                      as_stream(stream));
 }
@@ -634,6 +714,7 @@ qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int C
     qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
     if (!ws_ok(workspace, workspace_bytes, c.total)) return QCNN_ERR_WORKSPACE;
+    PdlScope pdl;
     return run_conv(c, x, D, codes, codes_layout, bias, y, relu, workspace, as_stream(stream));
 }
 
@@ -677,6 +758,7 @@ qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers, const float
     if (rc != QCNN_OK) return rc;
     if (!layer_pointers_ok(layers, n_layers)) return QCNN_ERR_INVALID_ARG;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
+    PdlScope pdl;
     return run_net(layers, np, x, y, workspace, as_stream(stream));
 }
 
@@ -690,6 +772,7 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
     if (!layer_pointers_ok(layers, n_layers)) return QCNN_ERR_INVALID_ARG;
     if (!ws_ok(workspace, workspace_bytes, np.total)) return QCNN_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
+    PdlScope pdl;
     uint8_t *base = static_cast<uint8_t *>(workspace);
     float *xd = reinterpret_cast<float *>(base + np.xin_off);
     float *yd = reinterpret_cast<float *>(base + np.yout_off);
@@ -726,6 +809,7 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
         }
         for (int c = 0; c < nc && rc == QCNN_OK; ++c) {
             rc = cuda_status(cudaStreamWaitEvent(st, hio->ready[c], 0));
+            pdl_break();  // the first kernel on slice c waits for its copy in full
             if (rc == QCNN_OK)
                 rc = run_step(layers[0], s0, xd + (size_t)c * (xs / sizeof(float)), y0 + c * ys,
                               base + np.scratch_off, st);
@@ -736,7 +820,7 @@ qcnn_status qcnn_net_forward_host(const qcnn_layer *layers, int n_layers, const 
         if (rc == QCNN_OK) rc = run_net(layers, np, xd, yd, workspace, st);
     }
     if (rc == QCNN_OK) rc = cuda_status(cudaMemcpyAsync(y_host, yd, yb, cudaMemcpyDeviceToHost, st));
-    const qcnn_status sync = cuda_status(cudaStreamSynchronize(st));
+    const qcnn_status sync = sync_and_check(st);
     return rc != QCNN_OK ? rc : sync;
 }
 

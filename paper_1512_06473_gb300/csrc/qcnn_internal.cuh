@@ -20,11 +20,80 @@ __host__ __device__ inline int cdiv(int a, int b) { return (a + b - 1) / b; }
 // Number of SMs of the current device (cached per device).
 int num_sms();
 
+// Device-check record of debug builds (QCNN_DEBUG_CHECKS): every translation
+// unit keeps its kernels' flags (QCNN_CHECK_* bits of include/qcnn.h) in a
+// device word of its own and registers a host function that reads and clears
+// it; collect_device_checks() ORs all of them into *flags.  Release builds
+// register nothing and collect nothing.
+using CheckReader = qcnn_status (*)(unsigned *flags);
+void register_check_reader(CheckReader r);
+qcnn_status collect_device_checks(unsigned *flags);
+// Synchronize `st`, then turn a non-empty device-check record into
+// QCNN_ERR_DEVICE_CHECK (debug builds); release builds only synchronize.
+qcnn_status sync_and_check(cudaStream_t st);
+
 // Book-keeping of launches and CUDA errors (qcnn_api.cu).
 void count_launch();
 qcnn_status cuda_status(cudaError_t e);
 // Check the launch that was just enqueued and count it.
 qcnn_status after_launch();
+
+// Programmatic dependent launch between the kernels of one library call.
+// An entry point that launches a chain of kernels opens a PdlScope; inside
+// it, the first launch is a plain one (it waits for everything queued before
+// it on the stream: the caller's kernels, copies, event waits) and the later
+// ones are programmatic: such a kernel may be scheduled while the kernel
+// before it is still running, and calls grid_dep_sync() before its first
+// access to global memory.  pdl_break() makes the next launch plain again
+// (after an event wait in the middle of a call).  Outside a scope every
+// launch is plain.
+struct PdlScope {
+    PdlScope();
+    ~PdlScope();
+    PdlScope(const PdlScope &) = delete;
+    PdlScope &operator=(const PdlScope &) = delete;
+    int saved;
+};
+void pdl_break();
+// true when the next launch may be programmatic; marks the launch as done
+bool pdl_next_launch();
+
+// Launch a kernel that calls grid_dep_sync() before touching global memory,
+// programmatically when the current PdlScope allows it.  Optional cluster
+// dimensions (cluster.x > 0).  Counts the launch and checks it.
+template <typename... P, typename... A>
+qcnn_status launch_k(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     dim3 cluster, A &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    unsigned n = 0;
+    if (pdl_next_launch()) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (cluster.x > 0) {
+        attr[n].id = cudaLaunchAttributeClusterDimension;
+        attr[n].val.clusterDim.x = cluster.x;
+        attr[n].val.clusterDim.y = cluster.y;
+        attr[n].val.clusterDim.z = cluster.z;
+        ++n;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = n;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<A &&>(args)...);
+    count_launch();
+    return cuda_status(e != cudaSuccess ? e : cudaGetLastError());
+}
+template <typename... P, typename... A>
+qcnn_status launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       A &&...args) {
+    return launch_k(kernel, grid, block, smem, st, dim3(0, 0, 0), static_cast<A &&>(args)...);
+}
 
 // ---------------------------------------------------------------- conv ----
 struct ConvShape {
@@ -174,6 +243,17 @@ namespace qcnn {
 // starts[k] = first slot of label k, starts[K] = P.
 __global__ void kmeans_order_kernel(const uint8_t *assign, int P, int K, int *order, int *starts);
 
+// Programmatic dependent launch.  A kernel started by launch_pdl may run
+// while the grid before it in the stream finishes; it calls grid_dep_sync()
+// before touching global memory.  That waits until every grid this one
+// depends on has completed and its writes are visible (a no-op for a kernel
+// launched without the attribute), then lets the next kernel of the stream
+// be scheduled; a kernel that has passed it has therefore all its inputs.
+__device__ __forceinline__ void grid_dep_sync() {
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
 __device__ __forceinline__ unsigned smem_addr(const void *p) {
     return static_cast<unsigned>(__cvta_generic_to_shared(p));
 }
@@ -241,4 +321,38 @@ __device__ __forceinline__ void accumulate(float (&acc)[P], F v) {
 }
 
 }  // namespace qcnn
+
+// ------------------------------------------------------- debug-build checks
+// QCNN_CHECK(cond, flag): in builds with QCNN_DEBUG_CHECKS, a kernel thread
+// that finds `cond` false ORs `flag` into its translation unit's record and
+// goes on (the kernels still clamp, so nothing is read out of bounds); the
+// host collects the records at the next synchronizing call.  Release builds
+// compile it to nothing.
+#ifdef QCNN_DEBUG_CHECKS
+namespace qcnn {
+namespace {
+__device__ unsigned g_check_flags;
+
+qcnn_status read_clear_check_flags(unsigned *flags) {
+    unsigned v = 0;
+    const unsigned zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_check_flags, sizeof v);
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_check_flags, &zero, sizeof zero);
+    *flags |= v;
+    return cuda_status(e);
+}
+struct CheckReaderRegistration {
+    CheckReaderRegistration() { register_check_reader(&read_clear_check_flags); }
+} g_check_reader_registration;
+}  // namespace
+}  // namespace qcnn
+#define QCNN_CHECK(cond, flag)                                             \
+    do {                                                                   \
+        if (!(cond)) atomicOr(&qcnn::g_check_flags, (unsigned)(flag));     \
+    } while (0)
+#else
+#define QCNN_CHECK(cond, flag) \
+    do {                       \
+    } while (0)
+#endif
 #endif

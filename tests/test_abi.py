@@ -21,9 +21,20 @@ def test_every_declared_symbol_is_exported():
 
 
 def test_status_strings():
-    for s in range(5):
-        assert lib.qcnn_status_string(s)
+    for s in range(7):
+        assert lib.qcnn_status_string(s) != b"unknown status"
     assert lib.qcnn_status_string(99) == b"unknown status"
+
+
+def test_debug_library_exports_every_symbol():
+    """libqcnn_debug.so (the device-checking build) has the same ABI; only
+    qcnn_debug_checks tells the two apart."""
+    from paper_1512_06473_gb300 import build as _build
+    dbg = _lib.load(_build.build_debug())
+    names = _lib.header_functions()
+    assert [n for n in names if not hasattr(dbg, n)] == []
+    assert dbg.qcnn_debug_checks() == 1
+    assert lib.qcnn_debug_checks() == 0
 
 
 N0 = None  # null device pointer

@@ -1,27 +1,30 @@
 """bfloat16 look-up tables (lut="bf16") through the C ABI against the oracle.
 
-Two references for every result:
-  * the oracle's bfloat16 table model (every entry rounded to the nearest
-    bfloat16, ties to even, sums exact).  The GPU rounds its fp32 entry and
-    the model the exact one, so an entry lying within an fp32 rounding of a
-    bfloat16 rounding boundary can round the other way (a few in 10^5): such
-    a "flip" moves the outputs that use the entry by one bfloat16 step of the
-    entry.  So every output must be within the fp32 bar (1e-5 of the output
-    range) plus two bfloat16 steps of the largest entry, and fewer than 1% of
-    the outputs may differ from the model by more than the fp32 bar.  A wrong
-    rounding direction, or a wrong copy of the pair tables, moves almost every
-    output.
-  * the exact oracle.  Rounding an entry v to bfloat16 moves it by at most
-    2^-8 |v| (half a step of 8 significant bits), so every output is within
-    2^-8 * (sum of |entries| it adds) of the exact one, plus fp32 slack; the
-    sums of |entries| come from a float64 conv2d of |LUT| with one-hot code
-    kernels.  On the benchmark's own layers the model is 1.2e-3 - 2.6e-3 of
-    the output range from exact (conv2 is the largest), and the GPU may add
-    at most a quarter of that on top (rounding flips).
-  * whole stacks: a rounding flip in one layer changes the next layer's
-    entries, so a GPU stack and the model stack drift apart to the size of
-    the bfloat16 error itself; a stack is held to twice the model's own
-    distance from the exact oracle.
+The stated bar for reduced-precision tables is max|err| / max|ref| <= 2e-3
+against the exact float64 oracle.  Rounding every table entry to bfloat16 (8
+significant bits) puts the exact rounding model itself 1.1e-3 - 2.6e-3 from
+exact on the benchmark's layers and 1.8e-3 - 5.3e-3 on its stacks, so the
+variant meets the bar on some layers and not on others.  The tests say which
+(test_benchmark_layers_bf16, test_net_bf16): in tolerance, the GPU result is
+held to 2e-3 of the exact oracle; out of tolerance, no claim is made and the
+GPU is only checked to implement the rounding model.
+
+Implementation checks on every case:
+  * against the oracle's bfloat16 table model (every entry rounded to the
+    nearest bfloat16, ties to even, sums exact).  The GPU rounds its fp32
+    entry and the model the exact one, so an entry lying within an fp32
+    rounding of a bfloat16 rounding boundary can round the other way (a few
+    in 10^5): such a "flip" moves the outputs that use the entry by one
+    bfloat16 step of the entry.  So every output must be within the fp32 bar
+    (1e-5 of the output range) plus two bfloat16 steps of the largest entry,
+    and fewer than 1% of the outputs may differ from the model by more than
+    the fp32 bar.  A wrong rounding direction, or a wrong copy of the pair
+    tables, moves almost every output.
+  * against the exact oracle, a bound that holds for any input: rounding an
+    entry v to bfloat16 moves it by at most 2^-8 |v| (half a step of 8
+    significant bits), so every output is within 2^-8 * (sum of |entries| it
+    adds) of the exact one, plus fp32 slack; the sums of |entries| come from a
+    float64 conv2d of |LUT| with one-hot code kernels.
 Integer data whose entries are exact in bfloat16 must match bit for bit,
 and a one-entry table (M = 1, K = 1, D = 1) must return bf16(x) exactly,
 ties included."""
@@ -262,37 +265,52 @@ def _bf16_net(w, params):
     return q.Net(net.layers, net.in_shape)
 
 
-@pytest.mark.parametrize("name,N,sample", [
-    ("alexnet_qcnn", 1, slice(None)),
-    ("alexnet_qcnn", 128, [0, 127]),
-    ("alexnet_fc678", 256, [0, 255]),
-    ("conv3x3_64x56x56_b1", 1, slice(None)),
-])
-def test_net_bf16(name, N, sample):
-    """Whole stacks against the exact oracle, held to twice the distance of
-    the model stack (the model is 5.3e-3 from exact after AlexNet's eight PQ
-    layers), and to 1e-2 at most."""
-    w = synth.WORKLOADS[name]
-    params = w.params()
-    x = w.input(N)
-    net = _bf16_net(w, params)
-    xin = x if x.ndim == 4 else x.reshape(N, -1, 1, 1)
-    got = host(net.forward(cuda(xin)))[sample]
-    ol = oracle_layers(w, params)
-    exact = oracle.net_forward(x[sample], ol)
-    model = oracle.net_forward(x[sample], [dict(d, lut_bf16=True) if d["kind"] != "maxpool" else d
-                                           for d in ol])
-    e_model = rel(model, exact)
-    e_got = rel(got.reshape(exact.shape), exact)
-    assert e_got <= 2 * e_model and e_got <= 1e-2, (e_got, e_model)
+# The stated bar for reduced-precision tables: max|err| / max|ref| <= 2e-3
+# against the exact (float64) oracle.
+BAR = 2e-3
+# A layer or stack is within the bar by construction only when the exact
+# bfloat16 table model itself -- every entry rounded exactly, sums exact,
+# the best any bfloat16 table can do -- stays clear of it: the GPU rounds its
+# fp32 entries, and a few entries within an fp32 rounding of a bfloat16
+# boundary round the other way ("flips"), so the model's distance gets a 5%
+# margin.  Where the model alone is beyond MODEL_MAX the variant is out of
+# tolerance for that layer, whatever the kernel does; there the GPU is only
+# checked to implement the rounding model, and no 2e-3 claim is made.
+MODEL_MAX = 0.95 * BAR
+# Which benchmark layers and stacks fall on which side (seeded inputs, see
+# the tests below).  Kept explicit so that the documentation of the variant
+# cannot drift from what is measured: (workload, layer index) -> in tolerance.
+IN_TOLERANCE_LAYERS = {
+    ("alexnet_qcnn", 0): True,    # conv1   model 1.73e-3
+    ("alexnet_qcnn", 2): False,   # conv2   model 2.08e-3
+    ("alexnet_qcnn", 4): False,   # conv3   model 2.15e-3
+    ("alexnet_qcnn", 5): False,   # conv4   model 1.91e-3 (within the margin)
+    ("alexnet_qcnn", 6): False,   # conv5   model 2.57e-3
+    ("alexnet_qcnn", 8): True,    # fc6     model 1.85e-3
+    ("alexnet_qcnn", 9): True,    # fc7     model 1.79e-3
+    ("alexnet_qcnn", 10): False,  # fc8     model 2.28e-3
+    ("conv3x3_64x56x56_b1", 0): True,   # model 1.83e-3
+    ("fc_512x256_b8", 0): True,         # model 1.55e-3
+    ("vgg16_conv_stack", 0): True,      # model 1.74e-3
+    ("vgg16_conv_stack", 1): True,      # model 1.72e-3
+    ("vgg16_conv_stack", 3): False,     # model 1.91e-3 (within the margin)
+    ("vgg16_conv_stack", 5): False,     # model 2.04e-3
+    ("vgg16_conv_stack", 6): True,      # model 1.87e-3
+    ("alexnet_fc678", 0): False,        # fc6 of the fc stack input: 2.00e-3
+    ("alexnet_fc678", 1): True,         # model 1.50e-3
+    ("alexnet_fc678", 2): True,         # model 1.15e-3
+}
 
 
 @pytest.mark.parametrize("name", ["alexnet_qcnn", "conv3x3_64x56x56_b1", "fc_512x256_b8",
-                                  "vgg16_conv_stack"])
+                                  "vgg16_conv_stack", "alexnet_fc678"])
 def test_benchmark_layers_bf16(name):
-    """Every PQ layer of the workloads, fed the exact activations of the
-    layer before it (two images): no further from the exact oracle than the
-    bfloat16 model is (times 1.25, plus 1e-4), and that within 3e-3."""
+    """Every PQ layer of the workloads with bfloat16 tables, fed the exact
+    activations of the layer before it (two images).  Where the rounding
+    model is within the margin, the GPU result must be within 2e-3 of the
+    exact oracle; elsewhere the variant is out of tolerance by construction
+    (the classification is asserted, so it stays true) and the GPU must
+    implement the rounding model."""
     w = synth.WORKLOADS[name]
     params = w.params()
     N = 2
@@ -314,12 +332,54 @@ def test_benchmark_layers_bf16(name):
         if isinstance(L, synth.Conv):
             model = oracle.conv_forward(h, d["D"], d["codes"], L.kh, L.kw, L.stride, L.pad,
                                         d["bias"], L.relu, lut_bf16=True)
+            emax = float(np.max(np.abs(oracle.conv_lut(h, d["D"]))))
         else:
             model = oracle.fc_forward(h.reshape(N, -1), d["D"], d["codes"], d["bias"], L.relu,
                                       lut_bf16=True)
+            emax = float(np.max(np.abs(oracle.fc_lut(h.reshape(N, -1), d["D"]))))
         e_model = rel(model.reshape(ref.shape), ref)
-        e_got = rel(host(got).reshape(ref.shape), ref)
-        assert e_model <= 3e-3 and e_got <= 1.25 * e_model + 1e-4, (name, i, e_got, e_model)
+        within = e_model <= MODEL_MAX
+        assert within == IN_TOLERANCE_LAYERS[(name, i)], (name, i, e_model)
+        got = host(got)
+        if within:
+            assert rel(got.reshape(ref.shape), ref) <= BAR, (name, i)
+        check_model(got.reshape(model.shape), model, emax)
+
+
+# whole stacks (batch as in the benchmark configs): in tolerance or not, by
+# the same rule as single layers
+IN_TOLERANCE_STACKS = {
+    "alexnet_qcnn": False,          # model 5.29e-3 after eight PQ layers
+    "vgg16_conv_stack": False,      # model 3.86e-3
+    "alexnet_fc678": False,         # model 2.25e-3
+    "conv3x3_64x56x56_b1": True,    # model 1.76e-3
+    "fc_512x256_b8": True,          # model 1.82e-3 at batch 8
+}
+
+
+@pytest.mark.parametrize("name,N", [("alexnet_qcnn", 2), ("vgg16_conv_stack", 1),
+                                    ("alexnet_fc678", 2), ("conv3x3_64x56x56_b1", 1),
+                                    ("fc_512x256_b8", 8)])
+def test_net_bf16(name, N):
+    """Whole stacks with bfloat16 tables against the exact oracle: within
+    2e-3 where the stack is in tolerance.  Through a stack, rounding flips in
+    one layer change the next layer's entries, so a GPU stack and the model
+    stack drift apart by about the size of the bfloat16 error itself: out of
+    tolerance, only the classification is asserted and no claim is made."""
+    w = synth.WORKLOADS[name]
+    params = w.params()
+    x = w.input(N)
+    net = _bf16_net(w, params)
+    xin = x if x.ndim == 4 else x.reshape(N, -1, 1, 1)
+    got = host(net.forward(cuda(xin)))
+    ol = oracle_layers(w, params)
+    exact = oracle.net_forward(x, ol)
+    model = oracle.net_forward(x, [dict(d, lut_bf16=True) if d["kind"] != "maxpool" else d
+                                   for d in ol])
+    within = rel(model, exact) <= MODEL_MAX
+    assert within == IN_TOLERANCE_STACKS[name], (name, rel(model, exact))
+    if within:
+        assert rel(got.reshape(exact.shape), exact) <= BAR
 
 
 @pytest.mark.parametrize("case", [(64, 64, 13, 13, 384, 3, 3, 1, 1, 4, 128),
