@@ -75,6 +75,45 @@ def _oracle_worker(args):
     return time.perf_counter() - t
 
 
+def _oracle_job(args):
+    """Time the float64 oracle on n seeded images of workload `name` (spawned
+    process; the images are drawn per job, so no batch is held)."""
+    name, salt, n = args
+    sys.path.insert(0, ROOT)
+    import oracle as orc
+    w = synth.WORKLOADS[name]
+    key = ("layers", name)
+    if key not in _CACHE:
+        _CACHE[key] = [synth.oracle_layer_dict(L, P) for L, P in zip(w.layers, w.params())]
+    x = w.input(n, 1000 + salt)
+    t = time.perf_counter()
+    orc.net_forward(x, _CACHE[key])
+    return time.perf_counter() - t
+
+
+def oracle_configs(pool, cores):
+    """The oracle beside every workload: one image (the smallest batch of the
+    workload when it is above 1) on one core, alone; and for workloads with
+    a large batch, images spread over all `cores` processes (images/s)."""
+    out = {}
+    for name in sorted(synth.WORKLOADS):
+        w = synth.WORKLOADS[name]
+        b0 = min(w.batches)
+        t1 = pool.apply(_oracle_job, ((name, 0, b0),))
+        r = {"single_thread": {"batch": b0, "s": round(t1, 4),
+                               "images_per_s": round(b0 / t1, 3)}}
+        big = max(w.batches)
+        if big > 8:
+            sample = cores * (4 if t1 < 0.5 else 1)
+            t = time.perf_counter()
+            pool.map(_oracle_job, [(name, i + 1, 1) for i in range(sample)], chunksize=1)
+            dt = time.perf_counter() - t
+            r["all_cores"] = {"batch": big, "images": sample, "cores": cores,
+                              "wall_s": round(dt, 3), "images_per_s": round(sample / dt, 3)}
+        out[name] = r
+    return out
+
+
 def _cpu_info():
     model = ""
     try:
@@ -385,34 +424,75 @@ def extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N, ba
         qres["oracle_ec_fc8_s"] = round(time.perf_counter() - t0, 3)
     res["quantizer"] = qres
 
-    # ---- the other workloads (parity cases of the tests), each net at its
-    # batches: forward time (L2 flushed), images/s, dense-equivalent GFLOP/s
-    # and the whole net's fraction of the shared-memory roofline
-    peak_smem = 152 * 128 * 2070e6
+    return res
+
+
+def build_layers(q, torch, w, params, dev, lut="fp32"):
+    """The workload's layers on the device, conv codes packed once (model load)."""
+    layers = []
+    for L, P in zip(w.layers, params):
+        if isinstance(L, synth.Conv):
+            codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
+            layers.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
+                                      torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
+                                      L.stride, L.pad, L.relu, packed=True, lut=lut))
+        elif isinstance(L, synth.FC):
+            layers.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
+                                    torch.from_numpy(P["codes"]).to(dev),
+                                    torch.from_numpy(P["bias"]).to(dev), L.relu, lut=lut))
+        else:
+            layers.append(q.PoolLayer(L.k, L.s))
+    return layers
+
+
+def layer_times(q, torch, qlayers, shapes, xin, ws, flush, stream, reps, lut="fp32"):
+    """Per-layer ms of a stack launched layer by layer through the C ABI, CUDA
+    events between the layers (L2 flushed before each pass; median of reps
+    after two untimed passes)."""
+    nb = xin.shape[0]
+    dev = xin.device
+    obufs = [torch.empty((nb, *sout), dtype=torch.float32, device=dev) for (_, sout) in shapes]
+    runs = []
+    for it in range(reps + 2):
+        flush.zero_()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(qlayers) + 1)]
+        ev[0].record(stream)
+        h = xin
+        for j, qL in enumerate(qlayers):
+            o = obufs[j]
+            if isinstance(qL, q.ConvLayer):
+                q.conv_forward(h, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias,
+                               qL.relu, packed=True, Ct=qL.Ct, out=o, workspace=ws, lut=lut)
+            elif isinstance(qL, q.FCLayer):
+                q.fc_forward(h.reshape(nb, -1), qL.D, qL.codes, qL.bias, qL.relu,
+                             out=o.reshape(nb, -1), workspace=ws, lut=lut)
+            else:
+                q.maxpool(h, qL.k, qL.s, out=o)
+            ev[j + 1].record(stream)
+            h = o
+        torch.cuda.synchronize(dev)
+        if it >= 2:
+            runs.append([ev[j].elapsed_time(ev[j + 1]) for j in range(len(qlayers))])
+    return [float(np.median([r[j] for r in runs])) for j in range(len(qlayers))]
+
+
+def measure_configs(q, torch, cm, dev, flush, stream, smem_gbs, hbm_gbs, reps):
+    """Every workload at each of its batches (the five configurations of the
+    target): the whole stack through qcnn_net_forward (device-resident input,
+    L2 flushed before each forward) -- ms, images/s, dense-equivalent GFLOP/s
+    and the stack's fraction of the shared-memory roofline -- and per layer
+    its ms and the fraction of its stage roofline (stage_rooflines)."""
     cfgs = {}
     for name in sorted(synth.WORKLOADS):
         wk = synth.WORKLOADS[name]
-        if name == w.name:
-            continue
         pk = wk.params()
-        lay = []
-        for L, P in zip(wk.layers, pk):
-            if isinstance(L, synth.Conv):
-                codes = q.conv_pack_codes(torch.from_numpy(P["codes"]).to(dev), L.K, L.kh, L.kw)
-                lay.append(q.ConvLayer(torch.from_numpy(P["D"]).to(dev), codes,
-                                       torch.from_numpy(P["bias"]).to(dev), L.Ct, L.kh, L.kw,
-                                       L.stride, L.pad, L.relu, packed=True))
-            elif isinstance(L, synth.FC):
-                lay.append(q.FCLayer(torch.from_numpy(P["D"]).to(dev),
-                                     torch.from_numpy(P["codes"]).to(dev),
-                                     torch.from_numpy(P["bias"]).to(dev), L.relu))
-            else:
-                lay.append(q.PoolLayer(L.k, L.s))
+        lay = build_layers(q, torch, wk, pk, dev)
         in_shape = tuple(wk.in_shape) if len(wk.in_shape) == 3 else (wk.in_shape[0], 1, 1)
         wnet = q.Net(lay, in_shape)
         costs = _layer_costs(wk, cm)
         dense = sum(c.dense_macs for c in costs)
         alg = 4.0 * sum(c.lookups + c.lut_entries for c in costs)
+        shapes = wk.shapes()
         per = []
         for B in wk.batches:
             xb = torch.from_numpy(wk.input(B, 3).reshape(B, *in_shape)).to(dev)
@@ -421,16 +501,30 @@ def extra_measurements(a, q, torch, w, params, x, out, flush, stream, dev, N, ba
             for _ in range(3):
                 wnet.forward(xb, out=wout, workspace=wws)
             torch.cuda.synchronize(dev)
-            ms_b = event_ms(lambda: wnet.forward(xb, out=wout, workspace=wws), 10)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ts = []
+            for _ in range(reps):
+                flush.zero_()
+                e0.record(stream)
+                wnet.forward(xb, out=wout, workspace=wws)
+                e1.record(stream)
+                torch.cuda.synchronize(dev)
+                ts.append(e0.elapsed_time(e1))
+            ms_b = float(np.median(ts))
+            xs = xb.reshape(B, *shapes[0][0]) if len(shapes[0][0]) == 3 else xb.reshape(B, -1)
+            lws = wnet.alloc_workspace(B, dev)
+            stage_ms = layer_times(q, torch, lay, shapes, xs, lws, flush, stream, reps)
             per.append({"batch": B, "ms": round(ms_b, 4), "images_per_s": round(B / (ms_b / 1e3), 1),
                         "dense_equiv_gflops": round(2 * dense * B / (ms_b / 1e3) / 1e9, 1),
-                        "frac_smem": round(alg * B / (ms_b / 1e3) / peak_smem, 4)})
+                        "frac_smem": round(alg * B / (ms_b / 1e3) / (smem_gbs * 1e9), 4),
+                        "stages": stage_rooflines(wk, cm, stage_ms, B, smem_gbs, hbm_gbs)})
         cfgs[name] = per
-    res["configs"] = {"note": "each workload's whole net, device-resident input, L2 flushed "
-                              "before every forward; frac_smem = 4 B x (look-ups + table "
-                              "entries) per second over 152 x 128 B x 2070 MHz",
-                      "workloads": cfgs}
-    return res
+    return {"note": "each workload's whole stack through qcnn_net_forward, device-resident "
+                    "input, L2 flushed before every forward; frac_smem = 4 B x (look-ups + "
+                    "table entries) per second over the measured shared-memory peak; stages: "
+                    "per layer, launched one by one, the fraction of the slower of its "
+                    "shared-memory roof and its HBM roof (stage_rooflines)",
+            "workloads": cfgs}
 
 
 def _layer_costs(w, cm):
@@ -602,7 +696,11 @@ def main():
     peaks = load_peaks()
     sm_max = float(peaks.get("sm_max_mhz") or 2070.0)
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
-    smem_peak_gbs = nsm * 128 * sm_max * 1e6 / 1e9
+    # shared-memory peak: 128 B per wavefront x the wavefronts per SM per cycle
+    # a conflict-free 16-byte-per-lane load stream sustains on this GPU,
+    # measured now (qcnn_smem_load_rate) x SMs x the maximum SM clock
+    smem_wpc = {"lds128": round(q.smem_load_rate(16), 4), "lds32": round(q.smem_load_rate(4), 4)}
+    smem_peak_gbs = nsm * 128 * smem_wpc["lds128"] * sm_max * 1e6 / 1e9
 
     def stage_report(stage_ms, entry_bytes):
         """Per-layer ms and shared-memory roofline fraction; algorithmic bytes =
@@ -637,7 +735,9 @@ def main():
         "traffic": recorded_traffic(WORKLOAD, N, dom["layer"]),
         "traffic_note": "DRAM read+write bytes per launch (ncu, profiles/dram_traffic.txt); "
                         "the kernel's algorithmic traffic is shared-memory, not DRAM",
-        "peak_basis": f"{nsm} SMs x 128 B/clk shared-memory loads x {sm_max:.0f} MHz max SM clock",
+        "peak_basis": (f"{nsm} SMs x 128 B x {smem_wpc['lds128']} wavefronts/clk "
+                       f"(measured now: conflict-free 16-byte shared loads, qcnn_smem_load_rate; "
+                       f"4-byte loads: {smem_wpc['lds32']}) x {sm_max:.0f} MHz max SM clock"),
         "alg_bytes_per_launch": dom_alg,
     }
 
@@ -705,29 +805,9 @@ def main():
     b1["roofline_note"] = (f"per stage: the slower of shared-memory bytes at {smem_peak_gbs:.0f} "
                            f"GB/s and HBM bytes at {hbm_gbs:.0f} GB/s (measured copy)")
 
-    # ---- bfloat16 tables: the same workload and timing, lut="bf16"
-    bf_layers = make_layers("bf16")
-    bf_net = q.Net(bf_layers, tuple(w.in_shape))
-    bf_ws = bf_net.alloc_workspace(N, dev)
-    for _ in range(max(a.warmup, 3)):
-        bf_net.forward(x, out=out, workspace=bf_ws)
-    torch.cuda.synchronize(dev)
-    bf_ms = 0.0
-    for i in range(a.steps):
-        flush.zero_()
-        starts[i].record(stream)
-        bf_net.forward(x, out=out, workspace=bf_ws)
-        ends[i].record(stream)
-    torch.cuda.synchronize(dev)
-    bf_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
-    if world > 1:
-        bf_ms = max_over_ranks(bf_ms, dev)
-    bf_stages, _ = stage_report(stage_times(bf_layers, "bf16"), 2.0)
-    bf16 = {"value": round(job_throughput(N, world, a.steps, bf_ms / 1e3), 1),
-            "unit": "images/s", "ms_per_step": round(bf_ms / a.steps, 4),
-            "note": "table entries rounded to bfloat16, sums in fp32; smem roofline at 2 B "
-                    "per look-up and per table entry; not the headline (fp32) number",
-            "batch1": batch1(bf_net), "stages": bf_stages}
+    # ---- every workload of the target at its batches, per layer (GPU)
+    configs = measure_configs(q, torch, cm, dev, flush, stream, smem_peak_gbs, hbm_gbs,
+                              max(5, a.steps // 3))
 
     extras = {}
     if not a.no_extras:
@@ -738,10 +818,15 @@ def main():
     if pool is not None:
         sample = a.cpu_sample or cores
         dt = time_oracle(pool, cores, sample, N)
+        cfg_oracle = oracle_configs(pool, cores)
         pool.close()
         cpu = {"value": sample / dt, "unit": "images/s", "cores": cores, "kind": "oracle",
                "sample": f"{sample} images of the batch-{N} workload, one per spawned process, "
-                         f"float64 C oracle, host {_cpu_info()}, {dt:.1f} s wall"}
+                         f"float64 C oracle, host {_cpu_info()}, {dt:.1f} s wall",
+               "configs": cfg_oracle,
+               "configs_note": "every workload: its smallest batch on one core alone "
+                               "(single_thread), and for workloads with a large batch, "
+                               "images on all cores (all_cores); same float64 C oracle"}
 
     if world > 1:
         dist.destroy_process_group()
@@ -758,7 +843,7 @@ def main():
                    "codes": "packed once at model load (outside the timed region)"},
         "dense_equiv_gflops": round(2 * dense_macs * value / 1e9, 1),
         "batch1": b1,
-        "roofline": roofline, "stages": stages, "bf16_lut": bf16, **extras,
+        "roofline": roofline, "stages": stages, "configs": configs, **extras,
         "cpu_baseline": cpu, "e2e": {k: (round(v, 1) if isinstance(v, float) else v)
                                      for k, v in e2e.items()},
         "gpu_launches": int(launches), "clocks": clk,

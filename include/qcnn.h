@@ -78,6 +78,11 @@ typedef enum {
     QCNN_ALGO_PHASE = 4,   /* full table rows of one stride phase of a tile
                               at a time in shared memory, any stride (fp32
                               tables)                                        */
+    QCNN_ALGO_NO_CLUSTER = 1 << 16, /* flag, OR-ed into any of the above:
+                              split sub-space ranges never form thread-block
+                              clusters (their partial sums all go through
+                              the workspace and a reduction kernel); for
+                              tests and tuning                              */
     QCNN_ALGO_FUSED_VARIANT = 256 /* + v: the fused kernel's tile variant v
                               (0 <= v < qcnn_conv_fused_variant_count()),
                               bypassing the planner's choice; for tests and
@@ -125,6 +130,20 @@ int qcnn_last_cuda_error(void);
 
 /* Number of kernels this library has launched in this process so far. */
 uint64_t qcnn_launch_count(void);
+
+/*
+ * qcnn_smem_load_rate -- the shared-memory load throughput of the current
+ * GPU, in 128-byte wavefronts per SM per clock cycle: the peak of the
+ * look-up stage's roofline (each look-up of Eq. 5 / Eq. 7 is one
+ * shared-memory load in the fused kernels; Table 1 counts them).  One CTA
+ * per SM streams conflict-free loads of vec_bytes (4 or 16) per lane from
+ * shared memory and times itself with the SM's cycle counter; the rate of
+ * the slowest CTA is returned, independent of the clock it ran at.
+ * Synchronizes `stream`.  Allocates nothing (its per-SM cycle counts live
+ * in a small array compiled into the library).  QCNN_ERR_INVALID_ARG for
+ * another vec_bytes or a NULL result pointer.
+ */
+qcnn_status qcnn_smem_load_rate(int vec_bytes, double *wavefronts_per_sm_clk, void *stream);
 
 /*
  * Device checks of the debug build.  The library can be built with
@@ -195,11 +214,14 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
  * would run, worked out on the host.  info receives: [0] images per CTA,
  * [1] outputs per CTA, [2] CTAs sharing the sub-spaces of one tile (1: no
  * partial sums), [3] sub-spaces per shared-memory chunk, [4] CTAs of the
- * main kernel.  QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for a
- * NULL info.
+ * main kernel, [5] CTAs per thread-block cluster: when it equals [2], the
+ * CTAs of a tile form one cluster and add their partial sums in
+ * distributed shared memory (small batches: no workspace, one kernel); 1
+ * for no cluster.  QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for
+ * a NULL info.
  */
 qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K,
-                              int lut_type, int info[5]);
+                              int lut_type, int info[6]);
 
 /*
  * Bit-packed codes: the storage model of Table 1 (Sec. 3.4), each code in
@@ -314,14 +336,18 @@ qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W,
  *   [3] output channels per CTA (0 for UNFUSED);
  *   [4] CTAs sharing the sub-spaces of one tile (1: no partial sums);
  *   [5] 1 when the FUSED kernel runs the stream-K schedule, else 0;
- *   [6] CTAs of the main kernel (0 for UNFUSED).
+ *   [6] CTAs of the main kernel (0 for UNFUSED);
+ *   [7] CTAs per thread-block cluster among those of [4]: they add their
+ *       partial sums in distributed shared memory, so only [4] / [7] partial
+ *       sums per output go through the workspace (none, and no second
+ *       kernel, when [7] == [4]); 1 for no cluster.
  * Errors are those of qcnn_conv_workspace_size, plus QCNN_ERR_INVALID_ARG
  * for a NULL info.
  */
 qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh,
                                 int kw, int stride, int pad, int Csp, int K,
                                 int codes_layout, int algo, int lut_type,
-                                int info[7]);
+                                int info[8]);
 
 /*
  * qcnn_maxpool -- k x k max-pool, stride s, no padding, floor output size

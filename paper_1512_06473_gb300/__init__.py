@@ -29,7 +29,7 @@ __all__ = ["lut_build", "fc_forward", "conv_forward", "conv_pack_codes", "maxpoo
            "code_bits", "pack_bits", "unpack_bits", "fc_pack_codes", "serialize_model",
            "model_info", "load_model",
            "ConvLayer", "FCLayer", "PoolLayer", "Net", "launch_count", "QcnnError", "load",
-           "set_debug", "debug_checks", "device_check"]
+           "set_debug", "debug_checks", "device_check", "smem_load_rate"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -77,6 +77,16 @@ def device_check(stream=None) -> int:
     if st not in (_lib.OK, _lib.ERR_DEVICE_CHECK):
         _lib.check(st, "qcnn_device_check")
     return int(flags.value)
+
+
+def smem_load_rate(vec_bytes: int = 16, stream=None) -> float:
+    """Shared-memory load wavefronts (128 B) per SM per cycle this GPU
+    sustains with conflict-free loads of vec_bytes (4 or 16) per lane
+    (qcnn_smem_load_rate): the peak of the look-up stage's roofline."""
+    r = ctypes.c_double(0.0)
+    _lib.check(load().qcnn_smem_load_rate(int(vec_bytes), ctypes.byref(r), _stream(stream)),
+               "qcnn_smem_load_rate")
+    return float(r.value)
 
 
 def launch_count() -> int:
@@ -213,16 +223,19 @@ _ALGO_NAMES = {v: k for k, v in _lib.ALGO.items()}
 
 
 def conv_plan(N, Cs, H, W, Ct, kh, kw, stride=1, pad=0, Csp=4, K=128, algo="auto",
-              packed=True, lut="fp32"):
+              packed=True, lut="fp32", cluster=True):
     """The plan conv_forward would run for these sizes (qcnn_conv_plan_info),
     worked out on the host: a dict with the algorithm's name, its kernel
-    variant, positions per tile, channels per CTA, splits, stream-K and CTAs."""
+    variant, positions per tile, channels per CTA, splits, stream-K, CTAs and
+    the CTAs per cluster among the splits (1: none)."""
     a = _lib.ALGO[algo] if isinstance(algo, str) else _lib.ALGO_FUSED_VARIANT + int(algo)
-    info = (ctypes.c_int * 7)()
+    if not cluster:
+        a |= _lib.ALGO_NO_CLUSTER
+    info = (ctypes.c_int * 8)()
     _lib.check(load().qcnn_conv_plan_info(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K,
                                           _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL,
                                           a, _lib.LUT[lut], info), "qcnn_conv_plan_info")
-    keys = ("algo", "variant", "positions", "channels", "splits", "stream_k", "ctas")
+    keys = ("algo", "variant", "positions", "channels", "splits", "stream_k", "ctas", "cluster")
     d = dict(zip(keys, list(info)))
     d["algo"] = _ALGO_NAMES[d["algo"]]
     return d
@@ -230,19 +243,21 @@ def conv_plan(N, Cs, H, W, Ct, kh, kw, stride=1, pad=0, Csp=4, K=128, algo="auto
 
 def fc_plan(N, Cs, Ct, Csp=4, K=32, lut="fp32"):
     """The plan fc_forward would run (qcnn_fc_plan_info): images and outputs
-    per CTA, splits, sub-spaces per chunk and CTAs."""
-    info = (ctypes.c_int * 5)()
+    per CTA, splits, sub-spaces per chunk, CTAs and CTAs per cluster (1: none)."""
+    info = (ctypes.c_int * 6)()
     _lib.check(load().qcnn_fc_plan_info(N, Cs, Ct, Csp, K, _lib.LUT[lut], info),
                "qcnn_fc_plan_info")
-    return dict(zip(("images", "outputs", "splits", "chunk", "ctas"), list(info)))
+    return dict(zip(("images", "outputs", "splits", "chunk", "ctas", "cluster"), list(info)))
 
 
 def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, algo="auto",
-                 packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32"):
+                 packed=False, Ct=None, out=None, workspace=None, stream=None, lut="fp32",
+                 cluster=True):
     """Eq. 7 conv response.  ``codes`` is [Ct, kh*kw, M] uint8, or (packed=True,
     then ``Ct`` is required) the output of conv_pack_codes.  ``algo`` is
     "auto", "fused", "unfused", "chunked", "phase", or an int v: fused tile variant v
-    of fused_variants()."""
+    of fused_variants().  cluster=False keeps split sub-space ranges out of
+    thread-block clusters (QCNN_ALGO_NO_CLUSTER)."""
     _need(x, "x", torch.float32, 4)
     _need(D, "D", torch.float32, 3)
     N, Cs, H, W = x.shape
@@ -258,6 +273,8 @@ def conv_forward(x, D, codes, kh, kw, stride=1, pad=0, bias=None, relu=False, al
         _need(bias, "bias", torch.float32, 1)
     layout = _lib.CODES_PACKED if packed else _lib.CODES_CANONICAL
     a = _lib.ALGO[algo] if isinstance(algo, str) else _lib.ALGO_FUSED_VARIANT + int(algo)
+    if not cluster:
+        a |= _lib.ALGO_NO_CLUSTER
     lt = _lib.LUT[lut]
     lib = load()
     nb = ctypes.c_size_t()

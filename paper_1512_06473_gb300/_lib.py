@@ -16,6 +16,7 @@ ERR_DEVICE_CHECK = 6
 CHECK_CODE, CHECK_TABLE, CHECK_GLOBAL = 1, 2, 4  # qcnn_device_check flag bits
 ALGO = {"auto": 0, "fused": 1, "unfused": 2, "chunked": 3, "phase": 4}
 ALGO_FUSED_VARIANT = 256  # + v: fused tile variant v
+ALGO_NO_CLUSTER = 1 << 16  # flag: no thread-block clusters for split sub-spaces
 CODES_CANONICAL, CODES_PACKED = 0, 1
 LUT = {"fp32": 0, "bf16": 1}
 LAYER_CONV, LAYER_FC, LAYER_MAXPOOL = 0, 1, 2
@@ -40,6 +41,7 @@ _SIGS = {
     "qcnn_last_cuda_error": (c_int, []),
     "qcnn_launch_count": (c_uint64, []),
     "qcnn_debug_checks": (c_int, []),
+    "qcnn_smem_load_rate": (c_int, [c_int, ctypes.POINTER(ctypes.c_double), c_void_p]),
     "qcnn_device_check": (c_int, [c_void_p, ctypes.POINTER(ctypes.c_uint)]),
     "qcnn_lut_build": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                                c_void_p, c_int, c_void_p]),

@@ -88,7 +88,8 @@ struct ConvFusedArgs {
     int pitch, ST, KS, HP, CtP, relu;  // ST: output positions per tile
     int xs_floats;  // floats of one x staging buffer (HP rounded up, times CSP4)
     int splits, m_per_split;    // sub-space ranges over several CTAs (small batches)
-    float *__restrict__ partial;  // [splits][N][Ct][Ho][Wo] when splits > 1
+    int cl;                     // the splits of a tile form clusters of cl CTAs (1: none)
+    float *__restrict__ partial;  // [splits / cl][N][Ct][Ho][Wo] when splits > cl
     // stream-K schedule (large batches): CTA c takes the (tile, sub-space)
     // units [u0, u1), u = tile * M + m, sk_base units each plus one for the
     // first sk_extra CTAs; tile = (n * ct_tiles + ct_tile) * pos_tiles + pos.
@@ -506,7 +507,42 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     }
 
-    if constexpr (!SK) store(a.splits > 1 ? 1 : 0, 0, 0);
+    if constexpr (!SK) {
+        if (a.cl > 1) {
+            // the cluster's CTAs (the splits of this tile) add their partial
+            // tiles in distributed shared memory; with more splits than one
+            // cluster, each cluster's sum is a partial for the split reduction
+            __syncthreads();  // every warp is done with the table
+            float *red = reinterpret_cast<float *>(smem);  // [CT_CTA][ST]
+#pragma unroll
+            for (int c = 0; c < CTW; ++c)
+#pragma unroll
+                for (int p = 0; p < P * E; ++p) {
+                    const int l = BF ? (wp * P + (p >> 1)) * 64 + 2 * lane + (p & 1)
+                                     : (wp * P + p) * 32 + lane;
+                    red[(wc * CTW + c) * ST + l] = acc[c][p];
+                }
+            const size_t plane = (size_t)a.N * a.Ct * a.Ho * a.Wo;
+            const int group = split / a.cl, groups = a.splits / a.cl;
+            cluster_tile_reduce(red, CT_CTA * ST, [&](int e, float v) {
+                const int ch = e / ST, l = e - ch * ST;
+                const int ct = cct0 + ch;
+                const int g = cl0 + l, oy = g / pitch, col = g - oy * pitch;
+                if (ct >= a.Ct || col >= a.Wo || oy >= a.Ho) return;
+                const size_t o = (((size_t)cn * a.Ct + ct) * a.Ho + oy) * a.Wo + col;
+                QCNN_CHECK(o < plane, QCNN_CHECK_GLOBAL);
+                if (groups > 1) {
+                    a.partial[(size_t)group * plane + o] = v;
+                } else {
+                    v += a.bias ? a.bias[ct] : 0.f;
+                    if (a.relu) v = fmaxf(v, 0.f);
+                    a.y[o] = v;
+                }
+            });
+        } else {
+            store(a.splits > 1 ? 1 : 0, 0, 0);
+        }
+    }
 }
 
 // Stream-K fix-up: the tile cut at the end of CTA b's range gets
@@ -650,7 +686,7 @@ void conv_fused_variant_info(int v, int info[9]) {
     for (int i = 0; i < 9; ++i) info[i] = vals[i];
 }
 
-ConvFusedPlan plan_conv_fused(const ConvShape &s, int force) {
+ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
     ConvFusedPlan best;
     if (s.stride != 1 || s.Csp > kMaxCsp) return best;
     const int csp4 = s.Csp <= 4 ? 4 : 8;
@@ -725,18 +761,41 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force) {
         // The 12-warp tiles lose to 16-warp ones when a CTA gets only a few
         // sub-spaces (measured: AlexNet conv3 at batch 1, 64 splits, 47 us
         // against 33 us), so they are split at most 8 ways.
+        // The splits of a tile can form a thread-block cluster (cl CTAs, a
+        // power of two dividing the split count, at most 16) whose partial
+        // tiles are added in distributed shared memory: then only
+        // splits / cl partial sums per output go through the workspace, and
+        // none (no reduction launch) when cl == splits.  The cluster's tile
+        // of sums reuses the table's shared memory.
         const int max_sp = fv.NW == 12 ? 8 : 64;
-        int splits = 1;
+        const bool red_fits = (size_t)ct_cta * ST * sizeof(float) <= smem;
+        int splits = 1, cl = 1;
         double score = 0;
         for (int sp = 1; sp <= std::min(s.M, max_sp); sp *= 2) {
             const int mps = cdiv(s.M, sp);
             const int sp_eff = cdiv(s.M, mps);
-            const double waves = std::ceil(ctas * sp_eff / (sms * cps));
-            const double part = sp_eff > 1 ? 2.0 * sp_eff * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
-            const double sc = waves * per_m * mps * cps + part / 3000.0 + (sp_eff > 1 ? 6000.0 : 0.0);
-            if (sp == 1 || sc < score) {
-                score = sc;
-                splits = sp_eff;
+            for (int c = 1; c <= std::min(sp_eff, 16); c *= 2) {
+                if (sp_eff % c != 0 || (c > 1 && (!red_fits || force_cl == 1))) continue;
+                if (force_cl > 1 && c != force_cl && sp_eff > 1) continue;
+                double slots = (double)sms * cps;
+                if (c > 1) {
+                    const int cap = cluster_capacity(reinterpret_cast<const void *>(fv.fn),
+                                                     fv.NW * 32, c, smem);
+                    if (cap < 1) continue;
+                    slots = std::min(slots, (double)cap * c);
+                }
+                const int groups = sp_eff / c;
+                const double waves = std::ceil(ctas * sp_eff / slots);
+                const double part =
+                    groups > 1 ? 2.0 * groups * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
+                const double red = c > 1 ? ((double)ct_cta * ST / 8.0 + 1500.0) * cps : 0.0;
+                const double sc = waves * per_m * mps * cps + part / 3000.0 +
+                                  (groups > 1 ? 6000.0 : 0.0) + red;
+                if ((sp == 1 && c == 1) || sc < score) {
+                    score = sc;
+                    splits = sp_eff;
+                    cl = c;
+                }
             }
             if (ctas * sp >= 2.0 * sms * cps) break;
         }
@@ -768,12 +827,15 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force) {
             score = sk_units * per_m * cps * 1.05 + part / 3000.0 + 6000.0;
             sk = 1;
             splits = 1;
+            cl = 1;
         }
         if (!best.ok || score < best.score) {
             best.splits = splits;
+            best.cl = cl;
             best.m_per_split = cdiv(s.M, splits);
-            best.partial_bytes =
-                splits > 1 ? (size_t)splits * s.N * s.Ct * s.Ho * s.Wo * sizeof(float) : 0;
+            best.partial_bytes = splits / cl > 1 ? (size_t)(splits / cl) * s.N * s.Ct * s.Ho *
+                                                       s.Wo * sizeof(float)
+                                                 : 0;
             best.sk = sk;
             if (sk) {
                 const long long units = (long long)s.N * pos_tiles * ct_tiles * s.M;
@@ -842,6 +904,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.xs_floats = cdiv(p.HP, 4) * 4 * fv.CSP4;
     a.splits = p.splits;
     a.m_per_split = p.m_per_split;
+    a.cl = p.cl;
     a.partial = partial_ws;
     a.sk = p.sk;
     a.sk_base = p.sk_base;
@@ -850,9 +913,12 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.ct_tiles = p.ct_tiles;
     cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
+    if (e == cudaSuccess && p.cl > 8)
+        e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return cuda_status(e);
     const dim3 grid = p.sk ? dim3(p.sk_ctas, 1, 1) : dim3(p.pos_tiles, p.ct_tiles, s.N * p.splits);
-    qcnn_status rc = launch_pdl(fv.fn, grid, dim3(fv.NW * 32), p.smem, st, a);
+    const dim3 cluster = p.cl > 1 ? dim3(1, 1, p.cl) : dim3(0, 0, 0);
+    qcnn_status rc = launch_k(fv.fn, grid, dim3(fv.NW * 32), p.smem, st, cluster, a);
     if (rc != QCNN_OK) return rc;
     if (p.sk) {
         if (p.sk_ctas < 2) return QCNN_OK;
@@ -862,9 +928,9 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
                           p.pos_tiles, p.ct_tiles, p.ST, p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
                           bias, relu, y);
     }
-    if (p.splits == 1) return rc;
-    return launch_split_reduce(partial_ws, p.splits, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
-                               s.Ho * s.Wo, bias, relu, y, st);
+    if (p.splits / p.cl == 1) return rc;
+    return launch_split_reduce(partial_ws, p.splits / p.cl, (size_t)s.N * s.Ct * s.Ho * s.Wo,
+                               s.Ct, s.Ho * s.Wo, bias, relu, y, st);
 }
 
 qcnn_status launch_split_reduce(const float *partial, int splits, size_t total, int Ct, int HoWo,

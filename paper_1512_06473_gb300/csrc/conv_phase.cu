@@ -33,10 +33,11 @@ struct PhaseArgs {
     const uint8_t *__restrict__ codes;  // packed [M][kk][CtP]
     const float *__restrict__ bias;
     float *__restrict__ y;
-    float *__restrict__ partial;  // [splits][N][Ct][Ho][Wo] when splits > 1
+    float *__restrict__ partial;  // [splits / cl][N][Ct][Ho][Wo] when splits > cl
     int N, Cs, H, W, Ct, kh, kw, s, pad, Csp, K, M, Ho, Wo;
     int pitch, dymin, dxmin, HP, KS, CtP, relu, xs_floats;
     int splits, units_per_split;
+    int cl;  // the splits of a tile form clusters of cl CTAs (1: none)
 };
 
 struct PhaseSmem {
@@ -235,6 +236,36 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
     }
     cp_async_wait<0>();
 
+    if (a.cl > 1) {
+        // the splits of this tile (one cluster) add their partial tiles in
+        // distributed shared memory; with more splits than one cluster, each
+        // cluster's sum is a partial for the split reduction
+        __syncthreads();  // every warp is done with the table
+        float *red = reinterpret_cast<float *>(smem);  // [CT_CTA][ST]
+#pragma unroll
+        for (int c = 0; c < CTW; ++c)
+#pragma unroll
+            for (int p = 0; p < P; ++p) red[(warp * CTW + c) * ST + p * 32 + lane] = acc[c][p];
+        const size_t plane = (size_t)a.N * a.Ct * a.Ho * a.Wo;
+        const int group = split / a.cl, groups = a.splits / a.cl;
+        cluster_tile_reduce(red, CT_CTA * ST, [&](int e, float v) {
+            const int ch = e / ST, l = e - ch * ST;
+            const int ct = ct0 + ch;
+            const int g = l0 + l, oy = g / pitch, ox = g - oy * pitch;
+            if (ct >= a.Ct || ox >= a.Wo || oy >= a.Ho) return;
+            const size_t o = (((size_t)n * a.Ct + ct) * a.Ho + oy) * a.Wo + ox;
+            QCNN_CHECK(o < plane, QCNN_CHECK_GLOBAL);
+            if (groups > 1) {
+                a.partial[(size_t)group * plane + o] = v;
+            } else {
+                v += a.bias ? a.bias[ct] : 0.f;
+                if (a.relu) v = fmaxf(v, 0.f);
+                a.y[o] = v;
+            }
+        });
+        return;
+    }
+
     // ---- epilogue: bias, ReLU, store; or raw partial sums -------------------
 #pragma unroll
     for (int c = 0; c < CTW; ++c) {
@@ -287,7 +318,7 @@ static int phase_ks(int need) {  // smallest KS >= need with KS % 32 == 1
 
 static int floor_div_i(int a, int b) { return a >= 0 ? a / b : -((-a + b - 1) / b); }
 
-ConvPhasePlan plan_conv_phase(const ConvShape &s) {
+ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl) {
     ConvPhasePlan best;
     if (s.Csp > kMaxCsp || s.bf16) return best;
     const int csp4 = s.Csp <= 4 ? 4 : 8;
@@ -325,16 +356,35 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s) {
         // not overlapped (about two wavefronts of time per 32 entries)
         const double per_u = (double)pv.P * ct_cta * kk / (s.stride * s.stride) +
                              (double)HP * s.K * 2.0 / 32.0;
-        int splits = 1;
+        // splits of a tile may form a cluster that adds its partial tiles in
+        // distributed shared memory (as in the fused planner)
+        const bool red_fits = (size_t)ct_cta * ST * sizeof(float) <= smem;
+        int splits = 1, cl = 1;
         double score = 0;
         for (int sp = 1; sp <= std::min(U, 64); sp *= 2) {
             const int ups = cdiv(U, sp), sp_eff = cdiv(U, ups);
-            const double waves = std::ceil(ctas * sp_eff / sms);
-            const double part = sp_eff > 1 ? 2.0 * sp_eff * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
-            const double sc = waves * per_u * ups + part / 3000.0 + (sp_eff > 1 ? 6000.0 : 0.0);
-            if (sp == 1 || sc < score) {
-                score = sc;
-                splits = sp_eff;
+            for (int c = 1; c <= std::min(sp_eff, 16); c *= 2) {
+                if (sp_eff % c != 0 || (c > 1 && (!red_fits || force_cl == 1))) continue;
+                if (force_cl > 1 && c != force_cl && sp_eff > 1) continue;
+                double slots = sms;
+                if (c > 1) {
+                    const int cap = cluster_capacity(reinterpret_cast<const void *>(pv.fn),
+                                                     pv.NW * 32, c, smem);
+                    if (cap < 1) continue;
+                    slots = std::min(slots, (double)cap * c);
+                }
+                const int groups = sp_eff / c;
+                const double waves = std::ceil(ctas * sp_eff / slots);
+                const double part =
+                    groups > 1 ? 2.0 * groups * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
+                const double red = c > 1 ? (double)ct_cta * ST / 8.0 + 1500.0 : 0.0;
+                const double sc = waves * per_u * ups + part / 3000.0 +
+                                  (groups > 1 ? 6000.0 : 0.0) + red;
+                if ((sp == 1 && c == 1) || sc < score) {
+                    score = sc;
+                    splits = sp_eff;
+                    cl = c;
+                }
             }
             if (ctas * sp >= 2.0 * sms) break;
         }
@@ -353,9 +403,11 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s) {
             best.pos_tiles = pos_tiles;
             best.ct_tiles = ct_tiles;
             best.splits = splits;
+            best.cl = cl;
             best.units_per_split = cdiv(U, splits);
-            best.partial_bytes =
-                splits > 1 ? (size_t)splits * s.N * s.Ct * s.Ho * s.Wo * sizeof(float) : 0;
+            best.partial_bytes = splits / cl > 1 ? (size_t)(splits / cl) * s.N * s.Ct * s.Ho *
+                                                       s.Wo * sizeof(float)
+                                                 : 0;
             best.smem = smem;
             best.score = score;
         }
@@ -398,13 +450,19 @@ qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const 
     a.xs_floats = cdiv(p.HP, 4) * 4 * pv.CSP4;
     a.splits = p.splits;
     a.units_per_split = p.units_per_split;
+    a.cl = p.cl;
     cudaError_t e = cudaFuncSetAttribute(pv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);
+    if (p.cl > 8) {
+        e = cudaFuncSetAttribute(pv.fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
     const dim3 grid(p.pos_tiles, p.ct_tiles, s.N * p.splits);
-    qcnn_status rc = launch_pdl(pv.fn, grid, dim3(pv.NW * 32), p.smem, st, a);
-    if (rc != QCNN_OK || p.splits == 1) return rc;
-    return launch_split_reduce(partial_ws, p.splits, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
+    const dim3 cluster = p.cl > 1 ? dim3(1, 1, p.cl) : dim3(0, 0, 0);
+    qcnn_status rc = launch_k(pv.fn, grid, dim3(pv.NW * 32), p.smem, st, cluster, a);
+    if (rc != QCNN_OK || p.splits / p.cl == 1) return rc;
+    return launch_split_reduce(partial_ws, p.splits / p.cl, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
                                s.Ho * s.Wo, bias, relu, y, st);
 }
 

@@ -83,6 +83,57 @@ qcnn_status sync_and_check(cudaStream_t st) {
     return QCNN_OK;
 }
 
+int cluster_capacity(const void *kernel, int threads, int C, size_t smem) {
+    struct Entry {
+        int dev;
+        const void *k;
+        int threads, C;
+        size_t smem;
+        int n;
+    };
+    static std::mutex mu;
+    static std::vector<Entry> cache;
+    int dev = 0, ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev < 1 || cudaGetDevice(&dev) != cudaSuccess) {
+        // No GPU (planning on a build host, e.g. for plan queries): the
+        // cluster occupancy measured on a GB300 (152 SMs) for 1..8 CTAs per
+        // SM; clusters do not span GPCs, so fewer SMs hold the large ones.
+        cudaGetLastError();
+        const int by_threads = std::max(1, 2048 / std::max(threads, 1));
+        const int per_sm = std::max(1, std::min(by_threads, (int)(228 * 1024 / (smem + 1024))));
+        const int sms_in_clusters = C <= 2 ? 152 : C == 4 ? 146 : C == 8 ? 128 : 112;
+        return per_sm * sms_in_clusters / C;
+    }
+    {
+        std::lock_guard<std::mutex> g(mu);
+        for (const Entry &e : cache)
+            if (e.dev == dev && e.k == kernel && e.threads == threads && e.C == C && e.smem == smem)
+                return e.n;
+    }
+    int n = 0;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+            cudaSuccess &&
+        cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+            cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(C, 1, 1);
+        cfg.blockDim = dim3(threads);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = C;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    std::lock_guard<std::mutex> g(mu);
+    cache.push_back({dev, kernel, threads, C, smem, n});
+    return n;
+}
+
 int num_sms() {
     static std::atomic<int> cached[64] = {};
     int dev = 0;
@@ -174,6 +225,8 @@ struct ConvCall {
 qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvCall *c) {
     if (codes_layout != QCNN_CODES_CANONICAL && codes_layout != QCNN_CODES_PACKED)
         return QCNN_ERR_INVALID_ARG;
+    const int force_cl = (algo & QCNN_ALGO_NO_CLUSTER) ? 1 : 0;
+    algo &= ~QCNN_ALGO_NO_CLUSTER;
     const bool forced = algo >= QCNN_ALGO_FUSED_VARIANT;
     if (forced) {
         if (algo - QCNN_ALGO_FUSED_VARIANT >= conv_fused_variant_count())
@@ -185,16 +238,16 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
     c->s = s;
     c->algo = QCNN_ALGO_UNFUSED;
     if (forced) {
-        c->fp = plan_conv_fused(s, algo - QCNN_ALGO_FUSED_VARIANT);
+        c->fp = plan_conv_fused(s, algo - QCNN_ALGO_FUSED_VARIANT, force_cl);
         if (!c->fp.ok) return QCNN_ERR_UNSUPPORTED;
         c->algo = QCNN_ALGO_FUSED;
     } else if (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_FUSED) {
-        c->fp = plan_conv_fused(s);
+        c->fp = plan_conv_fused(s, -1, force_cl);
         if (c->fp.ok) c->algo = QCNN_ALGO_FUSED;
         else if (algo == QCNN_ALGO_FUSED) return QCNN_ERR_UNSUPPORTED;
     }
     if (c->algo == QCNN_ALGO_UNFUSED && (algo == QCNN_ALGO_AUTO || algo == QCNN_ALGO_PHASE)) {
-        c->pp = plan_conv_phase(s);
+        c->pp = plan_conv_phase(s, force_cl);
         if (c->pp.ok) c->algo = QCNN_ALGO_PHASE;
         else if (algo == QCNN_ALGO_PHASE) return QCNN_ERR_UNSUPPORTED;
     }
@@ -649,15 +702,16 @@ qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh
 
 qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int kw, int stride,
                                 int pad, int Csp, int K, int codes_layout, int algo,
-                                int lut_type, int info[7]) {
+                                int lut_type, int info[8]) {
     ConvShape s;
     if (!info || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
     const qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
-    for (int i = 0; i < 7; ++i) info[i] = 0;
+    for (int i = 0; i < 8; ++i) info[i] = 0;
     info[0] = c.algo;
+    info[7] = 1;
     if (c.algo == QCNN_ALGO_FUSED) {
         const ConvFusedPlan &p = c.fp;
         info[1] = p.variant;
@@ -666,6 +720,7 @@ qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int
         info[4] = p.splits;
         info[5] = p.sk;
         info[6] = p.sk ? p.sk_ctas : p.pos_tiles * p.ct_tiles * s.N * p.splits;
+        info[7] = p.cl;
     } else if (c.algo == QCNN_ALGO_PHASE) {
         const ConvPhasePlan &p = c.pp;
         info[1] = p.variant;
@@ -673,6 +728,7 @@ qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int
         info[3] = p.ct_cta;
         info[4] = p.splits;
         info[6] = p.pos_tiles * p.ct_tiles * s.N * p.splits;
+        info[7] = p.cl;
     } else if (c.algo == QCNN_ALGO_CHUNKED) {
         const ConvChunkPlan &p = c.cp;
         info[1] = p.variant;
@@ -686,7 +742,7 @@ qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int
     return QCNN_OK;
 }
 
-qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_type, int info[5]) {
+qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_type, int info[6]) {
     FcShape s;
     if (!info || !fc_shape(N, Cs, Ct, Csp, K, lut_type, &s)) return QCNN_ERR_INVALID_ARG;
     const FcPlan p = plan_fc(s);
@@ -695,6 +751,7 @@ qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_typ
     info[2] = p.splits;
     info[3] = p.MCH;
     info[4] = p.ct_tiles * p.n_tiles * p.splits;
+    info[5] = p.small.ok ? p.small.C : 1;
     return QCNN_OK;
 }
 

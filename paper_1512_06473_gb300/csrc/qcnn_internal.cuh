@@ -116,6 +116,9 @@ struct ConvFusedPlan {
     int pos_tiles, ct_tiles;
     int splits = 1;     // CTAs sharing one tile's sub-spaces (small batches)
     int m_per_split;
+    int cl = 1;         // splits form clusters of cl CTAs that add their partial
+                        // sums in distributed shared memory; splits / cl
+                        // groups are left for the split reduction (1: none)
     int sk = 0;         // stream-K schedule (large batches): sk_ctas persistent
     int sk_ctas = 0;    // CTAs over the (tile, sub-space) units, sk_base each
     int sk_base = 0, sk_extra = 0;  // (+1 for the first sk_extra)
@@ -124,8 +127,16 @@ struct ConvFusedPlan {
     double score;       // estimated cost (lower is better)
 };
 
-// force >= 0: only that variant, without the planner's preference gates
-ConvFusedPlan plan_conv_fused(const ConvShape &s, int force = -1);
+// Clusters of C CTAs of `threads` threads and smem bytes of dynamic shared
+// memory that can be resident at once (cudaOccupancyMaxActiveClusters on the
+// current device, cached; with no device, the occupancy measured on a
+// GB300).  0 when such a cluster cannot be launched.
+int cluster_capacity(const void *kernel, int threads, int C, size_t smem);
+
+// force >= 0: only that variant, without the planner's preference gates;
+// force_cl: 0 = choose, 1 = no clusters, c > 1 = clusters of c CTAs wherever
+// the tile's sub-spaces are split
+ConvFusedPlan plan_conv_fused(const ConvShape &s, int force = -1, int force_cl = 0);
 int conv_fused_variant_count();
 void conv_fused_variant_info(int v, int info[9]);
 
@@ -158,11 +169,12 @@ struct ConvPhasePlan {
     int pitch, dymin, dxmin, HP, KS, ct_cta, pos_tiles, ct_tiles;
     int ST = 0;                           // output positions per tile
     int splits = 1, units_per_split = 0;  // (sub-space, phase) units per CTA
+    int cl = 1;                           // cluster of splits (as ConvFusedPlan)
     size_t partial_bytes = 0;             // workspace for split partial sums
     size_t smem;
     double score;
 };
-ConvPhasePlan plan_conv_phase(const ConvShape &s);
+ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl = 0);
 qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias, float *y,
                               int relu, float *partial_ws, cudaStream_t st);
@@ -200,7 +212,23 @@ qcnn_status launch_pack_bits(const uint8_t *codes, long long row_len, long long 
                              cudaStream_t st);
 qcnn_status launch_unpack_bits(const uint8_t *in, long long n, int b, uint8_t *codes,
                                cudaStream_t st);
+// Small batches (N <= 8, K <= 32; fc_small.cu): one thread-block cluster of C
+// CTAs per output tile, the sub-spaces split over its CTAs, tables in shared
+// memory read by warp shuffles, the partial sums added through distributed
+// shared memory -- one kernel, no workspace.
+struct FcSmallPlan {
+    bool ok = false;
+    int variant = -1;
+    int NB, OPL, ct_cta, tiles, C, m_per, MC, crow;
+    size_t smem;
+};
+FcSmallPlan plan_fc_small(const FcShape &s);
+qcnn_status launch_fc_small(const FcShape &s, const FcSmallPlan &p, const float *x,
+                            const float *D, const uint8_t *codes, const float *bias, float *y,
+                            int relu, cudaStream_t st);
+
 struct FcPlan {
+    FcSmallPlan small;  // used instead of the fields below when small.ok
     int variant;        // kernel table index
     int NT, CT_CTA;     // images and outputs per CTA
     int MCH;            // sub-spaces per shared-memory chunk
@@ -236,6 +264,7 @@ qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k,
 
 // ----------------------------------------------------------- device side ----
 #ifdef __CUDACC__
+#include <cooperative_groups.h>
 namespace qcnn {
 
 // quantize.cu: one CTA of kSortThreads (1024) threads per label array of P
@@ -279,6 +308,28 @@ __device__ __forceinline__ void cp_async_commit() {
 template <int N>
 __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// Sum of the partial tiles of the CTAs of a thread-block cluster.  Every CTA
+// has left its E partial sums in `red` (its own shared memory, same offset
+// in every CTA); after a cluster barrier, CTA r adds elements
+// [r*ceil(E/CL), ...) of all CL tiles in rank order -- a fixed order, so the
+// result does not depend on the schedule -- and hands each sum to emit(e, v).
+// A second barrier keeps every CTA's shared memory alive until all reads are
+// done.  Every thread of every CTA of the cluster must call it.
+template <typename F>
+__device__ __forceinline__ void cluster_tile_reduce(const float *red, int E, F &&emit) {
+    cooperative_groups::cluster_group cluster = cooperative_groups::this_cluster();
+    cluster.sync();
+    const int CL = (int)cluster.num_blocks(), r = (int)cluster.block_rank();
+    const int per = (E + CL - 1) / CL;
+    const int e1 = min(E, (r + 1) * per);
+    for (int e = r * per + (int)threadIdx.x; e < e1; e += (int)blockDim.x) {
+        float v = 0.f;
+        for (int q = 0; q < CL; ++q) v += cluster.map_shared_rank(red, q)[e];
+        emit(e, v);
+    }
+    cluster.sync();
 }
 
 // Byte b (0..3) of w, zero-extended.

@@ -358,13 +358,19 @@ def test_batch1_plans_split_the_subspaces():
         p = q.conv_plan(1, *shape, K=128)
         assert p["algo"] == ("phase" if name == "conv1" else "fused"), name
         assert p["splits"] > 1 and p["stream_k"] == 0 and p["ctas"] >= 64, (name, p)
+    # FC at batch 1: one cluster of CTAs per output tile shares the
+    # sub-spaces and adds its partial sums in distributed shared memory
+    # (no workspace, no second kernel)
+    nb = ctypes.c_size_t()
     for name, (Cs, Ct) in ALEX_FC.items():
         f = q.fc_plan(1, Cs, Ct)
-        assert f["images"] == 1 and f["splits"] >= 64, (name, f)
+        assert f["images"] == 1 and 8 <= f["splits"] <= 16 and f["ctas"] >= 64, (name, f)
+        assert lib.qcnn_fc_workspace_size(1, Cs, Ct, 4, 32, 0, ctypes.byref(nb)) == _lib.OK
+        assert nb.value == 0, name
 
 
 def test_plan_info_arguments():
-    info7, info5 = (ctypes.c_int * 7)(), (ctypes.c_int * 5)()
+    info7, info5 = (ctypes.c_int * 8)(), (ctypes.c_int * 6)()
     args = (2, 8, 9, 9, 4, 3, 3, 1, 1, 4, 16, 1)
     assert lib.qcnn_conv_plan_info(*args, 0, 0, None) == _lib.ERR_INVALID_ARG
     assert lib.qcnn_conv_plan_info(*args, 0, 0, info7) == _lib.OK

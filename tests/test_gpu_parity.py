@@ -183,6 +183,48 @@ def test_fc_sweep(case):
         assert rel(host(got), ref) <= TOL
 
 
+# Small batches (N <= 8, K <= 32) run one cluster kernel: (N, Cs, Ct, Csp, K)
+FC_SMALL = [
+    (1, 9216, 4096, 4, 32),    # fc6 at batch 1
+    (1, 4096, 1000, 4, 32),    # fc8 at batch 1: ragged last tile
+    (8, 512, 256, 4, 16),      # the single-layer FC workload
+    (3, 96, 70, 3, 5),         # odd batch, K not a power of two, tiny M
+    (5, 64, 1030, 8, 32),      # Ct % 4 == 2: codes copied byte by byte
+    (2, 40, 64, 1, 2),         # C's = 1, K = 2
+    (7, 2304, 513, 4, 32),     # many sub-spaces per CTA (several code chunks)
+    (1, 12, 3, 4, 32),         # M = 3 < cluster size: CTAs without sub-spaces
+]
+
+
+@pytest.mark.parametrize("case", FC_SMALL, ids=lambda c: "x".join(map(str, c)))
+def test_fc_small_batch(case):
+    N, Cs, Ct, Csp, K = case
+    M = Cs // Csp
+    plan = q.fc_plan(N, Cs, Ct, Csp, K)
+    assert plan["images"] <= 8 and plan["splits"] <= 16, plan  # the cluster kernel
+    x = synth.normal((N, Cs), 1.0, 24, *case)
+    D = synth.normal((M, K, Csp), 0.5, 25, *case)
+    codes = synth.uniform_codes((M, Ct), K, 26, *case)
+    b = synth.normal((Ct,), 0.1, 27, *case)
+    for relu in (False, True):
+        ref = oracle.fc_forward(x, D, codes, b, relu)
+        got = host(q.fc_forward(cuda(x), cuda(D), cuda(codes), cuda(b), relu=relu))
+        assert rel(got, ref) <= TOL
+    # bit-packed codes, same plan
+    rows = q.fc_pack_codes(cuda(codes), K)
+    got = host(q.fc_forward(cuda(x), cuda(D), rows, cuda(b), Ct=Ct))
+    assert rel(got, oracle.fc_forward(x, D, codes, b)) <= TOL
+    # integer data: exact in any summation order
+    xi = synth.small_integers((N, Cs), -8, 8, 28, *case)
+    Di = synth.small_integers((M, K, Csp), -8, 8, 29, *case)
+    bi = synth.small_integers((Ct,), -8, 8, 30, *case)
+    gi = host(q.fc_forward(cuda(xi), cuda(Di), cuda(codes), cuda(bi)))
+    assert np.array_equal(gi.astype(np.float64), oracle.fc_forward(xi, Di, codes, bi))
+    # deterministic
+    again = host(q.fc_forward(cuda(x), cuda(D), cuda(codes), cuda(b)))
+    assert np.array_equal(again, host(q.fc_forward(cuda(x), cuda(D), cuda(codes), cuda(b))))
+
+
 def test_fc_integer_bit_exact():
     N, Cs, Ct, Csp, K = 17, 256, 300, 4, 32
     M = Cs // Csp
@@ -374,6 +416,50 @@ def test_conv_stream_k(case):
     assert np.array_equal(goti.astype(np.float64), refi)
 
 
+# Small batches split a tile's sub-spaces over several CTAs; the CTAs of one
+# tile can form a thread-block cluster that adds their partial tiles in
+# distributed shared memory (all of them: no workspace partials and no
+# reduction kernel; or groups of them, whose sums the reduction kernel adds).
+CLUSTER = [
+    (1, 256, 13, 13, 384, 3, 3, 1, 1, 4, 128),    # AlexNet conv3 at batch 1
+    (1, 96, 27, 27, 256, 5, 5, 1, 2, 4, 128),     # conv2
+    (1, 3, 227, 227, 96, 11, 11, 4, 0, 3, 128),   # conv1 (stride-phase kernel)
+    (1, 64, 56, 56, 64, 3, 3, 1, 1, 4, 128),      # the single-layer conv workload
+    (1, 512, 14, 14, 512, 3, 3, 1, 1, 8, 128),    # VGG 14x14
+    (2, 128, 20, 17, 70, 3, 3, 1, 1, 8, 64),      # ragged tiles and channels
+    (1, 64, 9, 9, 40, 5, 5, 2, 2, 4, 32),         # strided, phase kernel
+]
+
+
+@pytest.mark.parametrize("case", CLUSTER, ids=lambda c: "x".join(map(str, c)))
+def test_conv_cluster_split_reduction(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    plan = q.conv_plan(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, packed=False)
+    flat = q.conv_plan(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, packed=False, cluster=False)
+    assert flat["cluster"] == 1
+    x, D, codes, b = conv_case(41, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), relu=True))
+    assert rel(got, ref) <= TOL, plan
+    nocl = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), relu=True,
+                               cluster=False))
+    assert rel(nocl, ref) <= TOL, flat
+    if plan["cluster"] == plan["splits"] and (plan["variant"], plan["splits"]) == \
+            (flat["variant"], flat["splits"]):
+        # the cluster adds the splits' tiles in the order the reduction kernel does
+        assert np.array_equal(got, nocl)
+    xi, Di, ci, bi = conv_case(42, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=True)
+    refi = oracle.conv_forward(xi, Di, ci, kh, kw, s, p, bi)
+    goti = host(q.conv_forward(cuda(xi), cuda(Di), cuda(ci), kh, kw, s, p, cuda(bi)))
+    assert np.array_equal(goti.astype(np.float64), refi), plan
+
+
+def test_some_small_batch_plans_use_clusters():
+    clustered = [q.conv_plan(*c[:9], Csp=c[9], K=c[10], packed=False)["cluster"] > 1
+                 for c in CLUSTER]
+    assert sum(clustered) >= 4, clustered
+
+
 # Every instantiated fused tile variant, forced through the C ABI (the
 # planner only ever picks some of them).  Integer inputs with |x|, |D| <= 4
 # keep every table entry within 256, so fp32 and bfloat16 tables alike give
@@ -406,3 +492,13 @@ def test_every_fused_variant_is_exact(case):
         assert np.array_equal(host(got).astype(np.float64), ref), (v, info)
         ran["sk" if info["SK"] else "bf" if info["BF"] else "pipe" if info["PIPE"] else "plain"] += 1
     assert ran["sk"] >= 2 and ran["bf"] >= 2 and ran["plain"] >= 4, ran
+
+
+def test_smem_load_rate():
+    """The roofline's shared-memory peak, measured: a conflict-free 16-byte
+    load stream reaches about one 128-byte wavefront per SM per cycle, a
+    4-byte one a little less; neither can exceed one."""
+    r16 = q.smem_load_rate(16)
+    r4 = q.smem_load_rate(4)
+    assert 0.8 <= r16 <= 1.01, r16
+    assert 0.5 <= r4 <= r16 + 0.01, (r4, r16)
