@@ -95,14 +95,16 @@ typedef enum {
 
 /*
  * The fused conv kernel's instantiated tile variants.  info receives
- * {P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK}: 32-position slots per warp,
+ * {P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK, TC}: 32-position slots per warp,
  * output channels per warp, warps along positions, C'_s register width (4
  * or 8), warps per CTA, CTAs per SM the registers are sized for, two table
- * buffers (1/0), bfloat16 tables (1/0), stream-K schedule (1/0).
+ * buffers (1/0), bfloat16 tables (1/0), stream-K schedule (1/0), table build
+ * on the tensor cores (1/0: tcgen05.mma kind::tf32 with the 3xTF32 split,
+ * for 4 < C'_s <= 8 and K a multiple of 32).
  * QCNN_ERR_INVALID_ARG for v out of range or a NULL info.
  */
 int qcnn_conv_fused_variant_count(void);
-qcnn_status qcnn_conv_fused_variant_info(int v, int info[9]);
+qcnn_status qcnn_conv_fused_variant_info(int v, int info[10]);
 
 /*
  * Precision of the look-up-table entries.  FP32: each entry is the fp32 dot
@@ -146,31 +148,35 @@ uint64_t qcnn_launch_count(void);
 qcnn_status qcnn_smem_load_rate(int vec_bytes, double *wavefronts_per_sm_clk, void *stream);
 
 /*
- * Device checks of the debug build.  The library can be built with
- * QCNN_DEBUG_CHECKS (libqcnn_debug.so); its kernels then test, as they run,
- * what the release kernels only clamp:
- *   QCNN_CHECK_CODE   a code >= K was read (the codes k_m(c_t) of Eq. 5 and
- *                     k_m(c_t, p_k) of Eq. 7 index K sub-codewords);
- *   QCNN_CHECK_TABLE  a look-up-table read in shared memory fell outside the
- *                     table the kernel built;
- *   QCNN_CHECK_GLOBAL a device-memory access fell outside its array.
+ * Device checks.  The library can be built with QCNN_DEBUG_CHECKS
+ * (libqcnn_debug.so); its kernels then test, as they run, what the release
+ * kernels only clamp:
+ *   QCNN_CHECK_CODE    a code >= K was read (the codes k_m(c_t) of Eq. 5 and
+ *                      k_m(c_t, p_k) of Eq. 7 index K sub-codewords);
+ *   QCNN_CHECK_TABLE   a look-up-table read in shared memory fell outside
+ *                      the table the kernel built;
+ *   QCNN_CHECK_GLOBAL  a device-memory access fell outside its array.
+ * In every build a kernel also records
+ *   QCNN_CHECK_TIMEOUT a bounded wait gave up (the tensor cores did not
+ *                      signal the completion of a table build in time); the
+ *                      kernel went on, so its outputs are unspecified.
  * A kernel that finds one ORs its bit into a device record and carries on
- * with the clamped value, so nothing faults.  The record is read, and
- * cleared, at the next synchronizing call: qcnn_device_check below, and the
- * calls that synchronize their stream anyway (qcnn_net_forward_host,
+ * (with the clamped value), so nothing faults or hangs.  The record is read,
+ * and cleared, at the next synchronizing call: qcnn_device_check below, and
+ * the calls that synchronize their stream anyway (qcnn_net_forward_host,
  * qcnn_ec_quantize_fc, qcnn_ec_quantize_conv, qcnn_model_upload), which then
  * return QCNN_ERR_DEVICE_CHECK instead of QCNN_OK.
  *
  * qcnn_debug_checks: 1 in a debug build, 0 in a release build.
  * qcnn_device_check: synchronizes `stream`; returns QCNN_ERR_DEVICE_CHECK
  *   when the record holds any bit (stored in *flags when flags is not NULL),
- *   and clears it.  In a release build it only synchronizes (*flags = 0).
- *   The record is per process and device-wide: work on other streams since
- *   the last check is included.
+ *   and clears it.  The record is per process and device-wide: work on
+ *   other streams since the last check is included.
  */
 #define QCNN_CHECK_CODE 1u
 #define QCNN_CHECK_TABLE 2u
 #define QCNN_CHECK_GLOBAL 4u
+#define QCNN_CHECK_TIMEOUT 8u
 int qcnn_debug_checks(void);
 qcnn_status qcnn_device_check(void *stream, unsigned *flags);
 
@@ -214,11 +220,9 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
  * would run, worked out on the host.  info receives: [0] images per CTA,
  * [1] outputs per CTA, [2] CTAs sharing the sub-spaces of one tile (1: no
  * partial sums), [3] sub-spaces per shared-memory chunk, [4] CTAs of the
- * main kernel, [5] CTAs per thread-block cluster: when it equals [2], the
- * CTAs of a tile form one cluster and add their partial sums in
- * distributed shared memory (small batches: no workspace, one kernel); 1
- * for no cluster.  QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for
- * a NULL info.
+ * main kernel, [5] CTAs per thread-block cluster among those of [2] (1:
+ * none; the FC kernel's partial sums always go through the workspace).
+ * QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for a NULL info.
  */
 qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K,
                               int lut_type, int info[6]);

@@ -210,10 +210,10 @@ def fused_variants():
     """The fused conv kernel's tile variants: a list of dicts (index = the
     variant number accepted by conv_forward's ``algo``)."""
     lib = load()
-    keys = ("P", "CTW", "WP", "CSP4", "NW", "MINB", "PIPE", "BF", "SK")
+    keys = ("P", "CTW", "WP", "CSP4", "NW", "MINB", "PIPE", "BF", "SK", "TC")
     out = []
     for v in range(lib.qcnn_conv_fused_variant_count()):
-        info = (ctypes.c_int * 9)()
+        info = (ctypes.c_int * 10)()
         _lib.check(lib.qcnn_conv_fused_variant_info(v, info), "qcnn_conv_fused_variant_info")
         out.append(dict(zip(keys, list(info))))
     return out

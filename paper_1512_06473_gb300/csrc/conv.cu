@@ -33,6 +33,8 @@
 //    read consecutive words for every kernel offset; a gather kernel then
 //    reads them through L1/L2.  Images are processed in chunks sized to
 //    stay L2 resident.
+// kernels of this unit record wait time-outs in every build
+#define QCNN_UNIT_RECORDS
 #include "qcnn_internal.cuh"
 
 #include <algorithm>
@@ -100,19 +102,35 @@ struct ConvFusedArgs {
 };
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
-// nlut = 2 table buffers when the sub-spaces are software pipelined.
+// nlut = 2 table buffers when the sub-spaces are software pipelined.  With
+// the tensor-core build (tc_rows > 0: halo positions rounded up to whole
+// 128-row MMA tiles), the staging buffers hold the operands in the tensor
+// core's K-major layout, plus the low halves of the 3xTF32 split (alo,
+// blo), the mbarrier of the MMAs and the tensor-memory address.
 struct FusedSmem {
-    size_t lut, xs, ds, cs, total;
+    size_t lut, xs, ds, cs, alo, blo, bar, total;
 };
 __host__ __device__ inline FusedSmem fused_smem_layout(int K, int KS, int xs_floats, int csp4,
-                                                       int kk, int ct_cta, int nlut) {
+                                                       int kk, int ct_cta, int nlut,
+                                                       int tc_rows = 0) {
     FusedSmem s;
     s.lut = 0;
     s.xs = ((size_t)nlut * K * KS * 4 + 15) / 16 * 16;
     s.ds = s.xs + (size_t)2 * xs_floats * 4;
     s.cs = s.ds + (size_t)2 * K * csp4 * 4;
-    s.total = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
+    s.alo = s.cs + ((size_t)2 * kk * ct_cta + 15) / 16 * 16;
+    s.blo = s.alo + (size_t)tc_rows * csp4 * 4;
+    s.bar = s.blo + (tc_rows ? (size_t)K * csp4 * 4 : 0);
+    s.total = s.bar + (tc_rows ? 16 : 0);
     return s;
+}
+
+// Offset (in floats) of element j of row r of a K-major tf32 operand with
+// 8 elements per row, in the tensor core's layout without swizzle: core
+// matrices of 8 rows x 4 elements (128 bytes), the two along K 128 bytes
+// apart, groups of 8 rows 256 bytes apart.
+__host__ __device__ inline int tc_off(int r, int j) {
+    return ((r >> 3) * 2 + (j >> 2)) * 32 + (r & 7) * 4 + (j & 3);
 }
 
 // Load CTW consecutive code bytes (16-byte aligned in shared memory).
@@ -147,9 +165,15 @@ __device__ __forceinline__ void load_code_words(const uint8_t *p, unsigned (&w)[
 //         gathered, with one barrier per sub-space instead of two
 // BF    : bfloat16 pair tables; a slot is then 64 positions (2 per lane)
 // SK    : stream-K schedule (a persistent grid over (tile, sub-space) units)
-template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF, bool SK>
+// TC    : table build on the tensor cores (tcgen05.mma kind::tf32, 3xTF32):
+//         positions x C'_s times C'_s x K per sub-space, accumulators in
+//         tensor memory, stored to the table by all warps
+template <int P, int CTW, int WP, int CSP4, int NW, int MINB, bool PIPE, bool BF, bool SK,
+          bool TC = false>
 __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFusedArgs a) {
     static_assert(!SK || !PIPE, "the stream-K schedule has one table buffer");
+    static_assert(!TC || (CSP4 == 8 && !PIPE && !BF && !SK),
+                  "tensor-core build: fp32 tables, C'_s width 8, one table buffer");
     constexpr int NT = NW * 32;
     constexpr int E = BF ? 2 : 1;  // positions per lane and slot
     constexpr int CT_CTA = (NW / WP) * CTW;
@@ -161,7 +185,9 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     extern __shared__ __align__(16) unsigned char smem[];
     const int kk = a.kh * a.kw;
     const int K = a.K, KS = a.KS, HP = a.HP, pitch = a.pitch;
-    const FusedSmem L = fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, PIPE ? 2 : 1);
+    const int tc_rows = TC ? a.xs_floats / CSP4 : 0;  // whole 128-row MMA tiles
+    const FusedSmem L =
+        fused_smem_layout(K, KS, a.xs_floats, CSP4, kk, CT_CTA, PIPE ? 2 : 1, tc_rows);
     float *lut0 = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
@@ -196,6 +222,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         for (int e = tid; e < 2 * a.xs_floats; e += NT) xs[e] = 0.f;
         for (int e = tid; e < 2 * K * CSP4; e += NT) ds[e] = 0.f;
     }
+    // tensor-core build: tensor memory for the accumulators of every
+    // 128-position tile (K columns each), one mbarrier for the MMAs
+    uint64_t *tc_bar = reinterpret_cast<uint64_t *>(smem + L.bar);
+    unsigned *tc_slot = reinterpret_cast<unsigned *>(smem + L.bar + 8);
+    if constexpr (TC) {
+        if (warp == 0) tmem_alloc(tc_slot, 512u);
+        if (tid == 0) {
+            mbar_init(tc_bar, 1);
+            asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+        }
+    }
     __syncthreads();
 
     // ---- asynchronous staging (callers commit) --------------------------
@@ -212,12 +249,14 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             const bool ok = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
             const float *src = ok ? xn + iy * a.W + ix : a.x;
             for (int j = 0; j < a.Csp; ++j)
-                cp_async4(xb + h * CSP4 + j, ok ? src + (size_t)j * HW : a.x, ok);
+                cp_async4(xb + (TC ? tc_off(h, j) : h * CSP4 + j),
+                          ok ? src + (size_t)j * HW : a.x, ok);
         }
         float *db = ds + b * K * CSP4;
         const float *dm = a.D + (size_t)m * K * a.Csp;
         for (int k = tid; k < K; k += NT)
-            for (int j = 0; j < a.Csp; ++j) cp_async4(db + k * CSP4 + j, dm + k * a.Csp + j, true);
+            for (int j = 0; j < a.Csp; ++j)
+                cp_async4(db + (TC ? tc_off(k, j) : k * CSP4 + j), dm + k * a.Csp + j, true);
     };
     // codes of sub-space m, channels ct0 ..; 16-byte pieces past the packed
     // row (CtP, a multiple of 256, may be short of the last tile) are zeros
@@ -325,6 +364,70 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 }
             }
         }
+    };
+
+    // ---- tensor-core build (TC): T[h][k] = sum_j x(h)[j] D[m][k][j] as the
+    // product of the positions x C'_s operand A and the C'_s x K operand B
+    // (3xTF32: A_hi B_hi + A_hi B_lo + A_lo B_hi, each tf32 product exact,
+    // accumulated in fp32 -- the fp32 accuracy of the FFMA build), one MMA of
+    // 128 positions x K codewords per tile and term; then every warp moves
+    // its tensor-memory lane quarter to the table, lut[k][h].
+    unsigned tc_phase = 0;
+    bool tc_failed = false;  // a wait gave up: no further MMAs or waits (bounded time)
+    auto build_tc = [&](int b, float *lut) {
+        float *ab = xs + b * a.xs_floats;  // raw fp32 A, split in place to A_hi
+        float *bb = ds + b * K * CSP4;     // raw fp32 B -> B_hi
+        float *al = reinterpret_cast<float *>(smem + L.alo);
+        float *bl = reinterpret_cast<float *>(smem + L.blo);
+        for (int e = tid; e < tc_rows * CSP4; e += NT) {
+            const float v = ab[e], hi = tf32_hi(v);
+            ab[e] = hi;
+            al[e] = v - hi;  // exact
+        }
+        for (int e = tid; e < K * CSP4; e += NT) {
+            const float v = bb[e], hi = tf32_hi(v);
+            bb[e] = hi;
+            bl[e] = v - hi;
+        }
+        fence_async_smem();
+        tc_fence_before_sync();
+        __syncthreads();
+        const unsigned tbase = *tc_slot;
+        const int n_mt = tc_rows / 128;
+        if (tid == 0 && !tc_failed) {
+            tc_fence_after_sync();
+            const uint32_t idesc = idesc_tf32(128, K);
+            const uint64_t bh = smem_desc_kmajor(bb, 128, 256), blw = smem_desc_kmajor(bl, 128, 256);
+            for (int t = 0; t < n_mt; ++t) {
+                const uint64_t ah = smem_desc_kmajor(ab + t * 128 * CSP4, 128, 256);
+                const uint64_t alw = smem_desc_kmajor(al + t * 128 * CSP4, 128, 256);
+                const unsigned d = tbase + (unsigned)(t * K);
+                mma_tf32(d, ah, bh, idesc, false);
+                mma_tf32(d, ah, blw, idesc, true);
+                mma_tf32(d, alw, bh, idesc, true);
+            }
+            mma_commit(tc_bar);
+        }
+        if (!tc_failed) {
+            const bool done = mbar_wait_bounded(tc_bar, tc_phase, 1u << 20);
+            tc_phase ^= 1u;
+            // the same decision in every thread of the CTA
+            tc_failed = __syncthreads_or(!done) != 0;
+            if (tid == 0) QCNN_RECORD_IF(tc_failed, QCNN_CHECK_TIMEOUT);
+        }
+        tc_fence_after_sync();
+        const int q = warp & 3, chunks = K / 32;
+        for (int u = warp >> 2; u < n_mt * chunks; u += NW / 4) {
+            const int t = u / chunks, c0 = (u - t * chunks) * 32;
+            const int h = t * 128 + q * 32 + lane;
+            float v[32];
+            tmem_ld32(tbase + ((unsigned)(q * 32) << 16) + (unsigned)(t * K + c0), v);
+            if (h < HP) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) lut[(c0 + j) * KS + h] = v[j];
+            }
+        }
+        tc_fence_before_sync();
     };
 
     // ---- gather: acc[c][p] += lut[code(c, pk)][pos(p) + ky*pitch + kx] -----
@@ -465,7 +568,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 stage_codes(m + 1, b ^ 1, sct0);
                 cp_async_commit();
             }
-            if constexpr (BF) build_bf16(b, lut0);
+            if constexpr (TC) build_tc(b, lut0);
+            else if constexpr (BF) build_bf16(b, lut0);
             else build(b, lut0);
             __syncthreads();
             gather(b, lut0);
@@ -542,6 +646,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         } else {
             store(a.splits > 1 ? 1 : 0, 0, 0);
         }
+        if constexpr (TC) {
+            __syncthreads();  // every warp's last tensor-memory load has completed
+            if (warp == 0) tmem_dealloc(*tc_slot, 512u);
+        }
     }
 }
 
@@ -608,6 +716,7 @@ struct FusedVariant {
     int P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK;
     double eff, build;
     void (*fn)(ConvFusedArgs);
+    int TC = 0;  // table build on the tensor cores
 };
 
 #define QCNN_FUSED(P, CTW, WP, C4, NW, MB, PIPE, EFF, BLD) \
@@ -622,6 +731,11 @@ struct FusedVariant {
 #define QCNN_FUSED_BF_SK(P, CTW, WP, C4, NW, MB, EFF, BLD) \
     {P, CTW, WP, C4, NW, MB, 0, 1, 1, EFF, BLD,            \
      conv_fused_kernel<P, CTW, WP, C4, NW, MB, false, true, true>}
+// tensor-core table build (C'_s 5..8): the build's FMAs leave the SM's FMA
+// pipe; its stores to the table remain
+#define QCNN_FUSED_TC(P, CTW, WP, NW, EFF, BLD)                                     \
+    {P, CTW, WP, 8, NW, 1, 0, 0, 0, EFF, BLD,                                       \
+     conv_fused_kernel<P, CTW, WP, 8, NW, 1, false, false, false, true>, 1}
 #define QCNN_FUSED_SET(C4)                                                                       \
     QCNN_FUSED(4, 8, 2, C4, 8, 2, false, 0.45, 1.0), /* small tiles for small batches */        \
     QCNN_FUSED(4, 16, 1, C4, 16, 1, false, 1.0, 1.0), /* 16 warps, 128 registers */             \
@@ -662,7 +776,13 @@ struct FusedVariant {
     QCNN_FUSED_BF_SK(4, 8, 1, C4, 16, 1, 1.0, 1.3)
 static const FusedVariant kFused[] = {QCNN_FUSED_SET(4),    QCNN_FUSED_SET(8),
                                       QCNN_FUSED_BF_SET(4), QCNN_FUSED_BF_SET(8),
-                                      QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8)};
+                                      QCNN_FUSED_SK_SET(4), QCNN_FUSED_SK_SET(8),
+                                      QCNN_FUSED_TC(6, 8, 1, 16, 1.0, 0.6),
+                                      QCNN_FUSED_TC(7, 8, 1, 16, 1.0, 0.6),
+                                      QCNN_FUSED_TC(4, 16, 1, 16, 1.0, 0.6),
+                                      QCNN_FUSED_TC(5, 16, 1, 16, 1.0, 0.6),
+                                      QCNN_FUSED_TC(4, 8, 1, 16, 1.0, 0.6)};
+#undef QCNN_FUSED_TC
 #undef QCNN_FUSED_SK_SET
 #undef QCNN_FUSED_BF_SK
 #undef QCNN_FUSED_SK
@@ -680,10 +800,10 @@ static int ks_for(int need) {  // smallest KS >= need with KS % 32 == 1
 
 int conv_fused_variant_count() { return kNumFused; }
 
-void conv_fused_variant_info(int v, int info[9]) {
+void conv_fused_variant_info(int v, int info[10]) {
     const FusedVariant &f = kFused[v];
-    const int vals[9] = {f.P, f.CTW, f.WP, f.CSP4, f.NW, f.MINB, f.PIPE, f.BF, f.SK};
-    for (int i = 0; i < 9; ++i) info[i] = vals[i];
+    const int vals[10] = {f.P, f.CTW, f.WP, f.CSP4, f.NW, f.MINB, f.PIPE, f.BF, f.SK, f.TC};
+    for (int i = 0; i < 10; ++i) info[i] = vals[i];
 }
 
 ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
@@ -741,11 +861,18 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
             KS = ks_for(ST + reach);
         }
         const int ct_cta = (fv.NW / fv.WP) * fv.CTW;
-        const int xs_floats = cdiv(HP, 4) * 4 * csp4;
-        const size_t smem =
-            fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta, fv.PIPE ? 2 : 1).total;
+        // tensor-core build: whole 128-row MMA tiles of halo positions, K
+        // (a multiple of 32, at most 256) accumulator columns per tile, all
+        // tiles within the 512 columns of tensor memory of the one CTA per SM
+        const int n_mt = cdiv(HP, 128);
+        if (fv.TC && (s.Csp <= 4 || s.K % 32 != 0 || s.K > 256 || n_mt * s.K > 512)) continue;
+        const int xs_floats = fv.TC ? n_mt * 128 * csp4 : cdiv(HP, 4) * 4 * csp4;
+        const size_t smem = fused_smem_layout(s.K, KS, xs_floats, csp4, kk, ct_cta,
+                                              fv.PIPE ? 2 : 1, fv.TC ? n_mt * 128 : 0)
+                                .total;
         if (smem > (size_t)smem_optin) continue;
         const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
+        if (fv.TC && cps != 1) continue;
         const int ct_tiles = cdiv(s.Ct, ct_cta);
         const double ctas = (double)s.N * pos_tiles * ct_tiles;
         // work per CTA and sub-space in shared-memory wavefronts (~cycles):
@@ -857,6 +984,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
             best.pos_tiles = pos_tiles;
             best.ct_tiles = ct_tiles;
             best.smem = smem;
+            best.xs_floats = xs_floats;
             best.score = score;
         }
     }
@@ -901,7 +1029,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.HP = p.HP;
     a.CtP = packed_ct(s.Ct);
     a.relu = relu;
-    a.xs_floats = cdiv(p.HP, 4) * 4 * fv.CSP4;
+    a.xs_floats = p.xs_floats;
     a.splits = p.splits;
     a.m_per_split = p.m_per_split;
     a.cl = p.cl;

@@ -385,22 +385,6 @@ static int fc_ntp(int NT, int bf16) { return (bf16 && NT % 2 == 0 ? NT / 2 : NT)
 
 FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
     FcPlan best{};
-    best.small = plan_fc_small(s);
-    if (best.small.ok) {  // one cluster kernel, no partial sums in a workspace
-        const FcSmallPlan &q = best.small;
-        best.variant = -1;
-        best.NT = q.NB;
-        best.CT_CTA = q.ct_cta;
-        best.MCH = q.MC;
-        best.n_chunks = cdiv(s.M, q.MC);
-        best.splits = q.C;
-        best.chunks_per_split = cdiv(q.m_per, q.MC);
-        best.n_tiles = cdiv(s.N, q.NB);
-        best.ct_tiles = q.tiles;
-        best.smem = q.smem;
-        best.partial_bytes = 0;
-        return best;
-    }
     double best_t = 1e300;
     const int sms = num_sms();
     const size_t sm_bytes = 228 * 1024;
@@ -471,7 +455,6 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const float *D,
                       const uint8_t *codes, const float *bias, float *y, int relu,
                       float *partial_ws, cudaStream_t st) {
-    if (p.small.ok) return launch_fc_small(s, p.small, x, D, codes, bias, y, relu, st);
     const FcVariant &fv = kFcVariants[p.variant];
     FcArgs a;
     a.x = x;

@@ -75,12 +75,9 @@ qcnn_status collect_device_checks(unsigned *flags) {
 qcnn_status sync_and_check(cudaStream_t st) {
     qcnn_status rc = cuda_status(cudaStreamSynchronize(st));
     if (rc != QCNN_OK) return rc;
-#ifdef QCNN_DEBUG_CHECKS
     unsigned flags = 0;
     if ((rc = collect_device_checks(&flags)) != QCNN_OK) return rc;
-    if (flags) return QCNN_ERR_DEVICE_CHECK;
-#endif
-    return QCNN_OK;
+    return flags ? QCNN_ERR_DEVICE_CHECK : QCNN_OK;
 }
 
 int cluster_capacity(const void *kernel, int threads, int C, size_t smem) {
@@ -681,7 +678,7 @@ qcnn_status qcnn_conv_pack_codes(const uint8_t *codes, int Ct, int kh, int kw, i
 
 int qcnn_conv_fused_variant_count(void) { return conv_fused_variant_count(); }
 
-qcnn_status qcnn_conv_fused_variant_info(int v, int info[9]) {
+qcnn_status qcnn_conv_fused_variant_info(int v, int info[10]) {
     if (!info || v < 0 || v >= conv_fused_variant_count()) return QCNN_ERR_INVALID_ARG;
     conv_fused_variant_info(v, info);
     return QCNN_OK;
@@ -751,7 +748,7 @@ qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_typ
     info[2] = p.splits;
     info[3] = p.MCH;
     info[4] = p.ct_tiles * p.n_tiles * p.splits;
-    info[5] = p.small.ok ? p.small.C : 1;
+    info[5] = 1;  // the FC kernel's splits never form clusters
     return QCNN_OK;
 }
 

@@ -124,6 +124,7 @@ struct ConvFusedPlan {
     int sk_base = 0, sk_extra = 0;  // (+1 for the first sk_extra)
     size_t partial_bytes = 0;  // workspace for split or stream-K partial sums
     size_t smem;        // dynamic shared memory bytes
+    int xs_floats;      // floats of one input staging buffer
     double score;       // estimated cost (lower is better)
 };
 
@@ -138,7 +139,7 @@ int cluster_capacity(const void *kernel, int threads, int C, size_t smem);
 // the tile's sub-spaces are split
 ConvFusedPlan plan_conv_fused(const ConvShape &s, int force = -1, int force_cl = 0);
 int conv_fused_variant_count();
-void conv_fused_variant_info(int v, int info[9]);
+void conv_fused_variant_info(int v, int info[10]);
 
 struct ConvUnfusedPlan {
     int NB;             // images per table chunk
@@ -212,23 +213,7 @@ qcnn_status launch_pack_bits(const uint8_t *codes, long long row_len, long long 
                              cudaStream_t st);
 qcnn_status launch_unpack_bits(const uint8_t *in, long long n, int b, uint8_t *codes,
                                cudaStream_t st);
-// Small batches (N <= 8, K <= 32; fc_small.cu): one thread-block cluster of C
-// CTAs per output tile, the sub-spaces split over its CTAs, tables in shared
-// memory read by warp shuffles, the partial sums added through distributed
-// shared memory -- one kernel, no workspace.
-struct FcSmallPlan {
-    bool ok = false;
-    int variant = -1;
-    int NB, OPL, ct_cta, tiles, C, m_per, MC, crow;
-    size_t smem;
-};
-FcSmallPlan plan_fc_small(const FcShape &s);
-qcnn_status launch_fc_small(const FcShape &s, const FcSmallPlan &p, const float *x,
-                            const float *D, const uint8_t *codes, const float *bias, float *y,
-                            int relu, cudaStream_t st);
-
 struct FcPlan {
-    FcSmallPlan small;  // used instead of the fields below when small.ok
     int variant;        // kernel table index
     int NT, CT_CTA;     // images and outputs per CTA
     int MCH;            // sub-spaces per shared-memory chunk
@@ -316,7 +301,8 @@ __device__ __forceinline__ void cp_async_wait() {
 // [r*ceil(E/CL), ...) of all CL tiles in rank order -- a fixed order, so the
 // result does not depend on the schedule -- and hands each sum to emit(e, v).
 // A second barrier keeps every CTA's shared memory alive until all reads are
-// done.  Every thread of every CTA of the cluster must call it.
+// done.  Every thread of every CTA of the cluster (at most 16 CTAs) must
+// call it.
 template <typename F>
 __device__ __forceinline__ void cluster_tile_reduce(const float *red, int E, F &&emit) {
     cooperative_groups::cluster_group cluster = cooperative_groups::this_cluster();
@@ -325,11 +311,137 @@ __device__ __forceinline__ void cluster_tile_reduce(const float *red, int E, F &
     const int per = (E + CL - 1) / CL;
     const int e1 = min(E, (r + 1) * per);
     for (int e = r * per + (int)threadIdx.x; e < e1; e += (int)blockDim.x) {
+        float part[16];  // every rank's partial in flight at once, then added in order
+#pragma unroll
+        for (int q = 0; q < 16; ++q) part[q] = q < CL ? cluster.map_shared_rank(red, q)[e] : 0.f;
         float v = 0.f;
-        for (int q = 0; q < CL; ++q) v += cluster.map_shared_rank(red, q)[e];
+#pragma unroll
+        for (int q = 0; q < 16; ++q)
+            if (q < CL) v += part[q];
         emit(e, v);
     }
     cluster.sync();
+}
+
+// ------------------------------------------------ tcgen05 (5th-gen tensor core)
+// Thin wrappers of the PTX instructions the tensor-core table build uses.
+
+// Tensor memory: one warp allocates ncols (a power of two >= 32) columns of
+// the SM's 512 and writes their base address to *dst (shared memory); the
+// same warp frees them before the CTA exits.
+__device__ __forceinline__ void tmem_alloc(unsigned *dst, unsigned ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                     smem_addr(dst)),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(unsigned taddr, unsigned ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand without swizzle: core
+// matrices of 8 rows x 16 bytes stored contiguously; lbo = bytes between
+// core matrices adjacent along K, sbo = bytes between groups of 8 rows.
+__device__ __forceinline__ uint64_t smem_desc_kmajor(const void *p, unsigned lbo, unsigned sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((smem_addr(p) >> 4) & 0x3FFFu);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;  // descriptor version of this architecture
+    return d;                // base offset 0, no swizzle
+}
+
+// Instruction descriptor of kind::tf32: fp32 accumulator, tf32 A and B,
+// both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+    return (1u << 4)                    // D: fp32
+           | (2u << 7) | (2u << 10)     // A, B: tf32
+           | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// D[tmem] (+)= A * B, issued by one thread.
+__device__ __forceinline__ void mma_tf32(unsigned tmem_d, uint64_t a, uint64_t b, uint32_t idesc,
+                                         bool accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
+        "l"(a), "l"(b), "r"(idesc), "r"((unsigned)accumulate)
+        : "memory");
+}
+
+// The mbarrier at `bar` gets one arrival when every tcgen05.mma this thread
+// issued so far has completed.
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
+            smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+
+// Wait until the phase with parity `parity` of the mbarrier has completed,
+// polling at most max_polls times; false when it gave up.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, unsigned parity,
+                                                  unsigned max_polls) {
+    for (unsigned i = 0; i < max_polls; ++i) {
+        unsigned done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}\n"
+            : "=r"(done)
+            : "r"(smem_addr(bar)), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void tc_fence_before_sync() {
+    asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after_sync() {
+    asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+}
+// Make this thread's generic-proxy writes to shared memory visible to the
+// tensor core (async proxy).
+__device__ __forceinline__ void fence_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+}
+
+// 32 consecutive fp32 columns of the warp's TMEM lane quarter: lane i of the
+// warp gets row (taddr lane field) + i, columns col .. col + 31.
+__device__ __forceinline__ void tmem_ld32(unsigned taddr, float (&v)[32]) {
+    unsigned r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, "
+        "[%32];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// fp32 value with the 13 low mantissa bits cleared: exactly representable
+// in tf32, so the tensor core reads it unchanged.
+__device__ __forceinline__ float tf32_hi(float x) {
+    return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
 }
 
 // Byte b (0..3) of w, zero-extended.
@@ -373,13 +485,15 @@ __device__ __forceinline__ void accumulate(float (&acc)[P], F v) {
 
 }  // namespace qcnn
 
-// ------------------------------------------------------- debug-build checks
-// QCNN_CHECK(cond, flag): in builds with QCNN_DEBUG_CHECKS, a kernel thread
-// that finds `cond` false ORs `flag` into its translation unit's record and
-// goes on (the kernels still clamp, so nothing is read out of bounds); the
-// host collects the records at the next synchronizing call.  Release builds
-// compile it to nothing.
-#ifdef QCNN_DEBUG_CHECKS
+// ------------------------------------------------------- device check record
+// Every translation unit keeps its kernels' flags (QCNN_CHECK_* bits of
+// include/qcnn.h) in a device word of its own and registers a host function
+// that reads and clears it; qcnn_device_check collects them all.
+//  * QCNN_CHECK(cond, flag): only in builds with QCNN_DEBUG_CHECKS, a thread
+//    that finds `cond` false ORs `flag` into the record and goes on (the
+//    kernels still clamp, so nothing is read out of bounds).  Release builds
+//    compile it to nothing.
+//  * QCNN_RECORD_IF(cond, flag): in every build (waits that gave up).
 namespace qcnn {
 namespace {
 __device__ unsigned g_check_flags;
@@ -392,15 +506,22 @@ qcnn_status read_clear_check_flags(unsigned *flags) {
     *flags |= v;
     return cuda_status(e);
 }
+// Release builds read back only the units whose kernels record in every
+// build (they define QCNN_UNIT_RECORDS before including this header): each
+// read is a synchronous copy.
+#if defined(QCNN_DEBUG_CHECKS) || defined(QCNN_UNIT_RECORDS)
 struct CheckReaderRegistration {
     CheckReaderRegistration() { register_check_reader(&read_clear_check_flags); }
 } g_check_reader_registration;
+#endif
 }  // namespace
 }  // namespace qcnn
-#define QCNN_CHECK(cond, flag)                                             \
+#define QCNN_RECORD_IF(cond, flag)                                         \
     do {                                                                   \
-        if (!(cond)) atomicOr(&qcnn::g_check_flags, (unsigned)(flag));     \
+        if (cond) atomicOr(&qcnn::g_check_flags, (unsigned)(flag));        \
     } while (0)
+#ifdef QCNN_DEBUG_CHECKS
+#define QCNN_CHECK(cond, flag) QCNN_RECORD_IF(!(cond), flag)
 #else
 #define QCNN_CHECK(cond, flag) \
     do {                       \

@@ -183,7 +183,7 @@ def test_fc_sweep(case):
         assert rel(host(got), ref) <= TOL
 
 
-# Small batches (N <= 8, K <= 32) run one cluster kernel: (N, Cs, Ct, Csp, K)
+# Small batches (the sub-spaces split over many CTAs): (N, Cs, Ct, Csp, K)
 FC_SMALL = [
     (1, 9216, 4096, 4, 32),    # fc6 at batch 1
     (1, 4096, 1000, 4, 32),    # fc8 at batch 1: ragged last tile
@@ -191,8 +191,8 @@ FC_SMALL = [
     (3, 96, 70, 3, 5),         # odd batch, K not a power of two, tiny M
     (5, 64, 1030, 8, 32),      # Ct % 4 == 2: codes copied byte by byte
     (2, 40, 64, 1, 2),         # C's = 1, K = 2
-    (7, 2304, 513, 4, 32),     # many sub-spaces per CTA (several code chunks)
-    (1, 12, 3, 4, 32),         # M = 3 < cluster size: CTAs without sub-spaces
+    (7, 2304, 513, 4, 32),     # many sub-spaces
+    (1, 12, 3, 4, 32),         # M = 3
 ]
 
 
@@ -200,8 +200,6 @@ FC_SMALL = [
 def test_fc_small_batch(case):
     N, Cs, Ct, Csp, K = case
     M = Cs // Csp
-    plan = q.fc_plan(N, Cs, Ct, Csp, K)
-    assert plan["images"] <= 8 and plan["splits"] <= 16, plan  # the cluster kernel
     x = synth.normal((N, Cs), 1.0, 24, *case)
     D = synth.normal((M, K, Csp), 0.5, 25, *case)
     codes = synth.uniform_codes((M, Ct), K, 26, *case)
@@ -458,6 +456,42 @@ def test_some_small_batch_plans_use_clusters():
     clustered = [q.conv_plan(*c[:9], Csp=c[9], K=c[10], packed=False)["cluster"] > 1
                  for c in CLUSTER]
     assert sum(clustered) >= 4, clustered
+
+
+# The table build on the tensor cores (tcgen05.mma kind::tf32, 3xTF32 split
+# of both operands), forced through the ABI on every tile variant that has
+# it: C'_s 5..8, K a multiple of 32, maps of VGG sizes and ragged ones.
+TC_CASES = [
+    (1, 32, 56, 56, 64, 3, 3, 1, 1, 8, 128),    # VGG 56x56 tile shape
+    (2, 48, 28, 28, 80, 3, 3, 1, 1, 8, 64),     # 28x28, ragged channel tile
+    (1, 40, 14, 14, 130, 3, 3, 1, 1, 5, 32),    # C'_s = 5 (zero slots), K = 32
+    (3, 16, 9, 11, 20, 3, 3, 1, 0, 8, 96),      # small map, K = 96, no padding
+]
+
+
+@pytest.mark.parametrize("case", TC_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_tensor_core_table_build(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(51, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    xi, Di, ci, bi = conv_case(52, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=True)
+    refi = oracle.conv_forward(xi, Di, ci, kh, kw, s, p, bi)
+    ran = 0
+    for v, info in enumerate(q.fused_variants()):
+        if not info["TC"]:
+            continue
+        try:
+            got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b),
+                                      relu=True, algo=v))
+        except q.QcnnError as e:
+            assert e.status == 2, (v, info)  # the variant cannot serve the shape
+            continue
+        assert rel(got, ref) <= TOL, (v, info)
+        goti = host(q.conv_forward(cuda(xi), cuda(Di), cuda(ci), kh, kw, s, p, cuda(bi), algo=v))
+        assert np.array_equal(goti.astype(np.float64), refi), (v, info)
+        ran += 1
+    assert ran >= 1
+    assert q.device_check() == 0  # no tensor-core wait gave up
 
 
 # Every instantiated fused tile variant, forced through the C ABI (the

@@ -60,19 +60,12 @@ def _noalloc(lib, x, D, codes, bias, Ct, relu, stream):
     return y
 
 
-@pytest.mark.parametrize("shape,scratch", [((16, 4096, 1000, 4, 32), True),
-                                           ((32, 512, 256, 4, 16), True),
-                                           ((8, 9216, 4096, 4, 32), False)])
-def test_noalloc_matches_workspace_entry_point_twice(shape, scratch):
-    """Batches of 16 and 32 split their sub-spaces with partial sums in the
-    fixed scratch; batch 8 runs the cluster kernel, which needs none."""
+@pytest.mark.parametrize("shape", [(8, 9216, 4096, 4, 32), (8, 512, 256, 4, 16)])
+def test_noalloc_matches_workspace_entry_point_twice(shape):
     lib = _lib.load()
     N, Cs, Ct, Csp, K = shape
     need = _ws_bytes(lib, *shape)
-    if scratch:
-        assert 0 < need <= LIMIT, "the case must use the fixed scratch and fit in it"
-    else:
-        assert need == 0, "the case must need no scratch"
+    assert 0 < need <= LIMIT, "the case must use the fixed scratch and fit in it"
     stream = torch.cuda.current_stream().cuda_stream
     for call, seed in enumerate((101, 202)):  # two calls in a row, different data
         x, D, codes, bias = _case(seed, *shape)
