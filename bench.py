@@ -47,6 +47,9 @@ def parse():
                    help="skip the model-blob and quantizer measurements")
     p.add_argument("--cpu-sample", type=int, default=0,
                    help="images in the CPU-baseline sample (default: one per worker)")
+    p.add_argument("--layer", default="",
+                   help="WORKLOAD:INDEX -- time that one layer alone at --batch (warm-up, "
+                        "then --steps launches; for profiling) and print one JSON line")
     return p.parse_args()
 
 
@@ -570,10 +573,65 @@ def stage_rooflines(w, cm, stage_ms, N, smem_gbs, hbm_gbs):
     return out
 
 
+def layer_arm(a):
+    """One layer of a workload, alone, at --batch: --warmup untimed launches,
+    then --steps launches timed with CUDA events (L2 flushed before each).
+    For kernel profiles of a single layer (ncu -k / -s / -c)."""
+    import torch
+
+    import paper_1512_06473_gb300 as q
+    name, idx = a.layer.split(":")
+    idx = int(idx)
+    dev = torch.device("cuda", 0)
+    w = synth.WORKLOADS[name]
+    params = w.params()
+    lay = build_layers(q, torch, w, params, dev)
+    qL, (sin, sout) = lay[idx], w.shapes()[idx]
+    N = a.batch
+    x = torch.from_numpy(synth.relu_normal((N, *sin), 0, idx)).to(dev)
+    y = torch.empty((N, *sout), dtype=torch.float32, device=dev)
+    ws = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def run():
+        if isinstance(qL, q.ConvLayer):
+            q.conv_forward(x, qL.D, qL.codes, qL.kh, qL.kw, qL.stride, qL.pad, qL.bias, qL.relu,
+                           packed=True, Ct=qL.Ct, out=y, workspace=ws)
+        elif isinstance(qL, q.FCLayer):
+            q.fc_forward(x.reshape(N, -1), qL.D, qL.codes, qL.bias, qL.relu,
+                         out=y.reshape(N, -1), workspace=ws)
+        else:
+            q.maxpool(x, qL.k, qL.s, out=y)
+
+    for _ in range(a.warmup):
+        run()
+    ts = []
+    for _ in range(a.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        run()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        ts.append(e0.elapsed_time(e1))
+    plan = None
+    if isinstance(qL, q.ConvLayer):
+        plan = q.conv_plan(N, sin[0], sin[1], sin[2], qL.Ct, qL.kh, qL.kw, qL.stride, qL.pad,
+                           w.layers[idx].Csp, w.layers[idx].K)
+    elif isinstance(qL, q.FCLayer):
+        L = w.layers[idx]
+        plan = q.fc_plan(N, L.Cs, L.Ct, L.Csp, L.K)
+    print(json.dumps({"layer": a.layer, "batch": N, "ms_median": float(np.median(ts)),
+                      "steps": a.steps, "plan": plan}), flush=True)
+    return 0
+
+
 def main():
     a = parse()
     if a.impl == "reference":
         return reference_arm(a)
+    if a.layer:
+        return layer_arm(a)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -7,6 +7,8 @@
 #include <atomic>
 #include <climits>
 #include <mutex>
+#include <string>
+#include <unordered_map>
 #include <vector>
 
 namespace qcnn {
@@ -81,15 +83,9 @@ qcnn_status sync_and_check(cudaStream_t st) {
 }
 
 int cluster_capacity(const void *kernel, int threads, int C, size_t smem) {
-    struct Entry {
-        int dev;
-        const void *k;
-        int threads, C;
-        size_t smem;
-        int n;
-    };
     static std::mutex mu;
-    static std::vector<Entry> cache;
+    // keyed by (device, kernel, threads, C, smem); planning asks for hundreds
+    static std::unordered_map<std::string, int> cache;
     int dev = 0, ndev = 0;
     if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev < 1 || cudaGetDevice(&dev) != cudaSuccess) {
         // No GPU (planning on a build host, e.g. for plan queries): the
@@ -101,11 +97,13 @@ int cluster_capacity(const void *kernel, int threads, int C, size_t smem) {
         const int sms_in_clusters = C <= 2 ? 152 : C == 4 ? 146 : C == 8 ? 128 : 112;
         return per_sm * sms_in_clusters / C;
     }
+    std::string key(reinterpret_cast<const char *>(&kernel), sizeof kernel);
+    const long long rest[4] = {dev, threads, C, (long long)smem};
+    key.append(reinterpret_cast<const char *>(rest), sizeof rest);
     {
         std::lock_guard<std::mutex> g(mu);
-        for (const Entry &e : cache)
-            if (e.dev == dev && e.k == kernel && e.threads == threads && e.C == C && e.smem == smem)
-                return e.n;
+        const auto it = cache.find(key);
+        if (it != cache.end()) return it->second;
     }
     int n = 0;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
@@ -127,7 +125,7 @@ int cluster_capacity(const void *kernel, int threads, int C, size_t smem) {
     }
     cudaGetLastError();
     std::lock_guard<std::mutex> g(mu);
-    cache.push_back({dev, kernel, threads, C, smem, n});
+    cache.emplace(std::move(key), n);
     return n;
 }
 
@@ -272,6 +270,44 @@ qcnn_status plan_conv_call(const ConvShape &s, int codes_layout, int algo, ConvC
         off += align_up(c->fp.partial_bytes, kWsAlign);
     }
     c->total = off;
+    return QCNN_OK;
+}
+
+// Plans of single conv calls, cached like the net plans: planning a layer
+// tries every tile variant, split count and cluster size (with cached
+// occupancy queries), tens of microseconds of host time, which at batch 1 is
+// as long as the layer.  Keyed by device, shape, code layout and algorithm;
+// at most kConvPlanCache entries, oldest replaced first.
+constexpr size_t kConvPlanCache = 32;
+qcnn_status plan_conv_call_cached(const ConvShape &s, int codes_layout, int algo, ConvCall *c) {
+    static std::mutex mu;
+    static std::vector<std::pair<std::vector<int>, ConvCall>> cache;
+    static size_t next = 0;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        dev = -1;
+    }
+    const std::vector<int> key = {dev,  s.N,  s.Cs,   s.H,          s.W,  s.Ct,   s.kh,
+                                  s.kw, s.stride, s.pad, s.Csp,     s.K,  s.bf16, codes_layout,
+                                  algo};
+    {
+        std::lock_guard<std::mutex> g(mu);
+        for (const auto &e : cache)
+            if (e.first == key) {
+                *c = e.second;
+                return QCNN_OK;
+            }
+    }
+    const qcnn_status rc = plan_conv_call(s, codes_layout, algo, c);
+    if (rc != QCNN_OK) return rc;
+    std::lock_guard<std::mutex> g(mu);
+    if (cache.size() < kConvPlanCache) {
+        cache.emplace_back(key, *c);
+    } else {
+        cache[next] = {key, *c};
+        next = (next + 1) % kConvPlanCache;
+    }
     return QCNN_OK;
 }
 
@@ -691,7 +727,7 @@ qcnn_status qcnn_conv_workspace_size(int N, int Cs, int H, int W, int Ct, int kh
     if (!bytes || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
-    qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    qcnn_status rc = plan_conv_call_cached(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
     *bytes = c.total;
     return QCNN_OK;
@@ -704,7 +740,7 @@ qcnn_status qcnn_conv_plan_info(int N, int Cs, int H, int W, int Ct, int kh, int
     if (!info || !conv_shape(N, Cs, H, W, Ct, kh, kw, stride, pad, Csp, K, lut_type, &s))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
-    const qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    const qcnn_status rc = plan_conv_call_cached(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
     for (int i = 0; i < 8; ++i) info[i] = 0;
     info[0] = c.algo;
@@ -765,7 +801,7 @@ qcnn_status qcnn_conv_forward(const float *x, int N, int Cs, int H, int W, int C
         (codes_layout == QCNN_CODES_PACKED && !aligned(codes, 16)))
         return QCNN_ERR_INVALID_ARG;
     ConvCall c;
-    qcnn_status rc = plan_conv_call(s, codes_layout, algo, &c);
+    qcnn_status rc = plan_conv_call_cached(s, codes_layout, algo, &c);
     if (rc != QCNN_OK) return rc;
     if (!ws_ok(workspace, workspace_bytes, c.total)) return QCNN_ERR_WORKSPACE;
     PdlScope pdl;

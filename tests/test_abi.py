@@ -230,8 +230,8 @@ def test_fused_variant_table():
     for v in range(n):
         assert lib.qcnn_conv_fused_variant_info(v, info) == 0
         P, CTW, WP, CSP4, NW, MINB, PIPE, BF, SK, TC = list(info)
-        if TC:  # tensor-core build: fp32 tables, C'_s width 8, one buffer, one CTA per SM
-            assert CSP4 == 8 and not (PIPE or BF or SK) and MINB == 1
+        if TC:  # tensor-core build: fp32 tables, 8-wide sub-vectors, one buffer, 1 CTA per SM
+            assert CSP4 == 8 and not (PIPE or BF) and MINB == 1
             seen_tc = True
         assert P >= 1 and (CTW in (4, 8) or CTW % 16 == 0)
         assert CSP4 in (4, 8) and NW in (8, 12, 16, 32) and MINB in (1, 2)
