@@ -234,7 +234,15 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
                                               fv.PIPE ? 2 : 1, fv.TC ? n_mt * 128 : 0)
                                 .total;
         if (smem > (size_t)smem_optin) continue;
-        const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem + 1024))));
+        // One tensor-core CTA per SM: each allocates all 512 columns of
+        // tensor memory, and an allocation waits until the columns are free.
+        // Two CTAs of one cluster on one SM would wait for each other (the
+        // first frees its columns only after the cluster's barrier), so
+        // the shared memory asked for keeps a second CTA off the SM.
+        size_t smem_launch = smem;
+        if (fv.TC) smem_launch = std::max(smem, ((size_t)smem_sm / 2 + 1024 + 15) / 16 * 16);
+        if (smem_launch > (size_t)smem_optin) continue;
+        const int cps = std::max(1, std::min(fv.MINB, (int)(smem_sm / (smem_launch + 1024))));
         if (fv.TC && cps != 1) continue;
         const int ct_tiles = cdiv(s.Ct, ct_cta);
         const double ctas = (double)s.N * pos_tiles * ct_tiles;
@@ -270,7 +278,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
                 double slots = (double)sms * cps;
                 if (c > 1) {
                     const int cap = cluster_capacity(reinterpret_cast<const void *>(fv.fn),
-                                                     fv.NW * 32, c, smem);
+                                                     fv.NW * 32, c, smem_launch);
                     if (cap < 1) continue;
                     slots = std::min(slots, (double)cap * c);
                 }
@@ -346,7 +354,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
             best.ct_cta = ct_cta;
             best.pos_tiles = pos_tiles;
             best.ct_tiles = ct_tiles;
-            best.smem = smem;
+            best.smem = smem_launch;
             best.xs_floats = xs_floats;
             best.score = score;
         }
@@ -365,7 +373,8 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
 
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias,
-                              float *y, int relu, float *partial_ws, cudaStream_t st) {
+                              float *y, int relu, float *partial_ws, cudaStream_t st,
+                              bool early) {
     const FusedVariant &fv = fused_table()[p.variant];
     ConvFusedArgs a;
     a.x = x;
@@ -402,6 +411,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
     a.sk_extra = p.sk_extra;
     a.pos_tiles = p.pos_tiles;
     a.ct_tiles = p.ct_tiles;
+    a.early = early ? 1 : 0;
     cudaError_t e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e == cudaSuccess && p.cl > 8)

@@ -28,6 +28,11 @@ struct ConvFusedArgs {
     // partial[c][0] (sub-spaces before the cut) and partial[c][1] (after),
     // each [CT_CTA][ST] over the tile's positions
     int sk, sk_base, sk_extra, pos_tiles, ct_tiles;
+    // 1: D and the packed codes are the caller's and no kernel of the same
+    // call writes them, so the first sub-space's D and codes are staged
+    // before the wait on the previous kernel (programmatic dependent launch),
+    // their fetch overlapping that kernel's tail; only x waits
+    int early;
 };
 
 // Shared memory carve-up of the fused kernel (byte offsets, 16-aligned);
@@ -121,7 +126,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
-    grid_dep_sync();
+    // (the tensor-core variants allocate tensor memory, which the kernel
+    // before may still hold: they wait first)
+    const bool early = !TC && a.early;
+    if (!early) grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wp = warp % WP, wc = warp / WP;
@@ -169,7 +177,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
     // position l0): halo position h is input (iy, ix) = (r - pad, c - pad)
     // with l0 + h = r*pitch + c, zero-filled where that falls in the padding;
     // sub-vector slots j >= C'_s stay zero.
-    auto stage_xd = [&](int m, int b, int n, int l0) {
+    auto stage_x = [&](int m, int b, int n, int l0) {
         float *xb = xs + b * a.xs_floats;
         const float *xn = a.x + ((size_t)n * a.Cs + (size_t)m * a.Csp) * HW;
         for (int h = tid; h < HP; h += NT) {
@@ -181,11 +189,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 cp_async4(xb + (TC ? tc_off(h, j) : h * CSP4 + j),
                           ok ? src + (size_t)j * HW : a.x, ok);
         }
+    };
+    auto stage_d = [&](int m, int b) {
         float *db = ds + b * K * CSP4;
         const float *dm = a.D + (size_t)m * K * a.Csp;
         for (int k = tid; k < K; k += NT)
             for (int j = 0; j < a.Csp; ++j)
                 cp_async4(db + (TC ? tc_off(k, j) : k * CSP4 + j), dm + k * a.Csp + j, true);
+    };
+    auto stage_xd = [&](int m, int b, int n, int l0) {
+        stage_x(m, b, n, l0);
+        stage_d(m, b);
     };
     // codes of sub-space m, channels ct0 ..; 16-byte pieces past the packed
     // row (CtP, a multiple of 256, may be short of the last tile) are zeros
@@ -199,6 +213,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             else
                 *reinterpret_cast<uint4 *>(cb + pk * CT_CTA + q * 16) = make_uint4(0, 0, 0, 0);
         }
+    };
+    // first stage of the CTA (sub-space m, and m+1's D and x when m2 is
+    // set): the constants first, then the wait on the previous kernel
+    auto stage_first = [&](int m, bool m2, int n, int l0, int ct0) {
+        stage_d(m, 0);
+        if (m2) stage_d(m + 1, 1);
+        stage_codes(m, 0, ct0);
+        if (early) grid_dep_sync();
+        stage_x(m, 0, n, l0);
+        if (m2) stage_x(m + 1, 1, n, l0);
+        cp_async_commit();
     };
 
     // ---- build: lut[k][h] = <x(h), D[m][k]>; lanes on k, warps on h -------
@@ -445,9 +470,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         // and last tile of the range may be cut (partial pieces)
         int m = (int)(u % a.M);
         int piece_m0 = m;  // first sub-space of the current piece
-        stage_xd(m, 0, sn, sl0);
-        stage_codes(m, 0, sct0);
-        cp_async_commit();
+        stage_first(m, false, sn, sl0, sct0);
         for (int b = 0;; b ^= 1) {
             cp_async_wait<0>();
             __syncthreads();  // unit u staged; gather of the previous unit finished
@@ -490,9 +513,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
         return;
     } else if constexpr (!PIPE) {
-        stage_xd(mb, 0, sn, sl0);
-        stage_codes(mb, 0, sct0);
-        cp_async_commit();
+        stage_first(mb, false, sn, sl0, sct0);
         for (int m = mb; m < me; ++m) {
             const int b = (m - mb) & 1;
             cp_async_wait<0>();
@@ -510,10 +531,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
         }
     } else {
         float *lut1 = lut0 + (size_t)K * KS;
-        stage_xd(mb, 0, sn, sl0);
-        if (mb + 1 < me) stage_xd(mb + 1, 1, sn, sl0);
-        stage_codes(mb, 0, sct0);
-        cp_async_commit();
+        stage_first(mb, mb + 1 < me, sn, sl0, sct0);
         cp_async_wait<0>();
         __syncthreads();
         if constexpr (BF) build_bf16(0, lut0);

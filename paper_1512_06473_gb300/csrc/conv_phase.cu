@@ -38,6 +38,10 @@ struct PhaseArgs {
     int pitch, dymin, dxmin, HP, KS, CtP, relu, xs_floats;
     int splits, units_per_split;
     int cl;  // the splits of a tile form clusters of cl CTAs (1: none)
+    // 1: D and the packed codes are constants of the caller (no kernel of the
+    // same call writes them): the first sub-space's are staged before the
+    // wait on the previous kernel
+    int early;
 };
 
 struct PhaseSmem {
@@ -75,7 +79,7 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
-    grid_dep_sync();
+    if (!a.early) grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int l0 = blockIdx.x * ST, ct0 = blockIdx.y * CT_CTA;
@@ -219,8 +223,9 @@ __global__ void __launch_bounds__(NW * 32, 1) conv_phase_kernel(const PhaseArgs 
     };
 
     // ---- units [ub, ue): one table buffer, two barriers per unit ----------
-    stage_x(ub, 0);
     stage_m(ub / S2);
+    if (a.early) grid_dep_sync();
+    stage_x(ub, 0);
     cp_async_commit();
     for (int u = ub, b = 0; u < ue; ++u, b ^= 1) {
         cp_async_wait<0>();
@@ -417,7 +422,7 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl) {
 
 qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias, float *y,
-                              int relu, float *partial_ws, cudaStream_t st) {
+                              int relu, float *partial_ws, cudaStream_t st, bool early) {
     const PhaseVariant &pv = kPhase[p.variant];
     PhaseArgs a;
     a.x = x;
@@ -451,6 +456,7 @@ qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const 
     a.splits = p.splits;
     a.units_per_split = p.units_per_split;
     a.cl = p.cl;
+    a.early = early ? 1 : 0;
     cudaError_t e = cudaFuncSetAttribute(pv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);

@@ -50,6 +50,10 @@ struct FcArgs {
     int cpitch;  // packed: bytes per code row (multiple of 16)
     int crb;     // bytes per staged code row in shared memory (CT_CTA + 16)
     int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
+    // 1: D and the codes are constants of the caller (no kernel of the same
+    // call writes them): the first chunk's are staged before the wait on the
+    // previous kernel (programmatic dependent launch), only x after it
+    int early;
 };
 
 constexpr int kFcThreads = 256;
@@ -101,7 +105,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
     uint8_t *cs = smem + L.cs;
-    grid_dep_sync();
+    if (!a.early) grid_dep_sync();
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wn = warp % WN, wc = warp / WN;
@@ -115,7 +119,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     const int CCH = a.MCH * a.Csp;  // staged x floats per image
     const unsigned kmax4 = (unsigned)(a.K - 1) * 0x01010101u;
 
-    auto stage = [&](int c, int b) {
+    auto stage_x = [&](int c, int b) {
         const int m0 = c * a.MCH;
         const int mch = min(a.MCH, a.M - m0);
         float *xb = xs + (size_t)b * CCH * a.NTX;
@@ -128,6 +132,10 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
             const float *src = ok ? a.x + (size_t)(n0 + nn) * a.Cs + (size_t)m0 * a.Csp + cc : a.x;
             cp_async4(xb + cc * a.NTX + nn, src, ok);
         }
+    };
+    auto stage_w = [&](int c, int b) {  // sub-codebooks and codes of chunk c
+        const int m0 = c * a.MCH;
+        const int mch = min(a.MCH, a.M - m0);
         float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
         const int dn = a.MCH * a.K * a.Csp, dv = mch * a.K * a.Csp;
         const float *dsrc = a.D + (size_t)m0 * a.K * a.Csp;
@@ -173,6 +181,10 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 cb[mm * a.crb + q] = (mm < mch && ct < a.Ct) ? a.codes[(size_t)(m0 + mm) * a.Ct + ct] : 0;
             }
         }
+    };
+    auto stage = [&](int c, int b) {
+        stage_x(c, b);
+        stage_w(c, b);
         cp_async_commit();
     };
 
@@ -182,7 +194,12 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
 #pragma unroll
         for (int i = 0; i < NW; ++i) acc[c][i] = 0.f;
 
-    if (c_begin < c_end) stage(c_begin, 0);
+    if (c_begin < c_end) stage_w(c_begin, 0);
+    if (a.early) grid_dep_sync();
+    if (c_begin < c_end) {
+        stage_x(c_begin, 0);
+        cp_async_commit();
+    }
     for (int c = c_begin; c < c_end; ++c) {
         const int b = (c - c_begin) & 1;
         const int mch = min(a.MCH, a.M - c * a.MCH);
@@ -375,7 +392,11 @@ static const FcVariant kFcVariants[] = {
     QCNN_FC(16, 2, 2, 0.8),   QCNN_FC(8, 2, 3, 0.84),   QCNN_FC(8, 4, 3, 0.6),
     QCNN_FC(4, 1, 3, 1.0),    QCNN_FC(1, 1, 3, 0.5),    QCNN_FC_BF(16, 2, 2, 0.8),
     QCNN_FC_BF(8, 2, 3, 0.84), QCNN_FC_BF(8, 4, 3, 0.6), QCNN_FC_BF(4, 1, 3, 1.0),
-    QCNN_FC_BF(1, 1, 3, 0.5), QCNN_FC(16, 1, 2, 1.2),  QCNN_FC_BF(16, 1, 2, 1.2)};
+    QCNN_FC_BF(1, 1, 3, 0.5), QCNN_FC(16, 1, 2, 1.2),  QCNN_FC_BF(16, 1, 2, 1.2),
+#ifdef QCNN_TUNING
+    QCNN_FC(1, 1, 4, 0.5),
+#endif
+};
 #undef QCNN_FC_BF
 #undef QCNN_FC
 constexpr int kNumFc = sizeof(kFcVariants) / sizeof(kFcVariants[0]);
@@ -404,6 +425,9 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         const int row_bytes = fc_row_bytes(NT, NTP, fv.BF);
         // largest chunk that lets MINB CTAs share an SM
         int MCH = std::min(kMchMax, std::max(1, 512 / s.K));
+#ifdef QCNN_TUNING
+        if (const char *e = getenv("QCNN_FC_MCH")) MCH = std::max(1, std::min(kMchMax, atoi(e)));
+#endif
         while (MCH > 1 &&
                (fc_smem_layout(MCH, s.K, row_bytes, NTX, s.Csp, CT_CTA).total + 1024) *
                        fv.MINB > sm_bytes)
@@ -416,6 +440,9 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         const int tiles = n_tiles * ct_tiles;
         const int target = 2 * sms * cps_sm;
         int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
+#ifdef QCNN_TUNING
+        if (const char *e = getenv("QCNN_FC_SPLITS")) splits = std::max(1, std::min(n_chunks, atoi(e)));
+#endif
         // at most max_partial_bytes of partial sums [splits][N][Ct]
         const size_t per_split = (size_t)s.N * s.Ct * sizeof(float);
         const size_t cap = max_partial_bytes / per_split;
@@ -489,6 +516,7 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.crb = p.CT_CTA + 16;
     a.cch_log2 = 0;
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
+    a.early = 1;  // no kernel of a library call writes D or the codes
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return cuda_status(e);

@@ -318,6 +318,9 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
         return launch_conv_chunked(c.s, c.cp, x, D, codes, codes_layout == QCNN_CODES_PACKED, bias,
                                    y, relu, static_cast<uint8_t *>(ws) + c.lut_off, st);
     const uint8_t *packed = codes;
+    // codes packed by this call are written by a kernel of the call: the
+    // conv kernel then reads them only after its wait on that kernel
+    const bool early = codes_layout == QCNN_CODES_PACKED;
     if (codes_layout == QCNN_CODES_CANONICAL) {
         uint8_t *p = static_cast<uint8_t *>(ws) + c.packed_off;
         qcnn_status rc =
@@ -327,9 +330,9 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
     }
     float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
     if (c.algo == QCNN_ALGO_FUSED)
-        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, lut, st);
+        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, lut, st, early);
     if (c.algo == QCNN_ALGO_PHASE)
-        return launch_conv_phase(c.s, c.pp, x, D, packed, bias, y, relu, lut, st);
+        return launch_conv_phase(c.s, c.pp, x, D, packed, bias, y, relu, lut, st, early);
     return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
 }
 

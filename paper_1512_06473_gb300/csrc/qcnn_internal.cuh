@@ -178,7 +178,7 @@ struct ConvPhasePlan {
 ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl = 0);
 qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias, float *y,
-                              int relu, float *partial_ws, cudaStream_t st);
+                              int relu, float *partial_ws, cudaStream_t st, bool early = false);
 
 size_t packed_codes_bytes(int Ct, int kk, int M);
 int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
@@ -192,7 +192,8 @@ qcnn_status launch_split_reduce(const float *partial, int splits, size_t total, 
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p,
                               const float *x, const float *D,
                               const uint8_t *packed, const float *bias, float *y,
-                              int relu, float *partial_ws, cudaStream_t st);
+                              int relu, float *partial_ws, cudaStream_t st,
+                              bool early = false);
 qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
                                 const float *x, const float *D,
                                 const uint8_t *packed, const float *bias,
