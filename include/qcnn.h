@@ -221,7 +221,9 @@ qcnn_status qcnn_fc_forward(const float *x, int N, int Cs, int Ct,
  * [1] outputs per CTA, [2] CTAs sharing the sub-spaces of one tile (1: no
  * partial sums), [3] sub-spaces per shared-memory chunk, [4] CTAs of the
  * main kernel, [5] CTAs per thread-block cluster among those of [2] (1:
- * none; the FC kernel's partial sums always go through the workspace).
+ * none).  A cluster adds its CTAs' partial sums in distributed shared
+ * memory; only [2] / [5] partial sums per output go through the workspace
+ * (none, and no second kernel, when [5] == [2]).
  * QCNN_ERR_INVALID_ARG as qcnn_fc_workspace_size, or for a NULL info.
  */
 qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K,

@@ -41,6 +41,7 @@ struct FcArgs {
     float *__restrict__ partial;  // [splits][N][Ct] when splits > 1
     int N, Cs, Ct, Csp, K, M;
     int NT, CT_CTA, MCH, n_chunks, chunks_per_split, splits, relu;
+    int cl;  // the splits of a tile form clusters of cl CTAs (1: none)
     int NTP;     // odd pitch of a table row (fp32: floats >= NT; bf16 pairs:
                  // words >= NT/2; bf16 singles: halves >= NT)
     int NTX;     // odd pitch of a staged x row (>= NT)
@@ -185,7 +186,6 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     auto stage = [&](int c, int b) {
         stage_x(c, b);
         stage_w(c, b);
-        cp_async_commit();
     };
 
     float acc[kCPL][NW];
@@ -196,16 +196,17 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
 
     if (c_begin < c_end) stage_w(c_begin, 0);
     if (a.early) grid_dep_sync();
-    if (c_begin < c_end) {
-        stage_x(c_begin, 0);
-        cp_async_commit();
-    }
+    if (c_begin < c_end) stage_x(c_begin, 0);
+    cp_async_commit();
     for (int c = c_begin; c < c_end; ++c) {
         const int b = (c - c_begin) & 1;
         const int mch = min(a.MCH, a.M - c * a.MCH);
         cp_async_wait<0>();
         __syncthreads();  // chunk c staged; gather of c-1 finished
-        if (c + 1 < c_end) stage(c + 1, b ^ 1);
+        if (c + 1 < c_end) {
+            stage(c + 1, b ^ 1);
+            cp_async_commit();
+        }
 
         // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>; (k, nn) with nn
         // fastest over the compile-time image tile: no division
@@ -322,6 +323,31 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
 
     // epilogue
     const int ct_lane = ct0 + lane_ct;
+    if (a.cl > 1) {
+        // the cluster's CTAs (consecutive splits of this tile) add their
+        // partial tiles in distributed shared memory, in rank order; with
+        // more splits than one cluster, each cluster's sum is a partial for
+        // the split reduction
+        __syncthreads();  // every warp is done with the table
+        float *red = reinterpret_cast<float *>(smem);  // [NT][CT_CTA]
+#pragma unroll
+        for (int i = 0; i < NW; ++i)
+#pragma unroll
+            for (int q = 0; q < kCPL; ++q) red[(nbase + i) * CT_CTA + lane_ct + q] = acc[q][i];
+        const int group = split / a.cl, groups = a.splits / a.cl;
+        cluster_tile_reduce(red, NT * CT_CTA, [&](int e, float v) {
+            const int n = n0 + (e >> kCtCtaLog2), ct = ct0 + (e & (CT_CTA - 1));
+            if (n >= a.N || ct >= a.Ct) return;
+            if (groups > 1) {
+                a.partial[((size_t)group * a.N + n) * a.Ct + ct] = v;
+            } else {
+                v += a.bias ? a.bias[ct] : 0.f;
+                if (a.relu) v = fmaxf(v, 0.f);
+                a.y[(size_t)n * a.Ct + ct] = v;
+            }
+        });
+        return;
+    }
 #pragma unroll
     for (int i = 0; i < NW; ++i) {
         const int n = n0 + nbase + i;
@@ -393,9 +419,6 @@ static const FcVariant kFcVariants[] = {
     QCNN_FC(4, 1, 3, 1.0),    QCNN_FC(1, 1, 3, 0.5),    QCNN_FC_BF(16, 2, 2, 0.8),
     QCNN_FC_BF(8, 2, 3, 0.84), QCNN_FC_BF(8, 4, 3, 0.6), QCNN_FC_BF(4, 1, 3, 1.0),
     QCNN_FC_BF(1, 1, 3, 0.5), QCNN_FC(16, 1, 2, 1.2),  QCNN_FC_BF(16, 1, 2, 1.2),
-#ifdef QCNN_TUNING
-    QCNN_FC(1, 1, 4, 0.5),
-#endif
 };
 #undef QCNN_FC_BF
 #undef QCNN_FC
@@ -409,9 +432,12 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
     double best_t = 1e300;
     const int sms = num_sms();
     const size_t sm_bytes = 228 * 1024;
-#ifdef QCNN_TUNING  // tuning builds only: force a variant from the environment
+#ifdef QCNN_TUNING  // tuning builds only: force a variant, split count, chunk or cluster
     const char *force_env = getenv("QCNN_FC_VARIANT");
     const int force = force_env ? atoi(force_env) : -1;
+    const char *sp_env = getenv("QCNN_FC_SPLITS");
+    const char *mch_env = getenv("QCNN_FC_MCH");
+    const char *cl_env = getenv("QCNN_FC_CLUSTER");
 #endif
     for (int v = 0; v < kNumFc; ++v) {
 #ifdef QCNN_TUNING
@@ -426,7 +452,7 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         // largest chunk that lets MINB CTAs share an SM
         int MCH = std::min(kMchMax, std::max(1, 512 / s.K));
 #ifdef QCNN_TUNING
-        if (const char *e = getenv("QCNN_FC_MCH")) MCH = std::max(1, std::min(kMchMax, atoi(e)));
+        if (mch_env) MCH = std::max(1, std::min(kMchMax, atoi(mch_env)));
 #endif
         while (MCH > 1 &&
                (fc_smem_layout(MCH, s.K, row_bytes, NTX, s.Csp, CT_CTA).total + 1024) *
@@ -441,7 +467,7 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         const int target = 2 * sms * cps_sm;
         int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
 #ifdef QCNN_TUNING
-        if (const char *e = getenv("QCNN_FC_SPLITS")) splits = std::max(1, std::min(n_chunks, atoi(e)));
+        if (sp_env) splits = std::max(1, std::min(n_chunks, atoi(sp_env)));
 #endif
         // at most max_partial_bytes of partial sums [splits][N][Ct]
         const size_t per_split = (size_t)s.N * s.Ct * sizeof(float);
@@ -449,8 +475,39 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         if (splits > 1 && (size_t)splits > cap) splits = cap >= 2 ? (int)cap : 1;
         const int cpsplit = cdiv(n_chunks, splits);
         splits = cdiv(n_chunks, cpsplit);
+        // Many splits of several tiles: clusters of 8 CTAs add their partial
+        // tiles in distributed shared memory, so an eighth of the partial
+        // sums goes through the workspace.  Measured (clusters / none): fc6
+        // batch 1 (144 splits, 4 tiles) 17.0 / 19.5 us, fc7 batch 8 24.0 /
+        // 27.8 us, fc8 batch 64 27.9 / 40.4 us; no change for fc7 batch 1,
+        // fc8 batch 8 and 128.  With a single tile (fc8 batch 1: 12.6 / 11.2
+        // us) or fewer splits (fc7 batch 64, 32 splits: 70.7 / 68.1 us) the
+        // cluster's scheduling constraint and barriers cost more than the
+        // partial sums they save.
+        int cl = 1;
+        if (splits >= 64 && tiles >= 2 && (size_t)NT * CT_CTA * sizeof(float) <= smem) {
+            for (int c = 8; c >= 2 && cl == 1; c /= 2)
+                if (splits % c == 0 &&
+                    cluster_capacity(reinterpret_cast<const void *>(fv.fn), kFcThreads, c, smem) >= 1)
+                    cl = c;
+        }
+#ifdef QCNN_TUNING
+        if (cl_env) {
+            const int c = atoi(cl_env);
+            if (c < 1 || splits % c != 0 ||
+                (c > 1 && ((size_t)NT * CT_CTA * sizeof(float) > smem ||
+                           cluster_capacity(reinterpret_cast<const void *>(fv.fn), kFcThreads, c,
+                                            smem) < 1)))
+                continue;
+            cl = c;
+        }
+#endif
+        double slots = (double)cps_sm * sms;
+        if (cl > 1)
+            slots = std::min(slots, (double)cl * cluster_capacity(reinterpret_cast<const void *>(fv.fn),
+                                                                   kFcThreads, cl, smem));
         const double ctas = (double)tiles * splits;
-        const double waves = std::ceil(ctas / ((double)cps_sm * sms));
+        const double waves = std::ceil(ctas / slots);
         // one CTA: shared-memory wavefronts (gather + build) per chunk; a wave
         // of cps_sm co-resident CTAs shares one SM
         const double per_chunk = (double)MCH * NT * CT_CTA / (fv.BF && fv.NW % 2 == 0 ? 64.0 : 32.0) +
@@ -458,9 +515,10 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         const double t_smem = waves * cpsplit * per_chunk * cps_sm / 1.2e9 / fv.eff;
         // (byte codes counted for both code layouts, so that packed and
         // unpacked calls make the same plan and share one workspace query)
+        const int parts = splits / cl;
         const double bytes = (double)s.M * s.Ct * n_tiles + 4.0 * s.N * s.Cs * ct_tiles +
-                             (splits > 1 ? 8.0 * splits * s.N * s.Ct : 0.0);
-        const double t = std::max(t_smem, bytes / 6.0e12) + (splits > 1 ? 3e-6 : 0.0);
+                             (parts > 1 ? 8.0 * parts * s.N * s.Ct : 0.0);
+        const double t = std::max(t_smem, bytes / 6.0e12) + (parts > 1 ? 3e-6 : 0.0);
         if (t < best_t) {
             best_t = t;
             best.variant = v;
@@ -469,11 +527,12 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
             best.MCH = MCH;
             best.n_chunks = n_chunks;
             best.splits = splits;
+            best.cl = cl;
             best.chunks_per_split = cpsplit;
             best.n_tiles = n_tiles;
             best.ct_tiles = ct_tiles;
             best.smem = smem;
-            best.partial_bytes = splits > 1 ? (size_t)splits * s.N * s.Ct * sizeof(float) : 0;
+            best.partial_bytes = parts > 1 ? (size_t)parts * per_split : 0;
         }
     }
     return best;
@@ -517,22 +576,27 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.cch_log2 = 0;
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     a.early = 1;  // no kernel of a library call writes D or the codes
+    a.cl = p.cl;
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    if (e == cudaSuccess && p.cl > 8)
+        e = cudaFuncSetAttribute(fv.fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return cuda_status(e);
-    dim3 grid(p.ct_tiles, p.n_tiles, p.splits);
-    qcnn_status rc = launch_pdl(fv.fn, grid, dim3(kFcThreads), p.smem, st, a);
-    if (rc != QCNN_OK || p.splits == 1) return rc;
+    const dim3 grid(p.ct_tiles, p.n_tiles, p.splits);
+    const dim3 cluster = p.cl > 1 ? dim3(1, 1, p.cl) : dim3(0, 0, 0);
+    qcnn_status rc = launch_k(fv.fn, grid, dim3(kFcThreads), p.smem, st, cluster, a);
+    const int groups = p.splits / p.cl;  // partial sums per output left
+    if (rc != QCNN_OK || groups == 1) return rc;
     const size_t total = (size_t)s.N * s.Ct;
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
-    if (total < 65536 && p.splits >= 16) {
+    if (total < 65536 && groups >= 16) {
         const int wblocks = (int)std::min<size_t>((total * 32 + 255) / 256, (size_t)num_sms() * 16);
         return launch_pdl(fc_reduce_warp_kernel, dim3(wblocks), dim3(256), 0, st,
-                          static_cast<const float *>(partial_ws), p.splits, s.N, s.Ct, bias,
-                          relu, y);
+                          static_cast<const float *>(partial_ws), groups, s.N, s.Ct, bias, relu,
+                          y);
     }
     return launch_pdl(fc_reduce_kernel, dim3(blocks), dim3(256), 0, st,
-                      static_cast<const float *>(partial_ws), p.splits, s.N, s.Ct, bias, relu, y);
+                      static_cast<const float *>(partial_ws), groups, s.N, s.Ct, bias, relu, y);
 }
 
 }  // namespace qcnn

@@ -787,7 +787,7 @@ qcnn_status qcnn_fc_plan_info(int N, int Cs, int Ct, int Csp, int K, int lut_typ
     info[2] = p.splits;
     info[3] = p.MCH;
     info[4] = p.ct_tiles * p.n_tiles * p.splits;
-    info[5] = 1;  // the FC kernel's splits never form clusters
+    info[5] = p.cl;
     return QCNN_OK;
 }
 

@@ -220,10 +220,13 @@ struct FcPlan {
     int MCH;            // sub-spaces per shared-memory chunk
     int n_chunks;       // ceil(M / MCH)
     int splits;         // CTAs along m (partial sums reduced afterwards)
+    int cl = 1;         // splits form clusters of cl CTAs that add their partial
+                        // tiles in distributed shared memory (splits / cl
+                        // partial sums per output left for the reduction)
     int chunks_per_split;
     int n_tiles, ct_tiles;
     size_t smem;
-    size_t partial_bytes;  // workspace for split partial sums (0 if splits == 1)
+    size_t partial_bytes;  // workspace for split partial sums (0 if splits == cl)
 };
 // max_partial_bytes: no split count whose partial sums need more is chosen
 // (1 split, without partial sums, always fits)

@@ -363,7 +363,26 @@ def test_batch1_plans_split_the_subspaces():
         assert p["splits"] > 1 and p["stream_k"] == 0 and p["ctas"] >= 64, (name, p)
     for name, (Cs, Ct) in ALEX_FC.items():
         f = q.fc_plan(1, Cs, Ct)
-        assert f["images"] == 1 and f["splits"] >= 64 and f["cluster"] == 1, (name, f)
+        # one image per CTA, the sub-spaces over >= 64 CTAs; with several
+        # output tiles (fc6, fc7) clusters of 8 add their partial sums in
+        # distributed shared memory first
+        assert f["images"] == 1 and f["splits"] >= 64, (name, f)
+        assert f["cluster"] == (8 if Ct > 1024 else 1), (name, f)
+
+
+@_planner
+def test_fc_clusters_only_with_many_splits():
+    """The FC planner groups split CTAs into clusters only from 64 splits
+    up (fewer splits measured slower with clusters), and then into clusters
+    that divide the split count."""
+    import paper_1512_06473_gb300 as q
+    for N in (1, 2, 8, 16, 64, 128, 256):
+        for Cs, Ct in list(ALEX_FC.values()) + [(512, 256)]:
+            f = q.fc_plan(N, Cs, Ct, K=16 if Cs == 512 else 32)
+            assert f["splits"] % f["cluster"] == 0, (N, Cs, Ct, f)
+            if f["splits"] < 64:
+                assert f["cluster"] == 1, (N, Cs, Ct, f)
+            assert f["cluster"] in (1, 2, 4, 8), (N, Cs, Ct, f)
 
 
 def test_plan_info_arguments():
