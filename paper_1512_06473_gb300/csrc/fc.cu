@@ -475,17 +475,19 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         if (splits > 1 && (size_t)splits > cap) splits = cap >= 2 ? (int)cap : 1;
         const int cpsplit = cdiv(n_chunks, splits);
         splits = cdiv(n_chunks, cpsplit);
-        // Many splits of several tiles: clusters of 8 CTAs add their partial
-        // tiles in distributed shared memory, so an eighth of the partial
-        // sums goes through the workspace.  Measured (clusters / none): fc6
-        // batch 1 (144 splits, 4 tiles) 17.0 / 19.5 us, fc7 batch 8 24.0 /
-        // 27.8 us, fc8 batch 64 27.9 / 40.4 us; no change for fc7 batch 1,
-        // fc8 batch 8 and 128.  With a single tile (fc8 batch 1: 12.6 / 11.2
-        // us) or fewer splits (fc7 batch 64, 32 splits: 70.7 / 68.1 us) the
-        // cluster's scheduling constraint and barriers cost more than the
-        // partial sums they save.
+        // Many splits of several tiles of few images: clusters of 8 CTAs add
+        // their partial tiles in distributed shared memory, so an eighth of
+        // the partial sums goes through the workspace.  Measured (clusters /
+        // none): fc6 batch 1 (144 splits, 4 tiles) 17.0 / 19.5 us, fc6 batch
+        // 8 36.9 / 39.0 us, fc7 batch 8 24.0 / 27.8 us; no change for fc7
+        // batch 1 and fc8 batch 8.  With a single tile (fc8 batch 1: 12.6 /
+        // 11.2 us), fewer splits (fc7 batch 64, 32 splits: 70.7 / 68.1 us) or
+        // 16-image tiles (64 KB of partial sums per CTA through distributed
+        // shared memory; fc8 batch 128: 46.8 / 43.0 us in the whole step) the
+        // cluster's scheduling constraint, barriers and remote reads cost
+        // more than the partial sums they save.
         int cl = 1;
-        if (splits >= 64 && tiles >= 2 && (size_t)NT * CT_CTA * sizeof(float) <= smem) {
+        if (splits >= 64 && tiles >= 2 && NT <= 4 && (size_t)NT * CT_CTA * sizeof(float) <= smem) {
             for (int c = 8; c >= 2 && cl == 1; c /= 2)
                 if (splits % c == 0 &&
                     cluster_capacity(reinterpret_cast<const void *>(fv.fn), kFcThreads, c, smem) >= 1)
