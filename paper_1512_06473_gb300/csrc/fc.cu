@@ -466,6 +466,11 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
         const int tiles = n_tiles * ct_tiles;
         const int target = 2 * sms * cps_sm;
         int splits = std::max(1, std::min(n_chunks, (int)std::lround((double)target / tiles)));
+        // 16-image tiles: at least two chunks per CTA (measured: fc8 at batch
+        // 128, 64 chunks, 32 splits 39.6 us against 47.8 us with 64; at batch
+        // 64 37.6 against 41.6 us).  Single-image tiles keep one chunk per CTA
+        // (fc6-8 at batch 1 are fastest with every chunk on its own CTA).
+        if (NT >= 16) splits = std::min(splits, std::max(1, n_chunks / 2));
 #ifdef QCNN_TUNING
         if (sp_env) splits = std::max(1, std::min(n_chunks, atoi(sp_env)));
 #endif
