@@ -51,6 +51,7 @@ struct FcArgs {
     int cpitch;  // packed: bytes per code row (multiple of 16)
     int crb;     // bytes per staged code row in shared memory (CT_CTA + 16)
     int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
+    int dvec16;    // 1: sub-codebooks staged in 16-byte pieces (K * Csp % 4 == 0, D 16-aligned)
     // 1: D and the codes are constants of the caller (no kernel of the same
     // call writes them): the first chunk's are staged before the wait on the
     // previous kernel (programmatic dependent launch), only x after it
@@ -99,9 +100,12 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     constexpr int NT = NW * WN;  // images per CTA (== a.NT)
     constexpr bool PAIRS = BF && NW % 2 == 0;  // bf16 words of two images
     static_assert(!BF || NW % 2 == 0 || NW == 1, "bf16 tiles: even NW or NW == 1");
+    // row pitches of the table and of the staged x (the host passes the same
+    // values in NTP, NTX): compile-time, so row addresses fold
+    constexpr int NTP = (BF && NT % 2 == 0 ? NT / 2 : NT) | 1;
+    constexpr int NTX = NT | 1;
     extern __shared__ __align__(16) unsigned char smem[];
-    const FcSmem L = fc_smem_layout(a.MCH, a.K, fc_row_bytes(NT, a.NTP, BF), a.NTX, a.Csp,
-                                    CT_CTA);
+    const FcSmem L = fc_smem_layout(a.MCH, a.K, fc_row_bytes(NT, NTP, BF), NTX, a.Csp, CT_CTA);
     float *lut = reinterpret_cast<float *>(smem + L.lut);
     float *xs = reinterpret_cast<float *>(smem + L.xs);
     float *ds = reinterpret_cast<float *>(smem + L.ds);
@@ -123,7 +127,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     auto stage_x = [&](int c, int b) {
         const int m0 = c * a.MCH;
         const int mch = min(a.MCH, a.M - m0);
-        float *xb = xs + (size_t)b * CCH * a.NTX;
+        float *xb = xs + (size_t)b * CCH * NTX;
         // (image nn, float cc) with cc on a power-of-two stride: no division
         const int cmask = (1 << a.cch_log2) - 1;
         for (int e = tid; e < (NT << a.cch_log2); e += kFcThreads) {
@@ -131,7 +135,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
             if (cc >= CCH) continue;
             const bool ok = cc < mch * a.Csp && n0 + nn < a.N;
             const float *src = ok ? a.x + (size_t)(n0 + nn) * a.Cs + (size_t)m0 * a.Csp + cc : a.x;
-            cp_async4(xb + cc * a.NTX + nn, src, ok);
+            cp_async4(xb + cc * NTX + nn, src, ok);
         }
     };
     auto stage_w = [&](int c, int b) {  // sub-codebooks and codes of chunk c
@@ -140,7 +144,11 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
         const int dn = a.MCH * a.K * a.Csp, dv = mch * a.K * a.Csp;
         const float *dsrc = a.D + (size_t)m0 * a.K * a.Csp;
-        for (int e = tid; e < dn; e += kFcThreads) cp_async4(db + e, e < dv ? dsrc + e : a.D, e < dv);
+        if (a.dvec16) {  // 16-byte pieces (the build reads only the chunk's mch sub-spaces)
+            for (int e = tid * 4; e < dv; e += kFcThreads * 4) cp_async16(db + e, dsrc + e);
+        } else {
+            for (int e = tid; e < dn; e += kFcThreads) cp_async4(db + e, e < dv ? dsrc + e : a.D, e < dv);
+        }
         // codes[m0 + mm][ct0 .. ct0 + CT_CTA) -> cs[b][mm][.]; zero outside
         uint8_t *cb = cs + (size_t)b * a.MCH * a.crb;
         if (a.cbits) {  // packed rows: this CTA's slice, whole 16-byte copies
@@ -211,7 +219,7 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         // build lut[mm][k][nn] = <x(nn, mm), D[m0 + mm][k]>; (k, nn) with nn
         // fastest over the compile-time image tile: no division
         {
-            const float *xb = xs + (size_t)b * CCH * a.NTX;
+            const float *xb = xs + (size_t)b * CCH * NTX;
             const float *db = ds + (size_t)b * a.MCH * a.K * a.Csp;
             for (int mm = 0; mm < mch; ++mm) {
                 if constexpr (PAIRS) {
@@ -219,28 +227,28 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                     unsigned *lw = reinterpret_cast<unsigned *>(lut);
                     for (int e = tid; e < a.K * NP; e += kFcThreads) {
                         const int np = e % NP, k = e / NP;
-                        const float *xp = xb + mm * a.Csp * a.NTX + 2 * np;
+                        const float *xp = xb + mm * a.Csp * NTX + 2 * np;
                         const float *dp = db + (mm * a.K + k) * a.Csp;
                         float v0 = 0.f, v1 = 0.f;
 #pragma unroll
                         for (int j = 0; j < kMaxCsp; ++j) {
                             if (j < a.Csp) {
-                                v0 = fmaf(xp[j * a.NTX], dp[j], v0);
-                                v1 = fmaf(xp[j * a.NTX + 1], dp[j], v1);
+                                v0 = fmaf(xp[j * NTX], dp[j], v0);
+                                v1 = fmaf(xp[j * NTX + 1], dp[j], v1);
                             }
                         }
-                        lw[(mm * a.K + k) * a.NTP + np] = pack_bf16x2(v0, v1);
+                        lw[(mm * a.K + k) * NTP + np] = pack_bf16x2(v0, v1);
                     }
                 } else if constexpr (BF) {
                     for (int e = tid; e < a.K * NT; e += kFcThreads) {
                         const int nn = e % NT, k = e / NT;
-                        const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                        const float *xp = xb + mm * a.Csp * NTX + nn;
                         const float *dp = db + (mm * a.K + k) * a.Csp;
                         float v = 0.f;
 #pragma unroll
                         for (int j = 0; j < kMaxCsp; ++j)
-                            if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
-                        reinterpret_cast<unsigned short *>(lut)[(mm * a.K + k) * a.NTP + nn] =
+                            if (j < a.Csp) v = fmaf(xp[j * NTX], dp[j], v);
+                        reinterpret_cast<unsigned short *>(lut)[(mm * a.K + k) * NTP + nn] =
                             (unsigned short)(pack_bf16x2(v, 0.f) & 0xffffu);
                     }
                 }
@@ -256,21 +264,21 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                     for (int mm = t_mm; mm < mch; mm += mm_step) {
                         for (int e = t_e; e < per_mm; e += lanes_mm) {
                             const int nn = e % NT, k = e / NT;
-                            const float *xp = xb + mm * a.Csp * a.NTX + nn;
+                            const float *xp = xb + mm * a.Csp * NTX + nn;
                             const float *dp = db + (mm * a.K + k) * a.Csp;
                             float v = 0.f;
                             if (a.Csp == 4) {  // one 16-byte load of the sub-codeword
                                 const float4 d = *reinterpret_cast<const float4 *>(dp);
                                 v = fmaf(xp[0], d.x, v);
-                                v = fmaf(xp[a.NTX], d.y, v);
-                                v = fmaf(xp[2 * a.NTX], d.z, v);
-                                v = fmaf(xp[3 * a.NTX], d.w, v);
+                                v = fmaf(xp[NTX], d.y, v);
+                                v = fmaf(xp[2 * NTX], d.z, v);
+                                v = fmaf(xp[3 * NTX], d.w, v);
                             } else {
 #pragma unroll
                                 for (int j = 0; j < kMaxCsp; ++j)
-                                    if (j < a.Csp) v = fmaf(xp[j * a.NTX], dp[j], v);
+                                    if (j < a.Csp) v = fmaf(xp[j * NTX], dp[j], v);
                             }
-                            lut[(mm * a.K + k) * a.NTP + nn] = v;
+                            lut[(mm * a.K + k) * NTP + nn] = v;
                         }
                     }
                 }
@@ -278,46 +286,50 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         }
         __syncthreads();
 
-        // gather
+        // gather: the lane's 4 codes of sub-space mm, as the bytes of w
         const uint8_t *cb = cs + (size_t)b * a.MCH * a.crb;
-        const int bit0 = lane_ct * a.cbits;  // packed: first bit of the lane's codes
-        const unsigned cmask = (1u << a.cbits) - 1u;
-#pragma unroll
-        for (int mm = 0; mm < kMchMax; ++mm) {
-            if (mm < mch) {
-                unsigned w;
-                if (a.cbits) {  // 4 codes of b bits -> 4 bytes
-                    const unsigned *cw = reinterpret_cast<const unsigned *>(cb + mm * a.crb);
-                    const unsigned v = __funnelshift_r(cw[bit0 >> 5], cw[(bit0 >> 5) + 1], bit0 & 31);
-                    w = (v & cmask) | (((v >> a.cbits) & cmask) << 8) |
-                        (((v >> (2 * a.cbits)) & cmask) << 16) | (((v >> (3 * a.cbits)) & cmask) << 24);
-                } else {
-                    w = *reinterpret_cast<const unsigned *>(cb + mm * a.crb + lane_ct);
-                }
+        auto gather_mm = [&](int mm, unsigned w) {
                 QCNN_CHECK(__vcmpgtu4(w, kmax4) == 0u, QCNN_CHECK_CODE);
                 w = __vminu4(w, kmax4);
 #pragma unroll
                 for (int q = 0; q < kCPL; ++q) {
                     const int code = (int)byte_of(w, q);
-                    QCNN_CHECK((mm * a.K + code + 1) * a.NTP <= a.MCH * a.K * a.NTP,
+                    QCNN_CHECK((mm * a.K + code + 1) * NTP <= a.MCH * a.K * NTP,
                                QCNN_CHECK_TABLE);
                     if constexpr (PAIRS) {
                         const unsigned *row = reinterpret_cast<const unsigned *>(lut) +
-                                              (mm * a.K + code) * a.NTP + nbase / 2;
+                                              (mm * a.K + code) * NTP + nbase / 2;
 #pragma unroll
                         for (int i = 0; i < NW / 2; ++i)
                             add_bf16x2(acc[q][2 * i], acc[q][2 * i + 1], row[i]);
                     } else if constexpr (BF) {
                         const unsigned short *row = reinterpret_cast<const unsigned short *>(lut) +
-                                                    (mm * a.K + code) * a.NTP + nbase;
+                                                    (mm * a.K + code) * NTP + nbase;
 #pragma unroll
                         for (int i = 0; i < NW; ++i) add_bf16(acc[q][i], row[i]);
                     } else {
-                        const float *row = lut + (mm * a.K + code) * a.NTP + nbase;
+                        const float *row = lut + (mm * a.K + code) * NTP + nbase;
                         accumulate<NW>(acc[q], [&](int i) { return row[i]; });
                     }
                 }
+        };
+        if (a.cbits) {  // packed rows: 4 codes of b bits from one funnel shift
+            const int cbits = a.cbits, bit0 = lane_ct * cbits;
+            const unsigned cmask = (1u << cbits) - 1u;
+#pragma unroll
+            for (int mm = 0; mm < kMchMax; ++mm) {
+                if (mm < mch) {
+                    const unsigned *cw = reinterpret_cast<const unsigned *>(cb + mm * a.crb);
+                    const unsigned v = __funnelshift_r(cw[bit0 >> 5], cw[(bit0 >> 5) + 1], bit0 & 31);
+                    gather_mm(mm, (v & cmask) | (((v >> cbits) & cmask) << 8) |
+                                      (((v >> (2 * cbits)) & cmask) << 16) |
+                                      (((v >> (3 * cbits)) & cmask) << 24));
+                }
             }
+        } else {
+#pragma unroll
+            for (int mm = 0; mm < kMchMax; ++mm)
+                if (mm < mch) gather_mm(mm, *reinterpret_cast<const unsigned *>(cb + mm * a.crb + lane_ct));
         }
     }
 
@@ -583,6 +595,7 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.cch_log2 = 0;
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     a.early = 1;  // no kernel of a library call writes D or the codes
+    a.dvec16 = (s.K * s.Csp) % 4 == 0 && reinterpret_cast<uintptr_t>(D) % 16 == 0;
     a.cl = p.cl;
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
