@@ -29,6 +29,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdlib>
+#include <type_traits>
 
 namespace qcnn {
 
@@ -46,12 +47,12 @@ struct FcArgs {
                  // words >= NT/2; bf16 singles: halves >= NT)
     int NTX;     // odd pitch of a staged x row (>= NT)
     int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
-    int cvec_log2;
     int cbits;   // 0: one byte per code; else bits per code (packed rows)
     int cpitch;  // packed: bytes per code row (multiple of 16)
     int crb;     // bytes per staged code row in shared memory (CT_CTA + 16)
     int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
     int dvec16;    // 1: sub-codebooks staged in 16-byte pieces (K * Csp % 4 == 0, D 16-aligned)
+    int k_log2;    // log2 K when K is a power of two, else -1
     // 1: D and the codes are constants of the caller (no kernel of the same
     // call writes them): the first chunk's are staged before the wait on the
     // previous kernel (programmatic dependent launch), only x after it
@@ -166,23 +167,29 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                              : "memory");
             }
         } else if (a.cvec > 0) {
-            const int row_log2 = kCtCtaLog2 - a.cvec_log2;  // copies per code row
-            const int per_row = 1 << row_log2;
-            for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
-                const int mm = e >> row_log2, q = e & (per_row - 1);
-                const int ct = ct0 + q * a.cvec;
-                const bool ok = mm < mch && ct < a.Ct;  // Ct % cvec == 0: all or nothing
-                const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
-                void *dst = cb + mm * a.crb + q * a.cvec;
-                const unsigned d = smem_addr(dst);
-                const int sz = ok ? a.cvec : 0;
-                if (a.cvec == 16)
-                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
-                else if (a.cvec == 8)
-                    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
-                else
-                    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
-            }
+            // copies of V bytes (the row's alignment), V fixed per loop
+            auto copy_rows = [&](auto vc) {
+                constexpr int V = decltype(vc)::value;
+                constexpr int row_log2 = kCtCtaLog2 - (V == 16 ? 4 : V == 8 ? 3 : 2);
+                constexpr int per_row = 1 << row_log2;  // copies per code row
+                for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
+                    const int mm = e >> row_log2, q = e & (per_row - 1);
+                    const int ct = ct0 + q * V;
+                    const bool ok = mm < mch && ct < a.Ct;  // Ct % V == 0: all or nothing
+                    const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
+                    const unsigned d = smem_addr(cb + mm * a.crb + q * V);
+                    const int sz = ok ? V : 0;
+                    if constexpr (V == 16)
+                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                    else if constexpr (V == 8)
+                        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                    else
+                        asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                }
+            };
+            if (a.cvec == 16) copy_rows(std::integral_constant<int, 16>());
+            else if (a.cvec == 8) copy_rows(std::integral_constant<int, 8>());
+            else copy_rows(std::integral_constant<int, 4>());
         } else {  // rows not 4-byte aligned: plain byte copies
             for (int e = tid; e < a.MCH * CT_CTA; e += kFcThreads) {
                 const int mm = e / CT_CTA, q = e % CT_CTA;
@@ -254,33 +261,28 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 }
             }
             if constexpr (!BF) {
-                // fp32: the chunk's (mm, k, nn) entries with every thread busy --
-                // several sub-spaces side by side when K * NT < the block
-                const int per_mm = a.K * NT;
-                const int lanes_mm = min(per_mm, kFcThreads);
-                const int mm_step = kFcThreads / lanes_mm;
-                const int t_mm = tid / lanes_mm, t_e = tid - t_mm * lanes_mm;
-                if (t_mm < mm_step) {
-                    for (int mm = t_mm; mm < mch; mm += mm_step) {
-                        for (int e = t_e; e < per_mm; e += lanes_mm) {
-                            const int nn = e % NT, k = e / NT;
-                            const float *xp = xb + mm * a.Csp * NTX + nn;
-                            const float *dp = db + (mm * a.K + k) * a.Csp;
-                            float v = 0.f;
-                            if (a.Csp == 4) {  // one 16-byte load of the sub-codeword
-                                const float4 d = *reinterpret_cast<const float4 *>(dp);
-                                v = fmaf(xp[0], d.x, v);
-                                v = fmaf(xp[NTX], d.y, v);
-                                v = fmaf(xp[2 * NTX], d.z, v);
-                                v = fmaf(xp[3 * NTX], d.w, v);
-                            } else {
+                // fp32: the chunk's (mm, k, nn) entries, flat over the block
+                // (several sub-spaces side by side when K * NT < the block);
+                // r = mm * K + k is the table row
+                const int kl = a.k_log2;
+                for (int e = tid; e < mch * a.K * NT; e += kFcThreads) {
+                    const int nn = e % NT, r = e / NT;
+                    const int mm = kl >= 0 ? r >> kl : r / a.K;
+                    const float *xp = xb + mm * a.Csp * NTX + nn;
+                    const float *dp = db + r * a.Csp;
+                    float v = 0.f;
+                    if (a.Csp == 4) {  // one 16-byte load of the sub-codeword
+                        const float4 d = *reinterpret_cast<const float4 *>(dp);
+                        v = fmaf(xp[0], d.x, v);
+                        v = fmaf(xp[NTX], d.y, v);
+                        v = fmaf(xp[2 * NTX], d.z, v);
+                        v = fmaf(xp[3 * NTX], d.w, v);
+                    } else {
 #pragma unroll
-                                for (int j = 0; j < kMaxCsp; ++j)
-                                    if (j < a.Csp) v = fmaf(xp[j * NTX], dp[j], v);
-                            }
-                            lut[(mm * a.K + k) * NTP + nn] = v;
-                        }
+                        for (int j = 0; j < kMaxCsp; ++j)
+                            if (j < a.Csp) v = fmaf(xp[j * NTX], dp[j], v);
                     }
+                    lut[r * NTP + nn] = v;
                 }
             }
         }
@@ -588,7 +590,6 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
              : (s.Ct % 8 == 0 && base % 8 == 0) ? 8
              : (s.Ct % 4 == 0 && base % 4 == 0) ? 4
                                                  : 0;
-    a.cvec_log2 = a.cvec == 16 ? 4 : a.cvec == 8 ? 3 : 2;
     a.cbits = s.code_bits;
     a.cpitch = s.code_bits ? (int)fc_packed_pitch(s.Ct, s.K) : 0;
     a.crb = p.CT_CTA + 16;
@@ -596,6 +597,9 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     a.early = 1;  // no kernel of a library call writes D or the codes
     a.dvec16 = (s.K * s.Csp) % 4 == 0 && reinterpret_cast<uintptr_t>(D) % 16 == 0;
+    a.k_log2 = -1;
+    for (int b = 0; b < 9; ++b)
+        if (s.K == 1 << b) a.k_log2 = b;
     a.cl = p.cl;
     cudaError_t e =
         cudaFuncSetAttribute(fv.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
