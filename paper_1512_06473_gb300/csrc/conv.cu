@@ -84,25 +84,46 @@ qcnn_status launch_pack_codes(const uint8_t *codes, int Ct, int kk, int M, int K
 // entries (one channel, four positions) with 16-byte loads; boundaries that
 // fall between tiles have nothing to do.  Entries on discarded positions were
 // never written and are read but not stored.
+// Stream-K fix-up.  CTA c owns units [u0(c), u1(c)), u = tile * M + m; a
+// tile whose units fall to several CTAs left pieces [CT_CTA][ST] in
+// part[c][1] (the CTA that began the tile and ended inside it: its head) and
+// part[c][0] (every later CTA: a middle or its tail).  Block row b handles
+// the tile cut at the boundary after CTA b when that CTA began the tile, and
+// adds its pieces in CTA order (a fixed order), then bias and ReLU.
+__device__ __forceinline__ long long sk_u0(int c, int base, int extra) {
+    return (long long)c * base + min(c, extra);
+}
+// the CTA whose range holds unit u
+__device__ __forceinline__ int sk_cta_of(long long u, int base, int extra) {
+    const long long big = (long long)extra * (base + 1);  // units of the first extra CTAs
+    return u < big ? (int)(u / (base + 1)) : extra + (int)((u - big) / base);
+}
 __global__ void conv_sk_fixup_kernel(const float *part, int base, int extra, int M,
                                      int pos_tiles, int ct_tiles, int ST, int ct_cta, int Ct,
                                      int pitch, int Ho, int Wo, const float *__restrict__ bias,
                                      int relu, float *__restrict__ y) {
     grid_dep_sync();
     const int b = blockIdx.x;
-    const long long ub = (long long)(b + 1) * base + min(b + 1, extra);
-    if (ub % M == 0) return;
+    const long long ub = sk_u0(b + 1, base, extra);  // first unit after CTA b
+    if (ub % M == 0) return;                          // no tile cut here
+    const long long t = ub / M;
+    if (t * M < sk_u0(b, base, extra)) return;  // CTA b did not begin tile t
+    const int c_last = sk_cta_of(t * M + M - 1, base, extra);
     const size_t piece = (size_t)ct_cta * ST;  // a multiple of 4: ST % 32 == 0
     const size_t o4 = ((size_t)blockIdx.y * blockDim.x + threadIdx.x) * 4;
     if (o4 >= piece) return;
-    const long long t = ub / M;
     const int n = (int)(t / ((long long)ct_tiles * pos_tiles));
     const int rest = (int)(t - (long long)n * ct_tiles * pos_tiles);
     const int ct0 = (rest / pos_tiles) * ct_cta, l0 = (rest % pos_tiles) * ST;
-    const float *p0 = part + (size_t)b * 2 * piece, *p1 = p0 + piece;
-    const float4 a = *reinterpret_cast<const float4 *>(p0 + o4);
-    const float4 c = *reinterpret_cast<const float4 *>(p1 + o4);
-    const float v4[4] = {a.x + c.x, a.y + c.y, a.z + c.z, a.w + c.w};
+    float4 a = *reinterpret_cast<const float4 *>(part + ((size_t)b * 2 + 1) * piece + o4);
+    for (int c = b + 1; c <= c_last; ++c) {
+        const float4 v = *reinterpret_cast<const float4 *>(part + (size_t)c * 2 * piece + o4);
+        a.x += v.x;
+        a.y += v.y;
+        a.z += v.z;
+        a.w += v.w;
+    }
+    const float v4[4] = {a.x, a.y, a.z, a.w};
     const int cl = (int)(o4 / ST), ct = ct0 + cl;
     if (ct >= Ct) return;
     const float bv = bias ? bias[ct] : 0.f;
@@ -314,11 +335,12 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
         // of the plain grid is well short of full.
         const double wave_fill = ctas / (std::ceil(ctas / G) * G);
         if (fv.SK) {
-            // At least as many tiles as CTA slots: every CTA then takes >= M
-            // units, so a tile is cut at most once (two partial pieces).  The
-            // planner's own choice also wants a short last wave on the plain
-            // grid.
-            if (ctas < G) continue;
+            // At least half as many tiles as CTA slots: every CTA then takes
+            // >= M / 2 units, so a tile spreads over at most three CTAs.
+            // (Fewer tiles -- small batches -- are split by sub-space ranges
+            // instead.)  The planner's own choice also wants a short last
+            // wave on the plain grid.
+            if (2 * ctas < G || ctas * s.M < G) continue;  // (and every CTA >= 1 unit)
             if (force < 0 && (!allow_sk || wave_fill >= 0.9)) continue;
             sk_units = std::ceil(ctas * s.M / G);
             const double part = 2.0 * 2.0 * (G - 1) * ct_cta * ST * 4.0;
@@ -340,7 +362,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
                 best.sk_ctas = G;
                 best.sk_base = (int)(units / G);
                 best.sk_extra = (int)(units % G);
-                best.partial_bytes = (size_t)(G - 1) * 2 * ct_cta * ST * sizeof(float);
+                best.partial_bytes = (size_t)G * 2 * ct_cta * ST * sizeof(float);
             }
             best.ok = true;
             best.variant = v;

@@ -24,9 +24,10 @@ struct ConvFusedArgs {
     // stream-K schedule (large batches): CTA c takes the (tile, sub-space)
     // units [u0, u1), u = tile * M + m, sk_base units each plus one for the
     // first sk_extra CTAs; tile = (n * ct_tiles + ct_tile) * pos_tiles + pos.
-    // A tile cut at the end of CTA c's range leaves two partial pieces,
-    // partial[c][0] (sub-spaces before the cut) and partial[c][1] (after),
-    // each [CT_CTA][ST] over the tile's positions
+    // A tile whose units fall to several CTAs leaves one partial piece per
+    // CTA, [CT_CTA][ST] over the tile's positions: partial[c][1] from the
+    // CTA that began it (its head), partial[c][0] from each later one (a
+    // middle part or its tail)
     int sk, sk_base, sk_extra, pos_tiles, ct_tiles;
     // 1: D and the packed codes are the caller's and no kernel of the same
     // call writes them, so the first sub-space's D and codes are staged
@@ -488,12 +489,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
             __syncthreads();
             gather(b, lut0);
             if (last_of_tile || last_of_range) {
-                // whole tile -> y; head of a tile cut at the range end -> piece
-                // 0 of this CTA's boundary; tail of a cut tile -> piece 1 of
-                // the previous CTA's boundary
+                // whole tile -> y; head of a tile cut at the range end ->
+                // piece 1 of this CTA; a middle part or the tail of a tile
+                // begun by an earlier CTA -> piece 0 of this CTA
                 const bool whole = piece_m0 == 0 && last_of_tile;
-                store(whole ? 0 : 2, piece_m0 == 0 ? blockIdx.x : blockIdx.x - 1,
-                      piece_m0 == 0 ? 0 : 1);
+                store(whole ? 0 : 2, blockIdx.x, piece_m0 == 0 ? 1 : 0);
                 if (last_of_range) break;
 #pragma unroll
                 for (int c = 0; c < CTW; ++c)

@@ -414,6 +414,41 @@ def test_conv_stream_k(case):
     assert np.array_equal(goti.astype(np.float64), refi)
 
 
+# Fewer tiles than CTA slots (but at least half as many): a tile's units
+# spread over two or three CTAs, whose pieces (head, middle, tail) the fix-up
+# adds in CTA order.
+# (case, stream-K tile forced: P, CTW, NW, TC)
+STREAM_K_SPREAD = [
+    ((48, 32, 13, 13, 384, 3, 3, 1, 1, 4, 64), (6, 16, 12, 0)),    # 96 tiles, M = 8
+    ((24, 64, 14, 14, 512, 3, 3, 1, 1, 8, 128), (7, 8, 16, 1)),    # 96 tiles, tensor-core build
+    ((40, 8, 13, 13, 256, 3, 3, 1, 1, 4, 32), (6, 8, 16, 0)),      # 80 tiles, M = 2
+]
+
+
+@pytest.mark.parametrize("case,tile", STREAM_K_SPREAD, ids=lambda c: "x".join(map(str, c)))
+def test_conv_stream_k_tiles_over_several_ctas(case, tile):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    v = [i for i, f in enumerate(q.fused_variants())
+         if f["SK"] and not f["BF"] and (f["P"], f["CTW"], f["NW"], f["TC"]) == tile
+         and f["CSP4"] == (8 if Csp > 4 else 4)][0]
+    plan = q.conv_plan(N, Cs, H, W, Ct, kh, kw, s, p, Csp, K, algo=v)
+    Ho, Wo = H + 2 * p - kh + 1, W + 2 * p - kw + 1
+    pitch = max(W + p, Wo)
+    npos = (Ho - 1) * pitch + Wo
+    tiles = N * -(-Ct // plan["channels"]) * -(-npos // plan["positions"])
+    # fewer tiles than CTAs, at least half as many
+    assert plan["stream_k"] == 1 and tiles < plan["ctas"] <= 2 * tiles, (plan, tiles)
+    x, D, codes, b = conv_case(33, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    got = host(q.conv_forward(cuda(x), cuda(D), cuda(codes), kh, kw, s, p, cuda(b), relu=True,
+                              algo=v))
+    assert rel(got, ref) <= TOL
+    xi, Di, ci, bi = conv_case(34, N, Cs, H, W, Ct, kh, kw, Csp, K, integer=True)
+    refi = oracle.conv_forward(xi, Di, ci, kh, kw, s, p, bi)
+    goti = host(q.conv_forward(cuda(xi), cuda(Di), cuda(ci), kh, kw, s, p, cuda(bi), algo=v))
+    assert np.array_equal(goti.astype(np.float64), refi)
+
+
 # Small batches split a tile's sub-spaces over several CTAs; the CTAs of one
 # tile can form a thread-block cluster that adds their partial tiles in
 # distributed shared memory (all of them: no workspace partials and no
