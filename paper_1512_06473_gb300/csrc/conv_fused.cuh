@@ -551,12 +551,13 @@ __global__ void __launch_bounds__(NW * 32, MINB) conv_fused_kernel(const ConvFus
                 if constexpr (BF) build_bf16(b ^ 1, b ? lut0 : lut1);
                 else build(b ^ 1, b ? lut0 : lut1);
             };
-            if (warp & 1) {
-                gather(b, b ? lut1 : lut0);
-                build_next();
-            } else {
-                build_next();
-                gather(b, b ? lut1 : lut0);
+            // (one loop of two steps, so that the gather and the build are
+            // each inlined once: the two orders as straight code doubled the
+            // loop and missed the instruction cache)
+#pragma unroll 1
+            for (int step = 0; step < 2; ++step) {
+                if ((step ^ warp) & 1) gather(b, b ? lut1 : lut0);
+                else build_next();
             }
             cp_async_wait<0>();
             __syncthreads();
