@@ -160,7 +160,7 @@ static const std::vector<FusedVariant> &fused_table() {
     static const std::vector<FusedVariant> table = [] {
         std::vector<FusedVariant> t;
         for (auto part : {fused_variants_plain, fused_variants_bf16, fused_variants_sk,
-                          fused_variants_tc, fused_variants_tc_sk}) {
+                          fused_variants_tc, fused_variants_tc_sk, fused_variants_narrow}) {
             int n = 0;
             const FusedVariant *v = part(&n);
             t.insert(t.end(), v, v + n);

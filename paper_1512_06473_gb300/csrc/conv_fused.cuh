@@ -683,5 +683,6 @@ const FusedVariant *fused_variants_bf16(int *n);   // conv_fused_bf16.cu
 const FusedVariant *fused_variants_sk(int *n);     // conv_fused_sk.cu
 const FusedVariant *fused_variants_tc(int *n);     // conv_fused_tc.cu
 const FusedVariant *fused_variants_tc_sk(int *n);  // conv_fused_tc_sk.cu
+const FusedVariant *fused_variants_narrow(int *n);  // conv_fused_plain.cu (64-channel tiles)
 
 }  // namespace qcnn

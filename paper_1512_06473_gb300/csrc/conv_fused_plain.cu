@@ -13,4 +13,14 @@ const FusedVariant *fused_variants_plain(int *n) {
     return kPart;
 }
 
+// 64-channel tiles (4 channels per warp): layers with Ct <= 64, where the
+// 128-channel tiles gather half their look-ups for channels past Ct
+static const FusedVariant kNarrow[] = {
+    QCNN_FUSED(7, 4, 1, 4, 16, 1, false, 0.9, 1.0), QCNN_FUSED(7, 4, 1, 8, 16, 1, false, 0.9, 1.0)};
+
+const FusedVariant *fused_variants_narrow(int *n) {
+    *n = (int)(sizeof(kNarrow) / sizeof(kNarrow[0]));
+    return kNarrow;
+}
+
 }  // namespace qcnn
