@@ -152,39 +152,52 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         }
         // codes[m0 + mm][ct0 .. ct0 + CT_CTA) -> cs[b][mm][.]; zero outside
         uint8_t *cb = cs + (size_t)b * a.MCH * a.crb;
+        // Each thread copies one column q of the rows mm = mm_first,
+        // mm_first + rows_step, ...: its source and destination advance by a
+        // fixed step (no per-copy index arithmetic)
         if (a.cbits) {  // packed rows: this CTA's slice, whole 16-byte copies
             const int slice = (CT_CTA * a.cbits) >> 3;
-            const int nq = slice >> 4;
-            const size_t off0 = (size_t)blockIdx.x * slice;
-            for (int e = tid; e < a.MCH * nq; e += kFcThreads) {
-                const int mm = e / nq, qq = e - mm * nq;
-                const size_t byte = off0 + (size_t)qq * 16;
-                const bool ok = mm < mch && byte < (size_t)a.cpitch;
-                const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.cpitch + byte : a.codes;
-                const unsigned d = smem_addr(cb + mm * a.crb + qq * 16);
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src),
-                             "r"(ok ? 16 : 0)
-                             : "memory");
+            const int nq = slice >> 4;  // copies per row (<= 64)
+            const int rows_step = kFcThreads / nq;
+            if (tid < rows_step * nq) {
+                const int mm_first = tid / nq, qq = tid - mm_first * nq;
+                const size_t byte = (size_t)blockIdx.x * slice + (size_t)qq * 16;
+                const bool col_ok = byte < (size_t)a.cpitch;
+                const uint8_t *src = a.codes + (size_t)(m0 + mm_first) * a.cpitch + byte;
+                const size_t src_step = (size_t)rows_step * a.cpitch;
+                unsigned d = smem_addr(cb + mm_first * a.crb + qq * 16);
+                const unsigned d_step = (unsigned)(rows_step * a.crb);
+                for (int mm = mm_first; mm < a.MCH; mm += rows_step, src += src_step, d += d_step) {
+                    const bool ok = col_ok && mm < mch;
+                    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d),
+                                 "l"(ok ? src : a.codes), "r"(ok ? 16 : 0)
+                                 : "memory");
+                }
             }
         } else if (a.cvec > 0) {
             // copies of V bytes (the row's alignment), V fixed per loop
             auto copy_rows = [&](auto vc) {
                 constexpr int V = decltype(vc)::value;
                 constexpr int row_log2 = kCtCtaLog2 - (V == 16 ? 4 : V == 8 ? 3 : 2);
-                constexpr int per_row = 1 << row_log2;  // copies per code row
-                for (int e = tid; e < a.MCH * per_row; e += kFcThreads) {
-                    const int mm = e >> row_log2, q = e & (per_row - 1);
-                    const int ct = ct0 + q * V;
-                    const bool ok = mm < mch && ct < a.Ct;  // Ct % V == 0: all or nothing
-                    const uint8_t *src = ok ? a.codes + (size_t)(m0 + mm) * a.Ct + ct : a.codes;
-                    const unsigned d = smem_addr(cb + mm * a.crb + q * V);
+                constexpr int per_row = 1 << row_log2;  // copies per code row (<= 256)
+                constexpr int rows_step = kFcThreads / per_row;
+                const int mm_first = tid >> row_log2, q = tid & (per_row - 1);
+                const int ct = ct0 + q * V;
+                const bool col_ok = ct < a.Ct;  // Ct % V == 0: all or nothing
+                const uint8_t *src = a.codes + (size_t)(m0 + mm_first) * a.Ct + ct;
+                const size_t src_step = (size_t)rows_step * a.Ct;
+                unsigned d = smem_addr(cb + mm_first * a.crb + q * V);
+                const unsigned d_step = (unsigned)(rows_step * a.crb);
+                for (int mm = mm_first; mm < a.MCH; mm += rows_step, src += src_step, d += d_step) {
+                    const bool ok = col_ok && mm < mch;
+                    const uint8_t *s = ok ? src : a.codes;
                     const int sz = ok ? V : 0;
                     if constexpr (V == 16)
-                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(s), "r"(sz) : "memory");
                     else if constexpr (V == 8)
-                        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(s), "r"(sz) : "memory");
                     else
-                        asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(sz) : "memory");
+                        asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(s), "r"(sz) : "memory");
                 }
             };
             if (a.cvec == 16) copy_rows(std::integral_constant<int, 16>());
