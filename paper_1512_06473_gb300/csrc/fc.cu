@@ -43,9 +43,6 @@ struct FcArgs {
     int N, Cs, Ct, Csp, K, M;
     int NT, CT_CTA, MCH, n_chunks, chunks_per_split, splits, relu;
     int cl;  // the splits of a tile form clusters of cl CTAs (1: none)
-    int NTP;     // odd pitch of a table row (fp32: floats >= NT; bf16 pairs:
-                 // words >= NT/2; bf16 singles: halves >= NT)
-    int NTX;     // odd pitch of a staged x row (>= NT)
     int cvec;    // bytes per code copy: 16, 8 or 4 (0: byte copies)
     int cbits;   // 0: one byte per code; else bits per code (packed rows)
     int cpitch;  // packed: bytes per code row (multiple of 16)
@@ -101,8 +98,9 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
     constexpr int NT = NW * WN;  // images per CTA (== a.NT)
     constexpr bool PAIRS = BF && NW % 2 == 0;  // bf16 words of two images
     static_assert(!BF || NW % 2 == 0 || NW == 1, "bf16 tiles: even NW or NW == 1");
-    // row pitches of the table and of the staged x (the host passes the same
-    // values in NTP, NTX): compile-time, so row addresses fold
+    // odd row pitches (compile-time, so row addresses fold): the table's
+    // (fp32: floats >= NT; bf16 pairs: words >= NT/2; bf16 singles: halves
+    // >= NT) and the staged x's (>= NT)
     constexpr int NTP = (BF && NT % 2 == 0 ? NT / 2 : NT) | 1;
     constexpr int NTX = NT | 1;
     extern __shared__ __align__(16) unsigned char smem[];
@@ -597,8 +595,6 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.chunks_per_split = p.chunks_per_split;
     a.splits = p.splits;
     a.relu = relu;
-    a.NTP = fc_ntp(p.NT, fv.BF);
-    a.NTX = p.NT | 1;
     const uintptr_t base = reinterpret_cast<uintptr_t>(codes);
     a.cvec = (s.Ct % 16 == 0 && base % 16 == 0) ? 16
              : (s.Ct % 8 == 0 && base % 8 == 0) ? 8
