@@ -522,11 +522,28 @@ def measure_configs(q, torch, cm, dev, flush, stream, smem_gbs, hbm_gbs, reps):
                         "frac_smem": round(alg * B / (ms_b / 1e3) / (smem_gbs * 1e9), 4),
                         "stages": stage_rooflines(wk, cm, stage_ms, B, smem_gbs, hbm_gbs)})
         cfgs[name] = per
+    # the floor of this timing for a single library call: one launch of the
+    # smallest library kernel (a 3x3 max-pool of one 3x3 map), timed the same way
+    tiny = torch.zeros((1, 1, 3, 3), dtype=torch.float32, device=dev)
+    tout = torch.empty((1, 1, 1, 1), dtype=torch.float32, device=dev)
+    for _ in range(3):
+        q.maxpool(tiny, 3, 2, out=tout)
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        q.maxpool(tiny, 3, 2, out=tout)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ts.append(e0.elapsed_time(e1))
     return {"note": "each workload's whole stack through qcnn_net_forward, device-resident "
                     "input, L2 flushed before every forward; frac_smem = 4 B x (look-ups + "
                     "table entries) per second over the measured shared-memory peak; stages: "
                     "per layer, launched one by one, the fraction of the slower of its "
-                    "shared-memory roof and its HBM roof (stage_rooflines)",
+                    "shared-memory roof and its HBM roof (stage_rooflines); launch_floor_ms: "
+                    "one call of the smallest library kernel, timed the same way",
+            "launch_floor_ms": round(float(np.median(ts)), 4),
             "workloads": cfgs}
 
 
