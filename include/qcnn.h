@@ -37,6 +37,10 @@
  *  - Codes >= K are a caller error.  Kernels clamp every index into [0, K),
  *    so such codes never cause an out-of-bounds access, but the outputs are
  *    then unspecified.
+ *  - Inputs (x, D, codes, bias) must not overlap the outputs or the
+ *    workspace, and must not change while the call runs: inside one call the
+ *    kernels after the first may read D and the codes before the kernel
+ *    before them has finished (programmatic dependent launch).
  *  - A failed launch returns QCNN_ERR_CUDA; the CUDA error is in
  *    qcnn_last_cuda_error().  The library is stateless apart from that
  *    value, a launch counter, a cache of qcnn_net_* plans (keyed by device,
