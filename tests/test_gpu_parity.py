@@ -540,6 +540,38 @@ FORCED = [
 ]
 
 
+# Ragged channel and position tiles for the narrow (64-channel) and the
+# 12-warp tiles: every forced fp32 variant that can serve the shape, against
+# the oracle, on real-valued data (tolerance) -- a channel count that is not a
+# multiple of any tile and a map whose positions end mid-slot.
+RAGGED = [
+    (3, 24, 19, 23, 40, 3, 3, 1, 1, 4, 64),    # Ct = 40 < one 64-channel tile
+    (2, 16, 31, 29, 100, 3, 3, 1, 1, 8, 32),   # Ct = 100: two 64-channel tiles, C'_s = 8
+]
+
+
+@pytest.mark.parametrize("case", RAGGED, ids=lambda c: "x".join(map(str, c)))
+def test_fused_variants_ragged_tiles(case):
+    N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
+    x, D, codes, b = conv_case(35, N, Cs, H, W, Ct, kh, kw, Csp, K)
+    ref = oracle.conv_forward(x, D, codes, kh, kw, s, p, b, relu=True)
+    xd, Dd, cd, bd = cuda(x), cuda(D), cuda(codes), cuda(b)
+    ran = 0
+    narrow = 0
+    for v, info in enumerate(q.fused_variants()):
+        if info["BF"]:
+            continue
+        try:
+            got = q.conv_forward(xd, Dd, cd, kh, kw, s, p, bd, relu=True, algo=v)
+        except q.QcnnError as e:
+            assert e.status == 2, (v, info)
+            continue
+        assert rel(host(got), ref) <= TOL, (v, info)
+        ran += 1
+        narrow += info["CTW"] * info["NW"] // info["WP"] == 64
+    assert ran >= 10 and narrow >= 1, (ran, narrow)
+
+
 @pytest.mark.parametrize("case", FORCED, ids=lambda c: "x".join(map(str, c)))
 def test_every_fused_variant_is_exact(case):
     N, Cs, H, W, Ct, kh, kw, s, p, Csp, K = case
