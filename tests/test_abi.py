@@ -371,6 +371,39 @@ def test_batch1_plans_split_the_subspaces():
 
 
 @_planner
+def test_fc_16_image_tiles_take_two_chunks():
+    """16-image FC tiles give every CTA at least two chunks of 16 sub-spaces
+    (one chunk per CTA measured slower at batches 64-128)."""
+    import paper_1512_06473_gb300 as q
+    seen = 0
+    for N in (64, 128, 256):
+        for Cs, Ct in ALEX_FC.values():
+            f = q.fc_plan(N, Cs, Ct)
+            if f["images"] == 16:
+                seen += 1
+                n_chunks = -(-(Cs // 4) // f["chunk"])
+                assert f["splits"] <= n_chunks // 2, (N, Cs, Ct, f)
+    assert seen >= 6
+
+
+@_planner
+def test_stream_k_needs_half_as_many_tiles_as_slots():
+    """A stream-K tile is taken with at least half as many tiles as CTA
+    slots (tiles then spread over at most three CTAs); with fewer it is
+    refused (the split sub-space plans serve small batches)."""
+    import paper_1512_06473_gb300 as q
+    V = q.fused_variants()
+    v = [i for i, f in enumerate(V) if f["SK"] and not f["BF"] and not f["TC"]
+         and (f["P"], f["CTW"], f["NW"], f["CSP4"]) == (6, 8, 16, 4)][0]
+    # 13x13 maps: one 192-position tile per image, 2 tiles of 128 channels
+    p = q.conv_plan(40, 8, 13, 13, 256, 3, 3, 1, 1, 4, 32, algo=v)   # 80 tiles
+    assert p["stream_k"] == 1 and p["ctas"] == 152, p
+    with pytest.raises(q.QcnnError) as e:
+        q.conv_plan(30, 8, 13, 13, 256, 3, 3, 1, 1, 4, 32, algo=v)   # 60 tiles
+    assert e.value.status == _lib.ERR_UNSUPPORTED
+
+
+@_planner
 def test_fc_clusters_only_with_many_splits():
     """The FC planner groups split CTAs into clusters only from 64 splits
     up (fewer splits measured slower with clusters), and then into clusters
