@@ -19,11 +19,13 @@
 // Codes can also come bit-packed (b = ceil(log2 K) bits each, every [M][Ct]
 // row padded to a 16-byte pitch): a CTA's slice of a row is then b * CT_CTA
 // / 8 bytes, staged with 16-byte copies, and a lane takes its 4 codes from one
-// funnel shift of two 32-bit words -- 8/b times fewer code bytes from HBM,
-// which is what bounds the layer at batch 1.
+// funnel shift of two 32-bit words -- 8/b times fewer code bytes from HBM.
 // When the sub-space range is split over several CTAs (to fill the GPU),
 // the partial sums go to the workspace and a second kernel adds them in a
-// fixed order (deterministic), then applies bias and ReLU.
+// fixed order (deterministic), then applies bias and ReLU.  With many splits
+// of small image tiles, clusters of CTAs first add their partial tiles in
+// distributed shared memory (rank order), so fewer partial sums per output
+// reach the workspace.
 #include "qcnn_internal.cuh"
 
 #include <algorithm>
