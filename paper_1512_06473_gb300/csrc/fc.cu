@@ -51,6 +51,13 @@ struct FcArgs {
     int crb;     // bytes per staged code row in shared memory (CT_CTA + 16)
     int cch_log2;  // log2 of MCH * Csp rounded up to a power of two
     int dvec16;    // 1: sub-codebooks staged in 16-byte pieces (K * Csp % 4 == 0, D 16-aligned)
+    // xgroups > 0: the input is the previous FC layer's output still as
+    // partial sums, x[n][c] = act(xbias[c] + sum_g xpart[g][n][c]) (act: ReLU
+    // when xrelu), added in g order while staging -- that layer's reduction
+    // kernel is not run.  (Written by the kernel before: coherent loads.)
+    const float *xpart;
+    const float *xbias;
+    int xgroups, xrelu;
     int k_log2;    // log2 K when K is a power of two, else -1
     // 1: D and the codes are constants of the caller (no kernel of the same
     // call writes them): the first chunk's are staged before the wait on the
@@ -131,6 +138,23 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
         float *xb = xs + (size_t)b * CCH * NTX;
         // (image nn, float cc) with cc on a power-of-two stride: no division
         const int cmask = (1 << a.cch_log2) - 1;
+        if (a.xgroups > 0) {  // sums of the previous layer's partials, in group order
+            const size_t plane = (size_t)a.N * a.Cs;
+            for (int e = tid; e < (NT << a.cch_log2); e += kFcThreads) {
+                const int cc = e & cmask, nn = e >> a.cch_log2;
+                if (cc >= CCH) continue;
+                float v = 0.f;
+                if (cc < mch * a.Csp && n0 + nn < a.N) {
+                    const size_t c = (size_t)m0 * a.Csp + cc;
+                    const float *src = a.xpart + (size_t)(n0 + nn) * a.Cs + c;
+                    for (int g = 0; g < a.xgroups; ++g) v += src[g * plane];
+                    if (a.xbias) v += a.xbias[c];
+                    if (a.xrelu) v = fmaxf(v, 0.f);
+                }
+                xb[cc * NTX + nn] = v;
+            }
+            return;
+        }
         for (int e = tid; e < (NT << a.cch_log2); e += kFcThreads) {
             const int cc = e & cmask, nn = e >> a.cch_log2;
             if (cc >= CCH) continue;
@@ -575,7 +599,8 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
 
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const float *D,
                       const uint8_t *codes, const float *bias, float *y, int relu,
-                      float *partial_ws, cudaStream_t st) {
+                      float *partial_ws, cudaStream_t st, const FcPartialInput *xin,
+                      bool leave_partials) {
     const FcVariant &fv = kFcVariants[p.variant];
     FcArgs a;
     a.x = x;
@@ -608,6 +633,10 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     a.cch_log2 = 0;
     while ((1 << a.cch_log2) < p.MCH * s.Csp) ++a.cch_log2;
     a.early = 1;  // no kernel of a library call writes D or the codes
+    a.xpart = xin ? xin->part : nullptr;
+    a.xbias = xin ? xin->bias : nullptr;
+    a.xgroups = xin ? xin->groups : 0;
+    a.xrelu = xin ? xin->relu : 0;
     a.dvec16 = (s.K * s.Csp) % 4 == 0 && reinterpret_cast<uintptr_t>(D) % 16 == 0;
     a.k_log2 = -1;
     for (int b = 0; b < 9; ++b)
@@ -622,7 +651,7 @@ qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const f
     const dim3 cluster = p.cl > 1 ? dim3(1, 1, p.cl) : dim3(0, 0, 0);
     qcnn_status rc = launch_k(fv.fn, grid, dim3(kFcThreads), p.smem, st, cluster, a);
     const int groups = p.splits / p.cl;  // partial sums per output left
-    if (rc != QCNN_OK || groups == 1) return rc;
+    if (rc != QCNN_OK || groups == 1 || leave_partials) return rc;
     const size_t total = (size_t)s.N * s.Ct;
     const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)num_sms() * 8);
     if (total < 65536 && groups >= 16) {

@@ -342,6 +342,10 @@ bool ws_ok(const void *ws, size_t have, size_t need) {
 }
 
 // -------------------------------------------------------------- net plan ---
+// FC layers hand their partial sums to the next FC layer up to this batch
+// (above it the next layer's staging would re-read many partials per input)
+constexpr int kChainMaxBatch = 8;
+
 struct NetStep {
     int kind;
     int N;              // batch this step is planned for
@@ -351,6 +355,10 @@ struct NetStep {
     int C, H, W;        // input of this layer (per image)
     int oC, oH, oW;     // output
     size_t scratch;     // bytes of layer scratch
+    // small batches, FC followed by FC: this layer leaves its partial sums
+    // (chain region part_region, 1 or 2) instead of reducing them, and the
+    // next layer adds them while staging its input (x_from_prev)
+    int leave_partials = 0, part_region = 0, x_from_prev = 0;
 };
 
 struct NetPlan {
@@ -364,6 +372,7 @@ struct NetPlan {
     size_t act_floats;  // floats of one ping-pong activation buffer
     size_t scratch;     // max layer scratch
     size_t act_off[2], scratch_off, xin_off, yout_off, total;
+    size_t chain_bytes = 0, chain_off[2] = {0, 0};  // partial sums handed between FC layers
 };
 
 qcnn_status plan_step(const qcnn_layer &L, int N, int c, int h, int w, NetStep *out) {
@@ -433,6 +442,20 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
         w = st.oW;
         np->steps.push_back(st);
     }
+    // FC -> FC at small batches: the first layer's partial sums go straight to
+    // the second layer's staging (no reduction kernel between them); the
+    // regions alternate so that a layer never overwrites the partials it reads
+    np->chain_bytes = 0;
+    for (int i = 0, r = 0; i + 1 < n_layers; ++i) {
+        NetStep &a = np->steps[i], &b = np->steps[i + 1];
+        if (a.kind == QCNN_LAYER_FC && b.kind == QCNN_LAYER_FC && N <= kChainMaxBatch &&
+            a.fcp.splits / a.fcp.cl > 1) {
+            a.leave_partials = 1;
+            a.part_region = 1 + (r++ & 1);
+            b.x_from_prev = 1;
+            np->chain_bytes = std::max(np->chain_bytes, a.fcp.partial_bytes);
+        }
+    }
     np->chunks = 1;
     if (host_io) {
         const int ch = (N % 4 == 0 && N / 4 >= 8) ? 4 : (N % 2 == 0 && N / 2 >= 8) ? 2 : 1;
@@ -448,6 +471,10 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
     }
     np->scratch_off = off;
     off += align_up(np->scratch, kWsAlign);
+    for (int r = 0; r < 2; ++r) {
+        np->chain_off[r] = off;
+        off += align_up(np->chain_bytes, kWsAlign);
+    }
     np->xin_off = np->yout_off = off;
     if (host_io) {
         np->xin_off = off;
@@ -520,13 +547,13 @@ qcnn_status plan_net_cached(const qcnn_layer *layers, int n_layers, int N, int C
 }
 
 qcnn_status run_step(const qcnn_layer &L, const NetStep &s, const float *in, float *out,
-                     void *scratch, cudaStream_t st) {
+                     void *scratch, cudaStream_t st, const FcPartialInput *xin = nullptr) {
     if (s.kind == QCNN_LAYER_CONV)
         return run_conv(s.conv, in, L.D, L.codes, L.codes_layout, L.bias, out, L.relu, scratch,
                         st);
     if (s.kind == QCNN_LAYER_FC)
         return launch_fc(s.fc, s.fcp, in, L.D, L.codes, L.bias, out, L.relu,
-                         reinterpret_cast<float *>(scratch), st);
+                         reinterpret_cast<float *>(scratch), st, xin, s.leave_partials != 0);
     return launch_maxpool(in, s.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
 }
 
@@ -536,8 +563,17 @@ qcnn_status run_net(const qcnn_layer *layers, const NetPlan &np, const float *in
     uint8_t *base = static_cast<uint8_t *>(ws);
     const int n = (int)np.steps.size();
     for (int i = first; i < n; ++i) {
+        const NetStep &s = np.steps[i];
         float *out = (i + 1 == n) ? y : reinterpret_cast<float *>(base + np.act_off[i & 1]);
-        qcnn_status rc = run_step(layers[i], np.steps[i], in, out, base + np.scratch_off, st);
+        uint8_t *scratch =
+            s.part_region ? base + np.chain_off[s.part_region - 1] : base + np.scratch_off;
+        FcPartialInput xin{};
+        if (s.x_from_prev) {  // (the previous step is an FC layer that left its partials)
+            const NetStep &p = np.steps[i - 1];
+            xin = {reinterpret_cast<const float *>(base + np.chain_off[p.part_region - 1]),
+                   p.fcp.splits / p.fcp.cl, layers[i - 1].bias, layers[i - 1].relu};
+        }
+        qcnn_status rc = run_step(layers[i], s, in, out, scratch, st, s.x_from_prev ? &xin : nullptr);
         if (rc != QCNN_OK) return rc;
         in = out;
     }

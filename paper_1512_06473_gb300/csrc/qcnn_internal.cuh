@@ -238,9 +238,22 @@ qcnn_status fc_forward_limited(const float *x, int N, int Cs, int Ct, const floa
                                int K, const uint8_t *codes, const float *bias, float *y,
                                int relu, size_t max_partial_bytes,
                                qcnn_status (*get_scratch)(void **), cudaStream_t st);
+// The input of an FC layer as the previous FC layer's partial sums
+// [groups][N][Cs] (that layer launched with leave_partials), its bias and
+// ReLU applied while staging.
+struct FcPartialInput {
+    const float *part;
+    int groups;
+    const float *bias;
+    int relu;
+};
+// xin: the input comes as partial sums (x is then unused); leave_partials:
+// a plan with several partial sums per output leaves them in partial_ws
+// (for the next FC layer) instead of reducing them into y
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x,
                       const float *D, const uint8_t *codes, const float *bias,
-                      float *y, int relu, float *partial_ws, cudaStream_t st);
+                      float *y, int relu, float *partial_ws, cudaStream_t st,
+                      const FcPartialInput *xin = nullptr, bool leave_partials = false);
 
 // ------------------------------------------------------------ lut, pool ----
 // lut: fp32 entries, or bfloat16 bit patterns when bf16 != 0
