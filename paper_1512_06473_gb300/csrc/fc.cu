@@ -302,8 +302,18 @@ __global__ void __launch_bounds__(kFcThreads, MINB) fc_fused_kernel(const FcArgs
                 // (several sub-spaces side by side when K * NT < the block);
                 // r = mm * K + k is the table row
                 const int kl = a.k_log2;
+                // 16-image tiles: a warp's 32 entries are 16 images of two rows;
+                // rows r and r + 16 (odd pitch 17: bank offsets 16 apart) instead
+                // of r and r + 1 (whose banks overlap in one) keep its stores
+                // conflict free, when the rows come in whole groups of 32
+                const bool rows16 = NT == 16 && ((mch * a.K) & 31) == 0;
                 for (int e = tid; e < mch * a.K * NT; e += kFcThreads) {
-                    const int nn = e % NT, r = e / NT;
+                    const int nn = e % NT;
+                    int r = e / NT;
+                    if (rows16) {
+                        const int q = e >> 5;
+                        r = ((q >> 4) << 5) + (q & 15) + (((e >> 4) & 1) << 4);
+                    }
                     const int mm = kl >= 0 ? r >> kl : r / a.K;
                     const float *xp = xb + mm * a.Csp * NTX + nn;
                     const float *dp = db + r * a.Csp;
