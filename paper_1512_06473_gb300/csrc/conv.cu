@@ -272,8 +272,17 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
         // over the variant's measured efficiency, plus the exposed part of the
         // table build (about 4 wavefronts of time per 32 entries:
         // latency-bound FMA chains)
-        const double per_m = (double)slots * ct_cta * kk / fv.eff +
-                             (double)HP * s.K * 4.0 / 32.0 * fv.build;
+        const double gather_m = (double)slots * ct_cta * kk / fv.eff;
+        const double build_m = (double)HP * s.K * 4.0 / 32.0;
+        const double per_m = gather_m + build_m * fv.build;
+        // a CTA with mps sub-spaces: the first table build is never hidden,
+        // the later ones at the variant's exposure (two-buffer tiles: a short
+        // run of sub-spaces hides little -- measured at batch 1, AlexNet conv3
+        // and conv5: 27.3 us with the 128-position two-buffer tile against
+        // 25.2 us with the 192-position one-buffer tile)
+        auto cta_work = [&](int mps) {
+            return gather_m * mps + build_m * (1.0 + fv.build * (mps - 1));
+        };
         // Small batches: split the sub-spaces of each tile over `splits` CTAs
         // (partial sums through the workspace, then a reduction) when the
         // grid would leave SMs idle.
@@ -308,8 +317,8 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
                 const double part =
                     groups > 1 ? 2.0 * groups * s.N * s.Ct * s.Ho * s.Wo * 4.0 : 0.0;
                 const double red = c > 1 ? ((double)ct_cta * ST / 8.0 + 1500.0) * cps : 0.0;
-                const double sc = waves * per_m * mps * cps + part / 3000.0 +
-                                  (groups > 1 ? 6000.0 : 0.0) + red;
+                const double sc = waves * cta_work(mps) * cps + part / 3000.0 +
+                                  (groups > 1 ? 3000.0 : 0.0) + red;
                 if ((sp == 1 && c == 1) || sc < score) {
                     score = sc;
                     splits = sp_eff;
