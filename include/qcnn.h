@@ -371,7 +371,16 @@ qcnn_status qcnn_maxpool(const float *x, int N, int C, int H, int W, int k,
  * Whole network: a stack of PQ conv / PQ FC / max-pool layers (Sec. 4.2.3,
  * Table 8).  An FC layer that follows a conv or pool layer reads its input
  * flattened in C*H*W order.  The input channel count of each layer is the
- * output channel count of the layer before it.
+ * output channel count of the layer before it.  Each layer runs the plan of
+ * its single-layer call (qcnn_conv_forward with the layer's algo,
+ * qcnn_fc_forward, qcnn_maxpool), with one launch fewer where a layer's
+ * split partial sums go straight to the next layer instead of a reduction:
+ *   - a conv layer to the max-pool after it (planes of at most 12288
+ *     elements): the pool adds them in split order, then the bias and ReLU,
+ *     as the reduction does, so the output is bit-identical;
+ *   - an FC layer to the FC layer after it (batches of at most 8): the next
+ *     layer adds them in split order while staging its input, which may
+ *     round differently from the single call's reduction.
  */
 typedef enum { QCNN_LAYER_CONV = 0, QCNN_LAYER_FC = 1, QCNN_LAYER_MAXPOOL = 2 } qcnn_layer_kind;
 
@@ -382,7 +391,7 @@ typedef struct {
     int stride, pad;    /* CONV: stride, zero padding; MAXPOOL: stride       */
     int Csp, K;         /* CONV / FC: sub-space dimension, sub-codewords     */
     int relu;           /* CONV / FC: 1 = ReLU after the bias                */
-    int algo;           /* CONV: qcnn_algo                                   */
+    int algo;           /* CONV: qcnn_algo, optionally | QCNN_ALGO_NO_CLUSTER */
     int codes_layout;   /* CONV: qcnn_codes_layout of `codes`; FC: CANONICAL
                            ([M][Ct] bytes) or PACKED (qcnn_fc_pack_codes)   */
     int lut_type;       /* CONV / FC: qcnn_lut_type of the table entries     */

@@ -423,6 +423,7 @@ class ConvLayer:
     algo: str = "auto"
     packed: bool = False
     lut: str = "fp32"
+    cluster: bool = True        # False: QCNN_ALGO_NO_CLUSTER (as conv_forward's cluster)
 
 
 @dataclass
@@ -455,6 +456,8 @@ class Net:
                 M, K, Csp = L.D.shape
                 d.kind, d.Ct, d.kh, d.kw, d.stride, d.pad = _lib.LAYER_CONV, L.Ct, L.kh, L.kw, L.stride, L.pad
                 d.Csp, d.K, d.relu, d.algo = Csp, K, int(L.relu), _lib.ALGO[L.algo]
+                if not L.cluster:
+                    d.algo |= _lib.ALGO_NO_CLUSTER
                 d.codes_layout = _lib.CODES_PACKED if L.packed else _lib.CODES_CANONICAL
                 d.lut_type = _lib.LUT[L.lut]
                 d.D, d.codes, d.bias = _ptr(L.D), _ptr(L.codes), _ptr(L.bias)

@@ -405,7 +405,7 @@ ConvFusedPlan plan_conv_fused(const ConvShape &s, int force, int force_cl) {
 qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias,
                               float *y, int relu, float *partial_ws, cudaStream_t st,
-                              bool early) {
+                              bool early, bool leave_partials) {
     const FusedVariant &fv = fused_table()[p.variant];
     ConvFusedArgs a;
     a.x = x;
@@ -460,7 +460,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p, const 
                           p.pos_tiles, p.ct_tiles, p.ST, p.ct_cta, s.Ct, p.pitch, s.Ho, s.Wo,
                           bias, relu, y);
     }
-    if (p.splits / p.cl == 1) return rc;
+    if (p.splits / p.cl == 1 || leave_partials) return rc;
     return launch_split_reduce(partial_ws, p.splits / p.cl, (size_t)s.N * s.Ct * s.Ho * s.Wo,
                                s.Ct, s.Ho * s.Wo, bias, relu, y, st);
 }

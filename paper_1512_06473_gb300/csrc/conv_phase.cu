@@ -422,7 +422,8 @@ ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl) {
 
 qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias, float *y,
-                              int relu, float *partial_ws, cudaStream_t st, bool early) {
+                              int relu, float *partial_ws, cudaStream_t st, bool early,
+                              bool leave_partials) {
     const PhaseVariant &pv = kPhase[p.variant];
     PhaseArgs a;
     a.x = x;
@@ -467,7 +468,7 @@ qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const 
     const dim3 grid(p.pos_tiles, p.ct_tiles, s.N * p.splits);
     const dim3 cluster = p.cl > 1 ? dim3(1, 1, p.cl) : dim3(0, 0, 0);
     qcnn_status rc = launch_k(pv.fn, grid, dim3(pv.NW * 32), p.smem, st, cluster, a);
-    if (rc != QCNN_OK || p.splits / p.cl == 1) return rc;
+    if (rc != QCNN_OK || p.splits / p.cl == 1 || leave_partials) return rc;
     return launch_split_reduce(partial_ws, p.splits / p.cl, (size_t)s.N * s.Ct * s.Ho * s.Wo, s.Ct,
                                s.Ho * s.Wo, bias, relu, y, st);
 }

@@ -609,7 +609,7 @@ FcPlan plan_fc(const FcShape &s, size_t max_partial_bytes) {
 
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x, const float *D,
                       const uint8_t *codes, const float *bias, float *y, int relu,
-                      float *partial_ws, cudaStream_t st, const FcPartialInput *xin,
+                      float *partial_ws, cudaStream_t st, const PartialInput *xin,
                       bool leave_partials) {
     const FcVariant &fv = kFcVariants[p.variant];
     FcArgs a;

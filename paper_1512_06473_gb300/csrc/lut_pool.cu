@@ -91,4 +91,48 @@ qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k, in
                       y);
 }
 
+// The same max-pool of a conv layer's output that is still in its split
+// partial sums [groups][N][C][H][W] (Eq. 7 summed over sub-space ranges): one
+// CTA per (n, c) plane first forms each element once -- the groups added in
+// order from zero, then the bias, then ReLU, the arithmetic of
+// conv_split_reduce_kernel, so the result is bit-identical to reducing and
+// pooling in two launches -- into shared memory, where the windows read it.
+__global__ void maxpool_partial_kernel(const float *part, int groups, size_t total, int C, int H,
+                                       int W, int k, int s, int Ho, int Wo,
+                                       const float *__restrict__ bias, int relu,
+                                       float *__restrict__ y) {
+    extern __shared__ float plane[];
+    grid_dep_sync();
+    const int HW = H * W;
+    const size_t nc = blockIdx.x;
+    const float *p = part + nc * HW;
+    for (int e = threadIdx.x; e < HW; e += blockDim.x) {
+        float v = 0.f;
+#pragma unroll 16
+        for (int g = 0; g < groups; ++g) v += p[(size_t)g * total + e];
+        if (bias) v += bias[nc % C];
+        if (relu) v = fmaxf(v, 0.f);
+        plane[e] = v;
+    }
+    __syncthreads();
+    for (int o = threadIdx.x; o < Ho * Wo; o += blockDim.x) {
+        const int oy = o / Wo, ox = o - oy * Wo;
+        const float *q = plane + oy * s * W + ox * s;
+        float v = q[0];
+        for (int dy = 0; dy < k; ++dy)
+            for (int dx = 0; dx < k; ++dx) v = fmaxf(v, q[dy * W + dx]);
+        y[nc * Ho * Wo + o] = v;
+    }
+}
+
+qcnn_status launch_maxpool_partial(const PartialInput &in, int N, int C, int H, int W, int k,
+                                   int s, float *y, cudaStream_t st) {
+    if ((size_t)H * W > kPoolPlaneMax || in.groups < 1) return QCNN_ERR_UNSUPPORTED;
+    const int Ho = (H - k) / s + 1, Wo = (W - k) / s + 1;
+    const size_t total = (size_t)N * C * H * W;
+    return launch_pdl(maxpool_partial_kernel, dim3((unsigned)(N * C)), dim3(256),
+                      (size_t)H * W * sizeof(float), st, in.part, in.groups, total, C, H, W, k, s,
+                      Ho, Wo, in.bias, in.relu, y);
+}
+
 }  // namespace qcnn

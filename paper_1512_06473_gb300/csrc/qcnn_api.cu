@@ -311,9 +311,20 @@ qcnn_status plan_conv_call_cached(const ConvShape &s, int codes_layout, int algo
     return QCNN_OK;
 }
 
+// Partial sums per output a conv call leaves for a reduction (fused and
+// stride-phase plans whose split sub-spaces are not all in one cluster), in
+// its workspace at lut_off; 1 when the call writes y itself.
+int conv_groups(const ConvCall &c) {
+    if (c.algo == QCNN_ALGO_FUSED && !c.fp.sk) return c.fp.splits / c.fp.cl;
+    if (c.algo == QCNN_ALGO_PHASE) return c.pp.splits / c.pp.cl;
+    return 1;
+}
+
+// leave_partials: a call with conv_groups(c) > 1 leaves its partial sums in
+// the workspace instead of reducing them into y (the net's conv -> max-pool)
 qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const uint8_t *codes,
                      int codes_layout, const float *bias, float *y, int relu, void *ws,
-                     cudaStream_t st) {
+                     cudaStream_t st, bool leave_partials = false) {
     if (c.algo == QCNN_ALGO_CHUNKED)
         return launch_conv_chunked(c.s, c.cp, x, D, codes, codes_layout == QCNN_CODES_PACKED, bias,
                                    y, relu, static_cast<uint8_t *>(ws) + c.lut_off, st);
@@ -330,9 +341,11 @@ qcnn_status run_conv(const ConvCall &c, const float *x, const float *D, const ui
     }
     float *lut = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + c.lut_off);
     if (c.algo == QCNN_ALGO_FUSED)
-        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, lut, st, early);
+        return launch_conv_fused(c.s, c.fp, x, D, packed, bias, y, relu, lut, st, early,
+                                 leave_partials);
     if (c.algo == QCNN_ALGO_PHASE)
-        return launch_conv_phase(c.s, c.pp, x, D, packed, bias, y, relu, lut, st, early);
+        return launch_conv_phase(c.s, c.pp, x, D, packed, bias, y, relu, lut, st, early,
+                                 leave_partials);
     return launch_conv_unfused(c.s, c.up, x, D, packed, bias, y, relu, lut, st);
 }
 
@@ -357,7 +370,9 @@ struct NetStep {
     size_t scratch;     // bytes of layer scratch
     // small batches, FC followed by FC: this layer leaves its partial sums
     // (chain region part_region, 1 or 2) instead of reducing them, and the
-    // next layer adds them while staging its input (x_from_prev)
+    // next layer adds them while staging its input (x_from_prev).  A conv
+    // layer followed by a max-pool leaves them in the scratch region, and
+    // the pool adds them while staging its planes.
     int leave_partials = 0, part_region = 0, x_from_prev = 0;
 };
 
@@ -464,6 +479,19 @@ qcnn_status plan_net(const qcnn_layer *layers, int n_layers, int N, int C, int H
             np->scratch = std::max(np->scratch, np->step0c.scratch);
         }
     }
+    // conv -> max-pool with split partial sums (small batches): the pool adds
+    // them (groups in order, then bias and ReLU: the reduction's arithmetic,
+    // so the output is bit-identical) instead of a reduction launch between
+    // the two.  Not for a first layer run on input slices (host I/O).
+    for (int i = 0; i + 1 < n_layers; ++i) {
+        NetStep &a = np->steps[i], &b = np->steps[i + 1];
+        if (a.kind == QCNN_LAYER_CONV && b.kind == QCNN_LAYER_MAXPOOL &&
+            conv_groups(a.conv) > 1 && (size_t)a.oH * a.oW <= kPoolPlaneMax &&
+            !(i == 0 && np->chunks > 1)) {
+            a.leave_partials = 1;
+            b.x_from_prev = 1;
+        }
+    }
     size_t off = 0;
     for (int b = 0; b < 2; ++b) {
         np->act_off[b] = off;
@@ -547,13 +575,14 @@ qcnn_status plan_net_cached(const qcnn_layer *layers, int n_layers, int N, int C
 }
 
 qcnn_status run_step(const qcnn_layer &L, const NetStep &s, const float *in, float *out,
-                     void *scratch, cudaStream_t st, const FcPartialInput *xin = nullptr) {
+                     void *scratch, cudaStream_t st, const PartialInput *xin = nullptr) {
     if (s.kind == QCNN_LAYER_CONV)
         return run_conv(s.conv, in, L.D, L.codes, L.codes_layout, L.bias, out, L.relu, scratch,
-                        st);
+                        st, s.leave_partials != 0);
     if (s.kind == QCNN_LAYER_FC)
         return launch_fc(s.fc, s.fcp, in, L.D, L.codes, L.bias, out, L.relu,
                          reinterpret_cast<float *>(scratch), st, xin, s.leave_partials != 0);
+    if (xin) return launch_maxpool_partial(*xin, s.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
     return launch_maxpool(in, s.N, s.C, s.H, s.W, L.kh, L.stride, out, st);
 }
 
@@ -567,11 +596,15 @@ qcnn_status run_net(const qcnn_layer *layers, const NetPlan &np, const float *in
         float *out = (i + 1 == n) ? y : reinterpret_cast<float *>(base + np.act_off[i & 1]);
         uint8_t *scratch =
             s.part_region ? base + np.chain_off[s.part_region - 1] : base + np.scratch_off;
-        FcPartialInput xin{};
-        if (s.x_from_prev) {  // (the previous step is an FC layer that left its partials)
+        PartialInput xin{};
+        if (s.x_from_prev) {  // (the previous step left its partial sums)
             const NetStep &p = np.steps[i - 1];
-            xin = {reinterpret_cast<const float *>(base + np.chain_off[p.part_region - 1]),
-                   p.fcp.splits / p.fcp.cl, layers[i - 1].bias, layers[i - 1].relu};
+            if (p.kind == QCNN_LAYER_FC)
+                xin = {reinterpret_cast<const float *>(base + np.chain_off[p.part_region - 1]),
+                       p.fcp.splits / p.fcp.cl, layers[i - 1].bias, layers[i - 1].relu};
+            else  // a conv layer: in the scratch region, where its call put them
+                xin = {reinterpret_cast<const float *>(base + np.scratch_off + p.conv.lut_off),
+                       conv_groups(p.conv), layers[i - 1].bias, layers[i - 1].relu};
         }
         qcnn_status rc = run_step(layers[i], s, in, out, scratch, st, s.x_from_prev ? &xin : nullptr);
         if (rc != QCNN_OK) return rc;

@@ -176,9 +176,12 @@ struct ConvPhasePlan {
     double score;
 };
 ConvPhasePlan plan_conv_phase(const ConvShape &s, int force_cl = 0);
+// leave_partials (fused and phase launches): a plan with several partial sums
+// per output leaves them in partial_ws, without the reduction launch
 qcnn_status launch_conv_phase(const ConvShape &s, const ConvPhasePlan &p, const float *x,
                               const float *D, const uint8_t *packed, const float *bias, float *y,
-                              int relu, float *partial_ws, cudaStream_t st, bool early = false);
+                              int relu, float *partial_ws, cudaStream_t st, bool early = false,
+                              bool leave_partials = false);
 
 size_t packed_codes_bytes(int Ct, int kk, int M);
 int packed_ct(int Ct);   // Ct rounded up to a multiple of 256
@@ -193,7 +196,7 @@ qcnn_status launch_conv_fused(const ConvShape &s, const ConvFusedPlan &p,
                               const float *x, const float *D,
                               const uint8_t *packed, const float *bias, float *y,
                               int relu, float *partial_ws, cudaStream_t st,
-                              bool early = false);
+                              bool early = false, bool leave_partials = false);
 qcnn_status launch_conv_unfused(const ConvShape &s, const ConvUnfusedPlan &p,
                                 const float *x, const float *D,
                                 const uint8_t *packed, const float *bias,
@@ -238,10 +241,11 @@ qcnn_status fc_forward_limited(const float *x, int N, int Cs, int Ct, const floa
                                int K, const uint8_t *codes, const float *bias, float *y,
                                int relu, size_t max_partial_bytes,
                                qcnn_status (*get_scratch)(void **), cudaStream_t st);
-// The input of an FC layer as the previous FC layer's partial sums
-// [groups][N][Cs] (that layer launched with leave_partials), its bias and
-// ReLU applied while staging.
-struct FcPartialInput {
+// The input of a layer as the previous layer's split partial sums (that
+// layer launched with leave_partials): [groups][N][Cs] for an FC layer after
+// an FC layer, [groups][N][C][H][W] for a max-pool after a conv layer; the
+// previous layer's bias and ReLU are applied after adding them.
+struct PartialInput {
     const float *part;
     int groups;
     const float *bias;
@@ -253,7 +257,7 @@ struct FcPartialInput {
 qcnn_status launch_fc(const FcShape &s, const FcPlan &p, const float *x,
                       const float *D, const uint8_t *codes, const float *bias,
                       float *y, int relu, float *partial_ws, cudaStream_t st,
-                      const FcPartialInput *xin = nullptr, bool leave_partials = false);
+                      const PartialInput *xin = nullptr, bool leave_partials = false);
 
 // ------------------------------------------------------------ lut, pool ----
 // lut: fp32 entries, or bfloat16 bit patterns when bf16 != 0
@@ -261,6 +265,11 @@ qcnn_status launch_lut_build(const float *x, int N, int Cs, int P, const float *
                              int Csp, int K, void *lut, int bf16, cudaStream_t st);
 qcnn_status launch_maxpool(const float *x, int N, int C, int H, int W, int k,
                            int s, float *y, cudaStream_t st);
+// The max-pool of a conv output left in partial sums (one CTA per plane,
+// staged in shared memory): planes of at most kPoolPlaneMax elements.
+constexpr size_t kPoolPlaneMax = 12288;
+qcnn_status launch_maxpool_partial(const PartialInput &in, int N, int C, int H, int W, int k,
+                                   int s, float *y, cudaStream_t st);
 
 }  // namespace qcnn
 

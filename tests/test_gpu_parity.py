@@ -309,6 +309,7 @@ def run_workload(name, N):
     ("alexnet_fc678", 1),
     ("alexnet_fc678", 64),
     ("alexnet_qcnn", 1),
+    ("alexnet_qcnn", 8),
 ])
 def test_workload(name, N):
     assert run_workload(name, N) <= TOL
@@ -327,6 +328,62 @@ def test_alexnet_batch128_bench_launch_all_images():
     with packed codes (stream-K cuts tiles between CTAs at batch-dependent
     points), every one of the 128 images against the oracle."""
     assert run_workload("alexnet_qcnn", 128) <= TOL
+
+
+@pytest.mark.parametrize("N,cluster", [(1, True), (1, False), (8, True), (2, False)])
+def test_net_conv_pool_partials_bit_identical_to_layer_calls(N, cluster):
+    """A conv layer whose plan leaves split partial sums hands them to the
+    max-pool after it instead of a reduction launch.  The AlexNet conv stack
+    (conv1 .. pool5) through qcnn_net_forward equals conv_forward and maxpool
+    called layer by layer bit for bit, with one launch fewer per such pair.
+    Without clusters the stride-phase conv1 leaves partial sums too."""
+    w = synth.alexnet()
+    params = w.params()
+    n = 8  # conv1 .. pool5
+    layers, shapes = w.layers[:n], w.shapes()[:n]
+    assert isinstance(layers[-1], synth.Pool) and isinstance(layers[-2], synth.Conv)
+    dev_layers = []
+    for L, P in zip(layers, params):
+        if isinstance(L, synth.Conv):
+            codes = q.conv_pack_codes(cuda(P["codes"]), L.K, L.kh, L.kw)
+            dev_layers.append(q.ConvLayer(cuda(P["D"]), codes, cuda(P["bias"]), L.Ct, L.kh, L.kw,
+                                          L.stride, L.pad, L.relu, packed=True, cluster=cluster))
+        else:
+            dev_layers.append(q.PoolLayer(L.k, L.s))
+    net = q.Net(dev_layers, tuple(w.in_shape))
+    x = cuda(w.input(N, 11))
+    ws = net.alloc_workspace(N)
+    torch.cuda.synchronize()
+
+    before = q.launch_count()
+    h = x
+    for L, d in zip(layers, dev_layers):
+        if isinstance(L, synth.Conv):
+            h = q.conv_forward(h, d.D, d.codes, L.kh, L.kw, L.stride, L.pad, d.bias, L.relu,
+                               packed=True, Ct=L.Ct, cluster=cluster)
+        else:
+            h = q.maxpool(h, L.k, L.s)
+    torch.cuda.synchronize()
+    calls = q.launch_count() - before
+
+    before = q.launch_count()
+    y = net.forward(x, workspace=ws)
+    torch.cuda.synchronize()
+    launches = q.launch_count() - before
+
+    handed = 0
+    for i in range(n - 1):
+        L, (sin, _) = layers[i], shapes[i]
+        if isinstance(L, synth.Conv) and isinstance(layers[i + 1], synth.Pool):
+            p = q.conv_plan(N, L.Cs, sin[1], sin[2], L.Ct, L.kh, L.kw, L.stride, L.pad, L.Csp,
+                            L.K, cluster=cluster)
+            if p["algo"] in ("fused", "phase") and not p["stream_k"] and \
+                    p["splits"] // p["cluster"] > 1:
+                handed += 1
+    if N == 1:
+        assert handed >= (3 if not cluster else 2)
+    assert torch.equal(y, h)
+    assert launches == calls - handed
 
 
 def test_net_forward_host_matches_device():
