@@ -544,6 +544,19 @@ qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers,
                                     int N, int C, int H, int W, int host_io,
                                     size_t *bytes);
 
+/*
+ * qcnn_net_plan_info -- where qcnn_net_forward (host_io = 0) or
+ * qcnn_net_forward_host (host_io = 1) hands split partial sums from one
+ * layer to the next instead of a reduction launch, worked out on the host
+ * (no GPU work; the plan is the one those calls cache).  info has
+ * 2 * n_layers ints: info[2i] = 1 when layer i leaves its partial sums to
+ * layer i + 1, info[2i + 1] = 1 when layer i takes its input as layer
+ * i - 1's partial sums.  Errors are those of qcnn_net_workspace_size, plus
+ * QCNN_ERR_INVALID_ARG for a NULL info.
+ */
+qcnn_status qcnn_net_plan_info(const qcnn_layer *layers, int n_layers, int N, int C, int H,
+                               int W, int host_io, int *info);
+
 /* x [N][C][H][W] device -> y [N][out_C][out_H][out_W] device. */
 qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers,
                              const float *x, int N, int C, int H, int W,

@@ -493,6 +493,19 @@ class Net:
                    "qcnn_net_workspace_size")
         return nb.value
 
+    def plan_info(self, N: int, host_io: bool = False):
+        """Per layer, whether qcnn_net_forward (host_io: qcnn_net_forward_host)
+        at batch N hands its split partial sums to the next layer instead of
+        a reduction launch (qcnn_net_plan_info): a list of dicts with
+        "leaves_partials" and "takes_partials"."""
+        n = len(self._arr)
+        info = (ctypes.c_int * (2 * n))()
+        C, H, W = self.in_shape
+        _lib.check(load().qcnn_net_plan_info(self._arr, n, N, C, H, W, int(host_io), info),
+                   "qcnn_net_plan_info")
+        return [{"leaves_partials": bool(info[2 * i]), "takes_partials": bool(info[2 * i + 1])}
+                for i in range(n)]
+
     def alloc_workspace(self, N: int, device="cuda", host_io: bool = False):
         nb = self.workspace_bytes(N, host_io)
         ws, _ = _workspace(max(nb, 1), torch.device(device), None)

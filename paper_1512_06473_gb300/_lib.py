@@ -70,6 +70,8 @@ _SIGS = {
                                       ctypes.POINTER(c_int)]),
     "qcnn_net_workspace_size": (c_int, [ctypes.POINTER(Layer), c_int, c_int, c_int, c_int, c_int,
                                         c_int, ctypes.POINTER(c_size_t)]),
+    "qcnn_net_plan_info": (c_int, [ctypes.POINTER(Layer), c_int, c_int, c_int, c_int, c_int,
+                                   c_int, ctypes.POINTER(c_int)]),
     "qcnn_net_forward": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int, c_int,
                                  c_int, c_void_p, c_void_p, c_size_t, c_void_p]),
     "qcnn_net_forward_host": (c_int, [ctypes.POINTER(Layer), c_int, c_void_p, c_int, c_int,

@@ -911,6 +911,19 @@ qcnn_status qcnn_net_workspace_size(const qcnn_layer *layers, int n_layers, int 
     return QCNN_OK;
 }
 
+qcnn_status qcnn_net_plan_info(const qcnn_layer *layers, int n_layers, int N, int C, int H,
+                               int W, int host_io, int *info) {
+    if (!info) return QCNN_ERR_INVALID_ARG;
+    NetPlan np;
+    qcnn_status rc = plan_net_cached(layers, n_layers, N, C, H, W, host_io, &np);
+    if (rc != QCNN_OK) return rc;
+    for (int i = 0; i < n_layers; ++i) {
+        info[2 * i] = np.steps[i].leave_partials;
+        info[2 * i + 1] = np.steps[i].x_from_prev;
+    }
+    return QCNN_OK;
+}
+
 qcnn_status qcnn_net_forward(const qcnn_layer *layers, int n_layers, const float *x, int N,
                              int C, int H, int W, float *y, void *workspace,
                              size_t workspace_bytes, void *stream) {

@@ -371,6 +371,46 @@ def test_batch1_plans_split_the_subspaces():
 
 
 @_planner
+def test_net_partial_sum_handoffs():
+    """qcnn_net_plan_info: a conv layer whose plan leaves split partial sums
+    hands them to a max-pool after it, an FC layer to an FC layer after it at
+    batch <= 8; every other layer reduces in its own launch.  In AlexNet at
+    batch 1 that is conv2 -> pool2, conv5 -> pool5 and fc6 -> fc7 -> fc8; at
+    batch 128 (stream-K conv plans, FC above batch 8) nothing."""
+    import paper_1512_06473_gb300 as q
+    w = synth.alexnet()
+    arr = _layers(w)
+    shapes = w.shapes()
+
+    def info(N, host_io=0):
+        out = (ctypes.c_int * (2 * len(arr)))()
+        assert lib.qcnn_net_plan_info(arr, len(arr), N, 3, 227, 227, host_io, out) == _lib.OK
+        return [(out[2 * i], out[2 * i + 1]) for i in range(len(arr))]
+
+    for N, host_io in ((1, 0), (1, 1), (2, 0), (8, 0), (128, 0), (128, 1)):
+        f = info(N, host_io)
+        assert f[0][1] == 0 and f[-1][0] == 0
+        for i, L in enumerate(w.layers[:-1]):
+            assert f[i][0] == f[i + 1][1], (N, i)  # seen from both sides
+            nxt = w.layers[i + 1]
+            if isinstance(L, synth.Conv):
+                sin = shapes[i][0]
+                p = q.conv_plan(N, L.Cs, sin[1], sin[2], L.Ct, L.kh, L.kw, L.stride, L.pad,
+                                L.Csp, L.K)
+                groups = 1 if p["stream_k"] else p["splits"] // p["cluster"]
+                want = isinstance(nxt, synth.Pool) and groups > 1
+            elif isinstance(L, synth.FC):
+                fp = q.fc_plan(N, L.Cs, L.Ct, L.Csp, L.K)
+                want = isinstance(nxt, synth.FC) and N <= 8 and fp["splits"] // fp["cluster"] > 1
+            else:
+                want = False
+            assert bool(f[i][0]) == want, (N, host_io, i)
+    assert [i for i, (leaves, _) in enumerate(info(1)) if leaves] == [2, 6, 8, 9]
+    assert not any(a or b for a, b in info(128))
+    assert lib.qcnn_net_plan_info(arr, len(arr), 1, 3, 227, 227, 0, None) == _lib.ERR_INVALID_ARG
+
+
+@_planner
 def test_fc_16_image_tiles_take_two_chunks():
     """16-image FC tiles give every CTA at least two chunks of 16 sub-spaces
     (one chunk per CTA measured slower at batches 64-128)."""
