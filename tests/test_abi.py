@@ -371,6 +371,43 @@ def test_batch1_plans_split_the_subspaces():
 
 
 @_planner
+@pytest.mark.parametrize("lut", ["fp32", "bf16"])
+def test_plans_are_consistent_on_every_workload(lut):
+    """Every layer of every workload at batches 1-256: a fused conv plan's CTAs
+    are its images x splits x position tiles x channel tiles (under stream-K
+    at most one per (tile, sub-space) unit), clusters divide the splits, tiles
+    are whole warps of positions and 16-channel code pieces; an FC plan's
+    CTAs are its splits x image tiles x output tiles."""
+    import paper_1512_06473_gb300 as q
+    for name, w in synth.WORKLOADS.items():
+        for N in (1, 2, 3, 4, 8, 16, 32, 64, 128, 256):
+            for i, (L, (sin, sout)) in enumerate(zip(w.layers, w.shapes())):
+                where = (name, N, i)
+                if isinstance(L, synth.Conv):
+                    p = q.conv_plan(N, L.Cs, sin[1], sin[2], L.Ct, L.kh, L.kw, L.stride, L.pad,
+                                    L.Csp, L.K, lut=lut)
+                    assert p["splits"] >= 1 and p["splits"] % p["cluster"] == 0, where
+                    assert p["cluster"] in (1, 2, 4, 8, 16), where
+                    if p["algo"] != "fused":
+                        continue
+                    Ho, Wo = sout[1], sout[2]
+                    pitch = max(sin[2] + L.pad, Wo)
+                    pos_tiles = -(-((Ho - 1) * pitch + Wo) // p["positions"])
+                    ct_tiles = -(-L.Ct // p["channels"])
+                    assert p["positions"] % 32 == 0 and p["channels"] % 16 == 0, where
+                    if p["stream_k"]:
+                        assert p["splits"] == 1 and p["cluster"] == 1, where
+                        assert p["ctas"] <= N * pos_tiles * ct_tiles * L.M, where
+                    else:
+                        assert p["ctas"] == N * p["splits"] * pos_tiles * ct_tiles, where
+                elif isinstance(L, synth.FC):
+                    f = q.fc_plan(N, L.Cs, L.Ct, L.Csp, L.K, lut=lut)
+                    assert f["splits"] % f["cluster"] == 0, where
+                    assert f["ctas"] == f["splits"] * -(-N // f["images"]) * \
+                        -(-L.Ct // f["outputs"]), where
+
+
+@_planner
 def test_net_partial_sum_handoffs():
     """qcnn_net_plan_info: a conv layer whose plan leaves split partial sums
     hands them to a max-pool after it, an FC layer to an FC layer after it at
