@@ -41,3 +41,29 @@ def test_batch128_conv2_matches_the_headline_roofline():
     assert st[2]["bound"] == "smem"
     alg = 58.477510656e9  # bytes per launch
     assert math.isclose(st[2]["frac"], alg / 2e-3 / (SMEM * 1e9), rel_tol=1e-4)
+
+
+def test_recorded_traffic_follows_the_kernel_sources(tmp_path, monkeypatch):
+    """The DRAM record counts only while the hashed kernel sources are the
+    ones it was taken with; another workload, batch or layer has none."""
+    import hashlib
+    import json
+    src = tmp_path / "k.cu"
+    src.write_text("kernel v1\n")
+    (tmp_path / "profiles").mkdir()
+    rec = {"workload": "w", "batch": 4, "layer": 2, "dram_read_bytes": 100,
+           "dram_write_bytes": 20, "sources": ["k.cu"],
+           "sha256": hashlib.sha256(b"kernel v1\n").hexdigest()}
+    (tmp_path / "profiles" / "dram_traffic.txt").write_text("# header\n" + json.dumps(rec) + "\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.recorded_traffic("w", 4, 2) == 120
+    assert bench.recorded_traffic("w", 8, 2) is None
+    assert bench.recorded_traffic("w", 4, 3) is None
+    src.write_text("kernel v2\n")
+    assert bench.recorded_traffic("w", 4, 2) is None
+
+
+def test_job_throughput_counts_every_rank():
+    """value = the images all ranks processed / the slowest rank's time."""
+    assert bench.job_throughput(128, 1, 20, 0.1331) == 128 * 20 / 0.1331
+    assert bench.job_throughput(128, 4, 20, 0.2) == 4 * bench.job_throughput(128, 1, 20, 0.2)
