@@ -511,3 +511,29 @@ def test_plan_info_arguments():
     assert lib.qcnn_fc_plan_info(2, 10, 4, 3, 16, 0, info5) == _lib.ERR_INVALID_ARG
     assert lib.qcnn_fc_plan_info(2, 12, 4, 3, 16, 0, info5) == _lib.OK
     assert info5[4] == info5[2] * -(-2 // info5[0]) * -(-4 // info5[1])
+
+
+@_planner
+def test_net_plan_info_binding():
+    """Net.plan_info marshals qcnn_net_plan_info (planning only: host tensors
+    stand in for the device weights)."""
+    import torch
+    import paper_1512_06473_gb300 as q
+    w = synth.alexnet()
+    layers = []
+    for L in w.layers:
+        if isinstance(L, synth.Conv):
+            layers.append(q.ConvLayer(torch.zeros(L.M, L.K, L.Csp),
+                                      torch.zeros(L.Ct, L.kh * L.kw, L.M, dtype=torch.uint8), None,
+                                      L.Ct, L.kh, L.kw, L.stride, L.pad, L.relu))
+        elif isinstance(L, synth.FC):
+            layers.append(q.FCLayer(torch.zeros(L.M, L.K, L.Csp),
+                                    torch.zeros(L.M, L.Ct, dtype=torch.uint8), None, L.relu))
+        else:
+            layers.append(q.PoolLayer(L.k, L.s))
+    net = q.Net(layers, tuple(w.in_shape))
+    b1 = net.plan_info(1)
+    assert [i for i, d in enumerate(b1) if d["leaves_partials"]] == [2, 6, 8, 9]
+    assert [i for i, d in enumerate(b1) if d["takes_partials"]] == [3, 7, 9, 10]
+    assert not any(d["leaves_partials"] or d["takes_partials"]
+                   for d in net.plan_info(128, host_io=True))
