@@ -33,7 +33,7 @@ def _rank(rank, world, port, out):
 
 def test_two_rank_timing_takes_the_slowest_rank():
     world, port = 2, _free_port()
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:  # (no fork of a threaded process)
         out = m.dict()
         mp.spawn(_rank, args=(world, port, out), nprocs=world, join=True)
         res = dict(out)
